@@ -1,0 +1,174 @@
+"""Oracle for the 4-bit weight-streaming GEMV and the decode-chain glue.
+
+TEST INFRASTRUCTURE ONLY: only the tests, ``__graft_entry__.smoke()`` and the
+benchmark's CPU-baseline leg may import this package.  The product library
+(``paper_2412_15803_gb300``) never imports it, and the two share no code.
+
+The arithmetic lives in ``wq4_oracle.c`` (plain C, fp64, single-threaded);
+this module compiles it with gcc and wraps it with ctypes and numpy.  Every
+array is passed as raw bit patterns: fp16 values travel as uint16.
+"""
+from __future__ import annotations
+
+import ctypes
+import os
+import subprocess
+
+import numpy as np
+
+_HERE = os.path.dirname(os.path.abspath(__file__))
+_SRC = os.path.join(_HERE, "wq4_oracle.c")
+_BUILD = os.path.join(_HERE, "_build")
+_LIB_PATH = os.path.join(_BUILD, "liboracle.so")
+
+# -ffp-contract=off keeps "acc += w * x" a rounded multiply then a rounded
+# add on every host (aarch64 gcc would otherwise fuse it into an fma).
+CFLAGS = ["-O2", "-std=c99", "-ffp-contract=off", "-fno-fast-math", "-fPIC", "-shared"]
+
+
+def build(force: bool = False) -> str:
+    """Compile the oracle into oracle/_build/liboracle.so (gcc)."""
+    os.makedirs(_BUILD, exist_ok=True)
+    if (not force and os.path.exists(_LIB_PATH)
+            and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC)):
+        return _LIB_PATH
+    tmp = _LIB_PATH + f".tmp{os.getpid()}"
+    subprocess.check_call(["gcc", *CFLAGS, _SRC, "-o", tmp, "-lm"])
+    os.replace(tmp, _LIB_PATH)
+    return _LIB_PATH
+
+
+_lib = None
+
+
+def lib() -> ctypes.CDLL:
+    global _lib
+    if _lib is None:
+        _lib = ctypes.CDLL(build())
+        P = ctypes.c_void_p
+        I = ctypes.c_int
+        I64 = ctypes.c_int64
+        D = ctypes.c_double
+        _lib.wq4o_half_to_double.argtypes = [ctypes.c_uint16]
+        _lib.wq4o_half_to_double.restype = D
+        _lib.wq4o_double_to_half.argtypes = [D]
+        _lib.wq4o_double_to_half.restype = ctypes.c_uint16
+        _lib.wq4o_half_to_double_array.argtypes = [P, P, I64]
+        _lib.wq4o_double_to_half_array.argtypes = [P, P, I64]
+        _lib.wq4o_ulp16.argtypes = [D]
+        _lib.wq4o_ulp16.restype = D
+        _lib.wq4o_code.argtypes = [P, I, I, I]
+        _lib.wq4o_code.restype = I
+        _lib.wq4o_pack.argtypes = [P, P, I, I]
+        _lib.wq4o_unpack.argtypes = [P, P, I, I, P, P]
+        _lib.wq4o_gemv.argtypes = [P, P, P, I, I, I, P, P, P, P]
+        _lib.wq4o_rms_factor.argtypes = [P, I, D]
+        _lib.wq4o_rms_factor.restype = D
+        _lib.wq4o_silu_mul.argtypes = [P, P, I, P, P]
+        _lib.wq4o_add_fp16.argtypes = [P, P, I, P]
+    return _lib
+
+
+def _p(a):
+    return None if a is None else a.ctypes.data_as(ctypes.c_void_p)
+
+
+def _c(a, dtype):
+    return np.ascontiguousarray(a, dtype=dtype)
+
+
+# ------------------------------------------------------------------- fp16 --
+
+def half_to_double(h) -> np.ndarray:
+    h = _c(h, np.uint16)
+    out = np.empty(h.shape, np.float64)
+    lib().wq4o_half_to_double_array(_p(h), _p(out), h.size)
+    return out
+
+
+def double_to_half(v) -> np.ndarray:
+    v = _c(v, np.float64)
+    out = np.empty(v.shape, np.uint16)
+    lib().wq4o_double_to_half_array(_p(v), _p(out), v.size)
+    return out
+
+
+def ulp16(v: float) -> float:
+    return lib().wq4o_ulp16(float(v))
+
+
+def ulp16_array(v) -> np.ndarray:
+    return np.array([ulp16(t) for t in np.ravel(v)]).reshape(np.shape(v))
+
+
+# ----------------------------------------------------------------- format --
+
+def pack(q) -> np.ndarray:
+    """codes uint8 [N][K] -> packed uint32 [N][K/8]."""
+    q = _c(q, np.uint8)
+    N, K = q.shape
+    W = np.empty((N, K // 8), np.uint32)
+    lib().wq4o_pack(_p(q), _p(W), N, K)
+    return W
+
+
+def unpack(W, s, K: int):
+    """-> (codes uint8 [N][K], w fp64 [N][K] = (q - 7) * s)."""
+    W = _c(W, np.uint32)
+    s = _c(s, np.uint16)
+    N = W.shape[0]
+    q = np.empty((N, K), np.uint8)
+    w = np.empty((N, K), np.float64)
+    lib().wq4o_unpack(_p(W), _p(s), N, K, _p(q), _p(w))
+    return q, w
+
+
+def gemv(W, s, x, r=None):
+    """The GEMV definition.  W uint32 [N][K/8], s fp16 bits [N][K/32],
+    x fp16 bits [batch][K], r optional fp64 [batch] RMS factors.
+
+    Returns (y fp64 [batch][N], A fp64 [batch][N], y16 fp16 bits [batch][N])."""
+    W = _c(W, np.uint32)
+    s = _c(s, np.uint16)
+    x = _c(x, np.uint16)
+    if x.ndim == 1:
+        x = x[None, :]
+    N = W.shape[0]
+    batch, K = x.shape
+    assert W.shape == (N, K // 8) and s.shape == (N, K // 32)
+    rr = None if r is None else _c(r, np.float64).reshape(batch)
+    y = np.empty((batch, N), np.float64)
+    A = np.empty((batch, N), np.float64)
+    y16 = np.empty((batch, N), np.uint16)
+    lib().wq4o_gemv(_p(W), _p(s), _p(x), N, K, batch, _p(rr), _p(y), _p(A), _p(y16))
+    return y, A, y16
+
+
+def tolerance(y_ref, A):
+    """Per-element bound |y_gpu - y_ref| <= 1e-3 * A + ulp16(|y_ref|)."""
+    return 1e-3 * np.asarray(A) + ulp16_array(np.abs(y_ref))
+
+
+# ------------------------------------------------------------------- glue --
+
+def rms_factor(v, eps: float) -> float:
+    v = _c(v, np.uint16)
+    return lib().wq4o_rms_factor(_p(v), v.size, float(eps))
+
+
+def silu_mul(g, u):
+    """-> (m fp64, m16 fp16 bits) with m = silu(g) * u."""
+    g = _c(g, np.uint16)
+    u = _c(u, np.uint16)
+    m = np.empty(g.shape, np.float64)
+    m16 = np.empty(g.shape, np.uint16)
+    lib().wq4o_silu_mul(_p(g), _p(u), g.size, _p(m), _p(m16))
+    return m, m16
+
+
+def add_fp16(a, b) -> np.ndarray:
+    a = _c(a, np.uint16)
+    b = _c(b, np.uint16)
+    z = np.empty(a.shape, np.uint16)
+    lib().wq4o_add_fp16(_p(a), _p(b), a.size, _p(z))
+    return z

@@ -1,0 +1,133 @@
+"""Seeded synthetic inputs shared by the tests, the benchmark and the oracle.
+
+This module holds no arithmetic of the method (no unpacking, no dequantization,
+no dot products): it only draws random bits and turns them into the input
+arrays, so that the oracle and the CUDA path can be fed identical bytes.
+
+Generator: SplitMix64 (Steele, Lea and Flood, "Fast splittable pseudorandom
+number generators", OOPSLA 2014), used counter-style so that any element of
+any stream can be produced independently:
+
+    mix64(z)        = the SplitMix64 output function
+                      (xor-shift 30, multiply, xor-shift 27, multiply,
+                      xor-shift 31, with the published multipliers)
+    key(seed, sid)  = mix64(seed * GAMMA + sid * SID_MUL)          (mod 2^64)
+    u64(key, i)     = mix64(key + (i + 1) * GAMMA)                 (mod 2^64)
+
+Streams (sid) name one tensor each; see ``stream_id``.
+
+Drawn tensors (the distributions of the 1-8B 4-bit decode workloads):
+  * packed codes: uint32 words; word 2m is the low half and word 2m+1 the high
+    half of u64(m), so every 4-bit code is uniform on 0..15;
+  * scales: fp16_RNE(lo + (hi - lo) * u), u = (u64(i) >> 11) * 2^-53,
+    evaluated in fp64 as one multiply then one add, lo = 0.005, hi = 0.02;
+  * activations: fp16_RNE(sqrt(-2 ln u1) * cos(2 pi u2)) (Box-Muller) with
+    u1 = ((u64(2i) >> 11) + 1) * 2^-53 and u2 = (u64(2i+1) >> 11) * 2^-53.
+
+The CUDA library carries a device implementation of the first two draws (for
+weight matrices too large to generate on the host in reasonable time); the
+tests check it against this module bit for bit.  Activations are always drawn
+here and copied.
+"""
+from __future__ import annotations
+
+import numpy as np
+
+GAMMA = 0x9E3779B97F4A7C15
+SID_MUL = 0xD1B54A32D192ED03
+_M1 = 0xBF58476D1CE4E5B9
+_M2 = 0x94D049BB133111EB
+MASK64 = (1 << 64) - 1
+
+SCALE_LO = 0.005
+SCALE_HI = 0.02
+
+# kinds of stream
+KIND_CODES = 0
+KIND_SCALES = 1
+KIND_X = 2
+
+# projection index within a layer
+MAT_QKV, MAT_O, MAT_GATE_UP, MAT_DOWN, MAT_LM_HEAD = 0, 1, 2, 3, 4
+
+
+def stream_id(kind: int, layer: int = 0, mat: int = 0) -> int:
+    """Stream number of one tensor: kind (codes/scales/x), layer, projection."""
+    return (kind & 0xFF) | ((mat & 0xFF) << 8) | ((layer & 0xFFFF) << 16)
+
+
+def _mix64_scalar(z: int) -> int:
+    z &= MASK64
+    z = ((z ^ (z >> 30)) * _M1) & MASK64
+    z = ((z ^ (z >> 27)) * _M2) & MASK64
+    return z ^ (z >> 31)
+
+
+def _mix64(z: np.ndarray) -> np.ndarray:
+    z = z.copy()
+    z ^= z >> np.uint64(30)
+    z *= np.uint64(_M1)
+    z ^= z >> np.uint64(27)
+    z *= np.uint64(_M2)
+    z ^= z >> np.uint64(31)
+    return z
+
+
+def key(seed: int, sid: int) -> int:
+    return _mix64_scalar((seed * GAMMA + sid * SID_MUL) & MASK64)
+
+
+def u64(k: int, start: int, count: int) -> np.ndarray:
+    """u64(k, i) for i in [start, start + count)."""
+    i = np.arange(start, start + count, dtype=np.uint64)
+    with np.errstate(over="ignore"):
+        z = (i + np.uint64(1)) * np.uint64(GAMMA) + np.uint64(k)
+    return _mix64(z)
+
+
+def codes_words(seed: int, sid: int, word_start: int, nwords: int) -> np.ndarray:
+    """Packed-code words [word_start, word_start + nwords) of a stream (uint32).
+
+    word_start and nwords must be even (two words per 64-bit draw)."""
+    if word_start % 2 or nwords % 2:
+        raise ValueError("codes are drawn two words at a time")
+    v = u64(key(seed, sid), word_start // 2, nwords // 2)
+    return v.view(np.uint32).copy()  # little endian: low half first
+
+
+def scales_fp16(seed: int, sid: int, start: int, count: int,
+                lo: float = SCALE_LO, hi: float = SCALE_HI) -> np.ndarray:
+    """Scales [start, start + count) of a stream, as fp16 bit patterns (uint16)."""
+    v = u64(key(seed, sid), start, count)
+    u = (v >> np.uint64(11)).astype(np.float64) * 2.0 ** -53
+    s = np.float64(lo) + np.float64(hi - lo) * u
+    return s.astype(np.float16).view(np.uint16)
+
+
+def normal_fp16(seed: int, sid: int, count: int) -> np.ndarray:
+    """count N(0,1) draws rounded to fp16, as bit patterns (uint16)."""
+    v = u64(key(seed, sid), 0, 2 * count)
+    u1 = ((v[0::2] >> np.uint64(11)).astype(np.float64) + 1.0) * 2.0 ** -53
+    u2 = (v[1::2] >> np.uint64(11)).astype(np.float64) * 2.0 ** -53
+    z = np.sqrt(-2.0 * np.log(u1)) * np.cos(2.0 * np.pi * u2)
+    return z.astype(np.float16).view(np.uint16)
+
+
+def matrix(seed: int, N: int, K: int, layer: int = 0, mat: int = 0,
+           row_start: int = 0, nrows: int | None = None):
+    """Rows [row_start, row_start + nrows) of one N x K packed matrix.
+
+    Returns (W uint32 [nrows][K/8], s uint16 [nrows][K/32]).  Row blocks of
+    the same matrix are consistent with the whole, so a sample of rows of a
+    large matrix can be regenerated on the host."""
+    if nrows is None:
+        nrows = N - row_start
+    wpr, gpr = K // 8, K // 32
+    W = codes_words(seed, stream_id(KIND_CODES, layer, mat), row_start * wpr, nrows * wpr)
+    s = scales_fp16(seed, stream_id(KIND_SCALES, layer, mat), row_start * gpr, nrows * gpr)
+    return W.reshape(nrows, wpr), s.reshape(nrows, gpr)
+
+
+def activations(seed: int, batch: int, K: int, layer: int = 0) -> np.ndarray:
+    """x fp16 bits [batch][K] ~ N(0,1)."""
+    return normal_fp16(seed, stream_id(KIND_X, layer, 0), batch * K).reshape(batch, K)

@@ -1,0 +1,343 @@
+#!/usr/bin/env python3
+"""Benchmark of the GEMV-bound decode chain (one JSON line on rank 0).
+
+Workload (the headline): the 3B-shaped decode chain at batch 1 -- 28 layers of
+fused QKV (5120 x 3072), O (3072 x 3072), gate_up (16384 x 3072) and down
+(3072 x 8192) projections plus the LM head (128256 x 3072), int4 codes in
+groups of 32 with fp16 scales (1.807 GB per token), seeded synthetic weights
+resident in HBM.  One step = one decoded token = one launch of the persistent
+chain kernel through wq4_decode_chain.  The weights (1.8 GB) are far larger
+than L2 (129 MB), so no L2 flush is needed between steps.
+
+    python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
+                    [--workload 3b|8b] [--batch B]
+
+--impl reference times the fp64 CPU oracle on a bounded sample of the same
+workload (the only reference this repository has: the paper's WebGPU/Metal
+engine cannot run here).  Under torchrun (N > 1) every rank decodes its own
+replica (no collective: the workload does not exchange data between GPUs).
+"""
+from __future__ import annotations
+
+import argparse
+import hashlib
+import json
+import os
+import re
+import statistics
+import subprocess
+import sys
+import time
+
+import numpy as np
+
+ROOT = os.path.dirname(os.path.abspath(__file__))
+sys.path.insert(0, ROOT)
+
+METRIC = "GEMV-bound decode tokens/s (batch 1) and achieved HBM GB/s vs ~8 TB/s peak"
+NOMINAL_HBM_GBS = 8000.0
+FALLBACK_HBM_GBS = 6800.0
+
+
+def parse():
+    ap = argparse.ArgumentParser()
+    ap.add_argument("--gpus", type=int, default=1)
+    ap.add_argument("--steps", type=int, default=2000)
+    ap.add_argument("--warmup", type=int, default=20)
+    ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
+    ap.add_argument("--workload", choices=["3b", "8b"], default="3b")
+    ap.add_argument("--batch", type=int, default=1)
+    ap.add_argument("--layers", type=int, default=0, help="override the layer count (profiling runs)")
+    ap.add_argument("--no-cpu-baseline", action="store_true")
+    return ap.parse_args()
+
+
+def dist_env():
+    rank = int(os.environ.get("RANK", "0"))
+    world = int(os.environ.get("WORLD_SIZE", "1"))
+    local = int(os.environ.get("LOCAL_RANK", "0"))
+    return rank, world, local
+
+
+def measured_peak():
+    path = os.path.join(ROOT, "MEASURED_PEAKS.json")
+    try:
+        d = json.load(open(path))
+        return float(d["hbm_gbs"]), "measured (MEASURED_PEAKS.json hbm_gbs, copy read+write)"
+    except Exception:
+        return FALLBACK_HBM_GBS, "fallback"
+
+
+def chain_source_sha() -> str:
+    h = hashlib.sha256()
+    for f in ("wq4_chain.cu", "wq4_device.cuh"):
+        h.update(open(os.path.join(ROOT, "paper_2412_15803_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def profiled_traffic(workload: str, batch: int):
+    """DRAM bytes per launch from the committed ncu summary, if it was taken
+    on the current kernel source (else None)."""
+    path = os.path.join(ROOT, "profiles", f"chain_kernel_{workload}_b{batch}.md")
+    if not os.path.exists(path):
+        return None
+    text = open(path).read()
+    m = re.search(r"traffic_bytes_per_launch:\s*(\d+)", text)
+    s = re.search(r"source_sha:\s*([0-9a-f]+)", text)
+    if not m or not s or s.group(1) != chain_source_sha():
+        return None
+    return int(m.group(1))
+
+
+class ClockSampler:
+    FIELDS = ("clocks.sm,clocks.max.sm,power.draw,clocks_event_reasons.active,"
+              "clocks_event_reasons.hw_slowdown,clocks_event_reasons.hw_thermal_slowdown,"
+              "clocks_event_reasons.sw_thermal_slowdown,clocks_event_reasons.sw_power_cap")
+
+    def __init__(self, device_index: int):
+        self.proc = None
+        self.out = None
+        try:
+            import torch
+            uuid = str(torch.cuda.get_device_properties(device_index).uuid)
+            sel = ["-i", uuid if uuid.startswith("GPU-") else "GPU-" + uuid]
+        except Exception:
+            sel = []
+        self.cmd = ["nvidia-smi", *sel, f"--query-gpu={self.FIELDS}", "--format=csv,noheader,nounits", "-lms", "100"]
+
+    def start(self):
+        try:
+            self.proc = subprocess.Popen(self.cmd, stdout=subprocess.PIPE, stderr=subprocess.DEVNULL, text=True)
+        except Exception:
+            self.proc = None
+
+    def stop(self):
+        if not self.proc:
+            return {"sm_mhz": None, "sm_max_mhz": None, "reasons": ["nvidia-smi unavailable"]}
+        self.proc.terminate()
+        try:
+            out, _ = self.proc.communicate(timeout=5)
+        except Exception:
+            self.proc.kill()
+            out, _ = self.proc.communicate()
+        sm, mx, reasons, power = [], [], set(), []
+        names = ["hw_slowdown", "hw_thermal_slowdown", "sw_thermal_slowdown", "sw_power_cap"]
+        for line in out.strip().splitlines():
+            f = [t.strip() for t in line.split(",")]
+            if len(f) < 8:
+                continue
+            try:
+                sm.append(float(f[0]))
+                mx.append(float(f[1]))
+                power.append(float(f[2]))
+            except ValueError:
+                continue
+            for n, v in zip(names, f[4:8]):
+                if v.lower().startswith("active"):
+                    reasons.add(n)
+        return {"sm_mhz": statistics.median(sm) if sm else None, "sm_max_mhz": max(mx) if mx else None,
+                "reasons": sorted(reasons), "samples": len(sm),
+                "power_w_median": statistics.median(power) if power else None}
+
+
+# ---------------------------------------------------------------- oracle --
+
+def oracle_sample(shape, batch: int, fraction: float, seed: int = 0):
+    """Times the fp64 oracle on the first ceil(fraction * N) rows of every
+    projection of the chain (all layers and the LM head).  Returns
+    (seconds, weights processed)."""
+    import oracle
+    from paper_2412_15803_gb300 import synth
+    x = {K: synth.activations(seed, batch, K) for K in {shape.hidden, shape.ffn}}
+    blocks = []
+    for l in range(shape.num_layers):
+        for name, N, K, mat in shape.mats(l):
+            blocks.append((N, K, l, mat))
+    blocks.append((shape.vocab, shape.hidden, shape.num_layers, synth.MAT_LM_HEAD))
+    total_t, total_w = 0.0, 0
+    for N, K, l, mat in blocks:
+        n = max(1, int(np.ceil(fraction * N)))
+        W, s = synth.matrix(seed, N, K, l, mat, 0, n)
+        t0 = time.perf_counter()
+        oracle.gemv(W, s, x[K])
+        total_t += time.perf_counter() - t0
+        total_w += n * K
+    return total_t, total_w
+
+
+def oracle_rate_estimate(shape, batch):
+    """Seconds per weight of the oracle on this host (short calibration)."""
+    import oracle
+    from paper_2412_15803_gb300 import synth
+    W, s = synth.matrix(1, 256, shape.hidden)
+    x = synth.activations(1, batch, shape.hidden)
+    t0 = time.perf_counter()
+    oracle.gemv(W, s, x)
+    return (time.perf_counter() - t0) / (256 * shape.hidden)
+
+
+def cpu_baseline(shape, batch, target_s=12.0):
+    per_w = oracle_rate_estimate(shape, batch)
+    frac = min(1.0, target_s / max(per_w * shape.weight_count(), 1e-9))
+    t, w = oracle_sample(shape, batch, frac)
+    tokens = batch * w / shape.weight_count()
+    return {"value": tokens / t, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+            "sample": f"first {frac:.4f} of the rows of all {4 * shape.num_layers + 1} projections "
+                      f"({w} weights = {w / shape.weight_count():.4f} of a token), batch {batch}, "
+                      f"single-threaded fp64 C oracle, {t:.1f} s"}
+
+
+def run_reference(args, rank, world):
+    from paper_2412_15803_gb300.model import SHAPES
+    if rank != 0:
+        return
+    shape = SHAPES[args.workload]
+    per_w = oracle_rate_estimate(shape, args.batch)
+    nsteps = args.steps + args.warmup
+    step_s = min(10.0, 120.0 / max(nsteps, 1))
+    frac = min(1.0, step_s / (per_w * shape.weight_count()))
+    times, wsum = [], 0
+    for i in range(nsteps):
+        t, w = oracle_sample(shape, args.batch, frac)
+        if i >= args.warmup:
+            times.append(t)
+            wsum += w
+    tok = args.batch * wsum / shape.weight_count()
+    value = tok / sum(times)
+    line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": 1e3 * sum(times) / len(times), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+            "config": {"workload": f"{shape.name}-shaped decode chain, {shape.num_layers} layers + LM head, "
+                                   f"batch {args.batch}", "sample_fraction_per_step": frac},
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+                             "sample": f"each step: first {frac:.5f} of the rows of every projection"},
+            "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+# ------------------------------------------------------------------- ours --
+
+def run_ours(args, rank, world, local):
+    import torch
+    import torch.distributed as dist
+    from paper_2412_15803_gb300 import synth, wq4
+    from paper_2412_15803_gb300.model import SHAPES, DecodeModel
+
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    shape = SHAPES[args.workload]
+    if args.layers:
+        import dataclasses
+        shape = dataclasses.replace(shape, name=f"{shape.name}-{args.layers}l", num_layers=args.layers)
+    B = args.batch
+    model = DecodeModel(shape, batch=B, seed=0)
+    x_np = synth.activations(1000 + rank, B, shape.hidden)
+    x = torch.from_numpy(x_np.view(np.int16)).cuda()
+    logits = torch.empty((B, shape.vocab), dtype=torch.int16, device="cuda")
+    stream = torch.cuda.current_stream()
+
+    # bytes one token streams: packed codes + scales of every projection,
+    # plus the activation vectors read and written (negligible)
+    weight_bytes = shape.weight_bytes()
+    vec_bytes = 2 * B * (shape.hidden * (4 * shape.num_layers + 1) + shape.vocab)
+    step_bytes = weight_bytes + vec_bytes
+
+    for _ in range(args.warmup):
+        model.decode(x, logits, stream)
+    torch.cuda.synchronize()
+    if wq4.wq4_device_status(stream) != 0:
+        raise RuntimeError("device wait timed out during warm-up")
+
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.3)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    for i in range(args.steps):
+        starts[i].record(stream)
+        model.decode(x, logits, stream)
+        ends[i].record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clocks = sampler.stop()
+    total_ms = starts[0].elapsed_time(ends[-1])
+    launch_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    if wq4.wq4_device_status(stream) != 0:
+        raise RuntimeError("device wait timed out during the timed region")
+
+    t = torch.tensor([total_ms], dtype=torch.float64, device="cuda")
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    total_ms_max = float(t.item())
+
+    # end to end through the host-buffer entry point: x H2D, chain, logits D2H
+    x_host = torch.from_numpy(x_np.view(np.int16)).pin_memory()
+    l_host = torch.empty((B, shape.vocab), dtype=torch.int16).pin_memory()
+    e2e_steps = max(10, min(args.steps, 500))
+    for _ in range(3):
+        model.decode_host(x_host.numpy(), l_host.numpy(), stream)
+    t0 = time.perf_counter()
+    for _ in range(e2e_steps):
+        model.decode_host(x_host.numpy(), l_host.numpy(), stream)
+    e2e_s = time.perf_counter() - t0
+    e2e_val = B * e2e_steps / e2e_s
+    if world > 1:
+        te = torch.tensor([e2e_s / e2e_steps], dtype=torch.float64, device="cuda")
+        dist.all_reduce(te, op=dist.ReduceOp.MAX)
+        e2e_val = world * B / float(te.item())
+
+    if rank == 0:
+        ms = total_ms_max / args.steps
+        tokens_per_s = world * B * args.steps / (total_ms_max / 1e3)
+        avg_launch_ms = statistics.mean(launch_ms)
+        peak, peak_src = measured_peak()
+        achieved = step_bytes / (avg_launch_ms * 1e-3) / 1e9
+        line = {
+            "metric": METRIC, "value": tokens_per_s, "unit": "tokens/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "precision": "int4 codes (group 32, fp16 scale, zero point 7), fp16 activations, fp32 accumulation",
+            "data": "synthetic (seeded SplitMix64 weights and activations)",
+            "config": {"workload": f"{shape.name}-shaped decode chain: {shape.num_layers} layers x "
+                                   f"(QKV {shape.n_qkv}x{shape.hidden}, O {shape.hidden}x{shape.hidden}, "
+                                   f"gate_up {2 * shape.ffn}x{shape.hidden}, down {shape.hidden}x{shape.ffn}) "
+                                   f"+ LM head {shape.vocab}x{shape.hidden}, batch {B}",
+                       "batch": B, "bytes_per_token": step_bytes,
+                       "l2": "inputs larger than L2 (1.8+ GB of weights per step), no flush",
+                       "parallelism": "replicas" if world > 1 else "single GPU"},
+            "hbm_gbs": step_bytes * args.steps / (total_ms_max / 1e3) / 1e9,
+            "hbm_frac_of_nominal_8tbs": step_bytes * args.steps / (total_ms_max / 1e3) / 1e9 / NOMINAL_HBM_GBS,
+            "roofline": {"bound": "hbm", "kernel": "chain_kernel", "achieved": achieved, "peak": peak,
+                         "peak_source": peak_src, "unit": "GB/s", "frac": achieved / peak,
+                         "frac_of_nominal_8tbs": achieved / NOMINAL_HBM_GBS,
+                         "traffic": profiled_traffic(args.workload, B),
+                         "algorithmic_bytes_per_launch": step_bytes,
+                         "avg_launch_ms": avg_launch_ms},
+            "e2e": {"value": e2e_val, "unit": "tokens/s", "h2d_bytes_per_step": 2 * B * shape.hidden,
+                    "d2h_bytes_per_step": 2 * B * shape.vocab},
+            "gpu_launches": args.steps,
+            "clocks": clocks,
+        }
+        if world == 1 and not args.no_cpu_baseline:
+            line["cpu_baseline"] = cpu_baseline(shape, B)
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
+def main():
+    args = parse()
+    rank, world, local = dist_env()
+    if args.impl == "reference":
+        run_reference(args, rank, world)
+    else:
+        run_ours(args, rank, world, local)
+
+
+if __name__ == "__main__":
+    main()

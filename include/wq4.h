@@ -1,0 +1,216 @@
+/*
+ * wq4.h -- C ABI of the GB300 (sm_103a) 4-bit weight-streaming GEMV library.
+ *
+ * The paper's decode workload is token generation with 4-bit quantized
+ * models (Section 3, Table 1; Section 1 quotes about 90 tokens/s for a 4-bit
+ * 3B model on a laptop GPU).  Each decoded token streams every weight matrix
+ * once: the fused QKV, attention-output, gate_up and down projections of each
+ * layer and the LM head.  The paper's compiler produces these kernels with
+ * "kernel fusion" and "GEMM tiling" (Section 2.3) and ships the weights as an
+ * offline-converted artifact (Section 2.3); this library is the GB300 form of
+ * that hot path, written by hand.
+ *
+ * Weight format (the paper says only "4-bit quantized"; this library fixes it):
+ *   W_packed  uint32 [N][K/8]  code k of row n is bits [4*(k%8), 4*(k%8)+4) of
+ *                              word W[n][k/8] (lowest nibble first), 0..15;
+ *   scales    fp16   [N][K/32] one scale per group of 32 consecutive codes;
+ *   weight    w(n,k) = (q(n,k) - 7) * scales[n][k/32].
+ * Activations x are fp16 [batch][K], outputs y are fp16 [batch][N]; products
+ * are accumulated in fp32 and y is rounded to nearest even.
+ * Accuracy contract: |y - y_ref| <= 1e-3 * sum_k |w*x| + ulp16(|y_ref|),
+ * y_ref being the exact (fp64) sum.
+ *
+ * Conventions for every call below:
+ *   - Pointers named W, scales, x, y, w_out, q_out, logits are DEVICE pointers
+ *     (unless the name says host) owned by the caller; the library never frees
+ *     them and never keeps them beyond the call, except the chain plan, which
+ *     remembers the layer table's pointers until wq4_chain_plan_destroy.
+ *   - `stream` is a cudaStream_t passed as void* (NULL = legacy default
+ *     stream).  Device calls are asynchronous: they validate, enqueue and
+ *     return; they never synchronize (except where stated) and never allocate
+ *     device memory.
+ *   - Argument errors return before anything is enqueued.  A CUDA launch
+ *     failure returns WQ4_ERR_CUDA.
+ *   - Device-side waits are bounded; a wait that gives up records a flag that
+ *     wq4_device_status() reports, and the kernel still terminates.
+ */
+#ifndef WQ4_H
+#define WQ4_H
+
+#include <stddef.h>
+#include <stdint.h>
+
+#ifdef __cplusplus
+extern "C" {
+#endif
+
+enum wq4_status {
+    WQ4_OK = 0,
+    WQ4_ERR_INVALID = -1,     /* bad size, null pointer, aliasing, bad table */
+    WQ4_ERR_ALIGN = -2,       /* a pointer is below the alignment the call needs */
+    WQ4_ERR_UNSUPPORTED = -3, /* valid arguments outside what this build handles */
+    WQ4_ERR_CUDA = -4,        /* a CUDA runtime call failed */
+    WQ4_ERR_TIMEOUT = -5      /* a device-side wait gave up (see wq4_device_status) */
+};
+
+/* Largest batch (rows of x) any call accepts. */
+#define WQ4_MAX_BATCH 32
+
+/*
+ * y[b][n] = fp16( sum_k (q(n,k) - 7) * scales[n][k/32] * x[b][k] )
+ * for b < batch, n < N: the fused dequantize-and-multiply projection of one
+ * decode step (Section 3, Table 1 workload; Section 2.3 "kernel fusion":
+ * dequantization happens in registers, the fp32 weights never exist in
+ * memory).
+ *   W_packed : uint32 [N][K/8], 16-byte aligned.
+ *   scales   : fp16 bits [N][K/32], 2-byte aligned (16-byte aligned and
+ *              K % 256 == 0 select the TMA-staged fast path).
+ *   x        : fp16 bits [batch][K], 16-byte aligned.
+ *   y        : fp16 bits [batch][N], 2-byte aligned; must not overlap x, W or
+ *              scales.
+ *   N >= 1, K >= 32 with K % 32 == 0, 1 <= batch <= WQ4_MAX_BATCH.
+ * Returns WQ4_OK, WQ4_ERR_INVALID (sizes, null, overlap), WQ4_ERR_ALIGN, or
+ * WQ4_ERR_CUDA.  Deterministic: the same inputs give the same bits.
+ */
+int wq4_gemv(const uint32_t* W_packed, const uint16_t* scales, const uint16_t* x,
+             uint16_t* y, int N, int K, int batch, void* stream);
+
+/*
+ * Test hook for the unpack step: runs the same in-register unpack the GEMV
+ * uses and writes its results, so that they can be compared bit for bit.
+ *   q_out : uint8 [N][K] codes 0..15 (may be NULL)
+ *   w_out : fp32  [N][K] = (q - 7) * scale, exact in fp32 (may be NULL)
+ * Same size and alignment rules as wq4_gemv (batch not used).
+ */
+int wq4_unpack_debug(const uint32_t* W_packed, const uint16_t* scales,
+                     float* w_out, uint8_t* q_out, int N, int K, void* stream);
+
+/*
+ * Host-side packer of the weight format (the offline weight conversion of
+ * Section 2.3): q_host uint8 [N][K] with values 0..15 -> W_host uint32
+ * [N][K/8].  HOST pointers.  Returns WQ4_ERR_INVALID for a code above 15,
+ * null pointers or bad sizes (K % 8 != 0).
+ */
+int wq4_pack_host(const uint8_t* q_host, uint32_t* W_host, int N, int K);
+
+/* Static, human-readable text of a status code. */
+const char* wq4_status_string(int status);
+
+/*
+ * Reads and clears the library's device status word on `stream` (this call
+ * synchronizes the stream).  *flags_out receives the bits that were set:
+ * bit 0 = an mbarrier wait of a weight pipeline gave up, bit 1 = a wait on
+ * another CTA's activations gave up.  Returns WQ4_ERR_TIMEOUT if any bit
+ * was set, WQ4_OK otherwise, WQ4_ERR_CUDA on a CUDA failure.
+ */
+int wq4_device_status(void* stream, int* flags_out);
+
+/* ------------------------------------------------------------------------ */
+/* Per-token decode chain                                                     */
+/* ------------------------------------------------------------------------ */
+
+/* One packed projection: W uint32 [N][K/8], s fp16 [N][K/32] (device). */
+typedef struct {
+    const uint32_t* W;
+    const uint16_t* s;
+} wq4_mat;
+
+/* One layer's four projections (shapes follow from the table below):
+ *   qkv     : N = (n_q_heads + 2*n_kv_heads) * head_dim, K = hidden
+ *   o       : N = hidden,  K = hidden
+ *   gate_up : N = 2*ffn,   K = hidden (rows [0,ffn) gate, [ffn,2ffn) up)
+ *   down    : N = hidden,  K = ffn                                          */
+typedef struct {
+    wq4_mat qkv, o, gate_up, down;
+} wq4_layer;
+
+/*
+ * A decoder's weights and the caller-owned workspace of the chain.
+ *   layers     : HOST array of num_layers entries holding device pointers.
+ *   lm_head    : N = vocab, K = hidden.
+ *   n_q_heads * head_dim must equal hidden (the query block of the QKV output
+ *   is the stand-in attention output, see wq4_decode_chain).
+ *   workspace  : device buffer of at least wq4_chain_workspace_bytes(table)
+ *                bytes, 256-byte aligned, used only by this table's chain.
+ *   All dimensions must be multiples of 256 except vocab (any >= 1); batch
+ *   1..4 (WQ4_ERR_UNSUPPORTED above).
+ */
+typedef struct {
+    int num_layers, hidden, ffn, n_q_heads, n_kv_heads, head_dim, vocab, batch;
+    float rms_eps;
+    const wq4_layer* layers;
+    wq4_mat lm_head;
+    void* workspace;
+    size_t workspace_bytes;
+} wq4_layer_table;
+
+/* Bytes of workspace the chain needs for this table (0 if the table is
+ * invalid).  Host-only, no CUDA call. */
+size_t wq4_chain_workspace_bytes(const wq4_layer_table* table);
+
+/*
+ * One decoded token through every projection of every layer and the LM head
+ * (the per-token GPU work measured by Table 1, Section 3), as ONE persistent
+ * kernel whose CTAs stream the weights through shared memory and pass the
+ * activations between stages through flagged words in the workspace.
+ * Layer l takes u (fp16 [batch][hidden]: x for l = 0, else the previous
+ * layer's output), re-feeds it after RMS normalisation, and rounds every
+ * stage output to fp16:
+ *   v   = r(u) * u                     r(t) = 1/sqrt(mean(t^2) + rms_eps)
+ *   qkv = W_qkv . v
+ *   o   = r(a)  * W_o   . a            a = qkv[:, :hidden] (stands in for
+ *   x1  = v + o                            attention, which is not in the chain)
+ *   gu  = r(x1) * W_gu  . x1
+ *   m   = silu(gu[:, :ffn]) * gu[:, ffn:]
+ *   x2  = x1 + W_down . m              (the layer output, next layer's u)
+ * then logits = W_lm . (r(xL) * xL).  RMS normalisation has no learned gain;
+ * before O and gate_up it enters as a per-row factor of the projection
+ * (Section 2.3 "kernel fusion").
+ *   x      : fp16 [batch][hidden] device, 16-byte aligned
+ *   logits : fp16 [batch][vocab]  device, 2-byte aligned
+ * The first call for a table (or after its contents changed) validates it and
+ * uploads its pointer table into the workspace (cudaMemcpyAsync on `stream`);
+ * later calls only launch.  Calls on one table must not overlap on the GPU.
+ * Returns WQ4_OK, WQ4_ERR_INVALID, WQ4_ERR_ALIGN, WQ4_ERR_UNSUPPORTED or
+ * WQ4_ERR_CUDA (including a GPU that cannot co-schedule the persistent grid).
+ */
+int wq4_decode_chain(const wq4_layer_table* table, const uint16_t* x,
+                     uint16_t* logits, void* stream);
+
+/*
+ * The same token with HOST buffers: copies x_host (pinned or pageable fp16
+ * [batch][hidden]) into the workspace, runs wq4_decode_chain, copies the
+ * logits back into logits_host (fp16 [batch][vocab]) and synchronizes
+ * `stream` before returning.
+ */
+int wq4_decode_chain_host(const wq4_layer_table* table, const uint16_t* x_host,
+                          uint16_t* logits_host, void* stream);
+
+/* Releases the cached plan of `table` (host-side state only; the workspace
+ * stays the caller's).  Returns WQ4_ERR_INVALID if no plan exists. */
+int wq4_chain_plan_destroy(const wq4_layer_table* table);
+
+/*
+ * Byte offsets into the workspace of the plain fp16 copies of one layer's
+ * stage outputs, each [batch][len] row-major, for inspection after a call
+ * (layer in [0, num_layers)); layer == num_layers gives the LM head's input
+ * in x_in and 0 in the other fields.
+ */
+typedef struct {
+    size_t x_in;     /* [batch][hidden]  v: layer input after RMS norm */
+    size_t qkv;      /* [batch][n_qkv]   QKV projection              */
+    size_t o;        /* [batch][hidden]  O projection                */
+    size_t x_mid;    /* [batch][hidden]  x + o                        */
+    size_t gate_up;  /* [batch][2*ffn]   gate_up projection           */
+    size_t act;      /* [batch][ffn]     silu(gate) * up              */
+    size_t down;     /* [batch][hidden]  down projection              */
+    size_t x_out;    /* [batch][hidden]  x2: layer output (not normalised) */
+} wq4_chain_trace;
+
+int wq4_chain_trace_offsets(const wq4_layer_table* table, int layer, wq4_chain_trace* out);
+
+#ifdef __cplusplus
+}
+#endif
+
+#endif /* WQ4_H */

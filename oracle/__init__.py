@@ -64,6 +64,7 @@ def lib() -> ctypes.CDLL:
         _lib.wq4o_gemv.argtypes = [P, P, P, I, I, I, P, P, P, P]
         _lib.wq4o_rms_factor.argtypes = [P, I, D]
         _lib.wq4o_rms_factor.restype = D
+        _lib.wq4o_rms_normalize.argtypes = [P, I, D, P]
         _lib.wq4o_silu_mul.argtypes = [P, P, I, P, P]
         _lib.wq4o_add_fp16.argtypes = [P, P, I, P]
     return _lib
@@ -154,6 +155,18 @@ def tolerance(y_ref, A):
 def rms_factor(v, eps: float) -> float:
     v = _c(v, np.uint16)
     return lib().wq4o_rms_factor(_p(v), v.size, float(eps))
+
+
+def rms_normalize(u, eps: float) -> np.ndarray:
+    """fp16 bits of fp16_RNE(r(u) * u), r(u) = 1 / sqrt(mean(u^2) + eps), per row."""
+    u = np.atleast_2d(_c(u, np.uint16))
+    v = np.empty(u.shape, np.uint16)
+    for b in range(u.shape[0]):
+        row = np.ascontiguousarray(u[b])
+        out = np.empty(row.shape, np.uint16)
+        lib().wq4o_rms_normalize(_p(row), row.size, float(eps), _p(out))
+        v[b] = out
+    return v
 
 
 def silu_mul(g, u):

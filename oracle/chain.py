@@ -6,24 +6,28 @@ The paper's workload is token decoding of 4-bit quantized transformer models
 (Section 3, Table 1); the weight stream of every projection of every layer is
 read once per token.  Attention itself (PagedAttention / FlashAttention,
 Section 2.3) is not part of this chain: the query block of the fused QKV
-output stands in for the attention output, as stated below.
+output stands in for the attention output.
 
-One layer, input x (fp16 [batch][H]); every stage output is rounded to fp16:
+Layer l takes u (fp16 [batch][H]: the token input for l = 0, else the previous
+layer's output) and re-feeds it after RMS normalisation; every stage output
+is rounded to fp16:
 
-    qkv = fp16( r(x)   * W_qkv  . x  )          [batch][Nqkv]
+    v   = fp16( r(u) * u )                       layer input, RMS-normalised
+    qkv = fp16(          W_qkv  . v  )          [batch][Nqkv]
     a   = qkv[:, :H]                             (stands in for attention)
     o   = fp16( r(a)   * W_o    . a  )          [batch][H]
-    x1  = fp16( x + o )
+    x1  = fp16( v + o )
     gu  = fp16( r(x1)  * W_gu   . x1 )          [batch][2F]  (gate | up)
     m   = fp16( silu(gu[:, :F]) * gu[:, F:] )   [batch][F]
     d   = fp16(          W_down . m  )          [batch][H]
-    x2  = fp16( x1 + d )                         (layer output)
+    x2  = fp16( x1 + d )                         layer output
 
-and after the last layer: logits = fp16( r(xL) * W_lm . xL ).
+and after the last layer: logits = fp16( W_lm . fp16(r(xL) * xL) ).
 
-r(v) = 1 / sqrt(mean(v^2) + eps) is RMS normalisation without a learned gain,
-applied as a per-row factor of the projection (r(v) W.v = W.(r(v) v) exactly
-in real arithmetic), so the projection input stays the fp16 vector v.
+r(v) = 1 / sqrt(mean(v^2) + eps) is RMS normalisation without a learned gain.
+Where it precedes a projection of an unnormalised vector (O, gate_up) it is
+applied as a per-row factor of the projection (r(v) W.v = W.(r(v) v) in real
+arithmetic), so that projection's input stays the fp16 vector.
 
 Each step calls the primitives of ``oracle`` and nothing else.
 """
@@ -31,7 +35,7 @@ from __future__ import annotations
 
 import numpy as np
 
-from . import add_fp16, gemv, rms_factor, silu_mul
+from . import add_fp16, gemv, rms_factor, rms_normalize, silu_mul
 
 
 def rms_factors(v, eps):
@@ -39,20 +43,21 @@ def rms_factors(v, eps):
     return np.array([rms_factor(row, eps) for row in v])
 
 
-def layer(x, w, H: int, F: int, eps: float):
+def layer(u, w, H: int, F: int, eps: float):
     """One layer.  w = dict(qkv=(W, s), o=..., gate_up=..., down=...).
 
     Returns (x2, trace) where trace holds every stage's fp16 output and the
     fp64 values with their magnitudes A for the projections."""
-    t = {"x": x}
-    r1 = rms_factors(x, eps)
-    y, A, qkv = gemv(*w["qkv"], x, r1)
-    t.update(r_x=r1, qkv=qkv, qkv_ref=y, qkv_A=A)
+    t = {"u": u}
+    v = rms_normalize(u, eps)
+    t["v"] = v
+    y, A, qkv = gemv(*w["qkv"], v)
+    t.update(qkv=qkv, qkv_ref=y, qkv_A=A)
     a = np.ascontiguousarray(qkv[:, :H])
     r2 = rms_factors(a, eps)
     y, A, o = gemv(*w["o"], a, r2)
     t.update(r_a=r2, o=o, o_ref=y, o_A=A)
-    x1 = add_fp16(x, o)
+    x1 = add_fp16(v, o)
     t["x1"] = x1
     r3 = rms_factors(x1, eps)
     y, A, gu = gemv(*w["gate_up"], x1, r3)
@@ -67,13 +72,14 @@ def layer(x, w, H: int, F: int, eps: float):
 
 
 def token(x, layers, lm_head, H: int, F: int, eps: float):
-    """Whole token: all layers, final RMS factor and LM head.
+    """Whole token: all layers, final RMS normalisation and LM head.
 
     Returns (logits fp16 bits, logits fp64, traces)."""
     traces = []
     for w in layers:
         x, t = layer(x, w, H, F, eps)
         traces.append(t)
-    rf = rms_factors(x, eps)
-    y, A, logits = gemv(*lm_head, x, rf)
+    v = rms_normalize(x, eps)
+    y, A, logits = gemv(*lm_head, v)
+    traces.append({"u": x, "v": v, "logits_ref": y, "logits_A": A})
     return logits, y, traces

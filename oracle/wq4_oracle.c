@@ -190,6 +190,15 @@ WQ4O_EXPORT double wq4o_rms_factor(const uint16_t* v, int n, double eps)
     return 1.0 / sqrt(ss / (double)n + eps);
 }
 
+/* v[i] = fp16_RNE(r * u[i]) with r = 1 / sqrt(mean(u^2) + eps): the RMS
+ * normalisation (no learned gain) that turns a layer's output into the next
+ * layer's input. */
+WQ4O_EXPORT void wq4o_rms_normalize(const uint16_t* u, int n, double eps, uint16_t* v)
+{
+    double r = wq4o_rms_factor(u, n, eps);
+    for (int i = 0; i < n; ++i) v[i] = wq4o_double_to_half(r * wq4o_half_to_double(u[i]));
+}
+
 /* m[i] = silu(g[i]) * u[i] with silu(t) = t / (1 + exp(-t)); fp64 result
  * and its fp16 rounding (either output may be NULL). */
 WQ4O_EXPORT void wq4o_silu_mul(const uint16_t* g, const uint16_t* u, int n,

@@ -1,0 +1,878 @@
+// wq4_chain.cu -- one decoded token through every projection of every layer
+// and the LM head, as one persistent kernel (the per-token GPU work whose
+// throughput Table 1 of Section 3 reports).
+//
+// Structure (GB300-first; the paper's WebGPU engine launches one compiled
+// kernel per operator, Section 2.3):
+//  * One CTA per SM, co-resident (cooperative launch).  Each CTA owns a fixed
+//    slice of the output rows of every stage (QKV, O, gate_up, down per layer,
+//    then the LM head).
+//  * A producer warp walks the CTA's slices of ALL stages in order and streams
+//    their packed weights through a ring of shared-memory slots with 1-D bulk
+//    copies (TMA) and mbarriers.  Weights do not depend on activations, so the
+//    stream runs ahead across stage boundaries and HBM keeps working while the
+//    consumers wait for the next activation vector.
+//  * Each layer re-feeds its input after RMS normalisation: the QKV stage (and
+//    the LM head) normalise the staged vector in shared memory; every CTA
+//    computes the same factor in the same order, so all CTAs hold identical
+//    bits, and the first CTA publishes them for the O stage's residual add.
+//  * Consumer warps stage each stage's input vector in shared memory, take
+//    two-row items (four rows for gate_up: gate j, j+1 and up j, j+1)
+//    round-robin, unpack in registers, accumulate in fp32, and apply the
+//    fused epilogue (RMS factor, residual add, SiLU(gate) * up).
+//  * Stage outputs travel between CTAs as 8-byte words {2 x fp16 data, 32-bit
+//    token epoch} written with single 64-bit stores; a consumer polls the
+//    words of its input until every epoch matches.  No grid-wide barrier and
+//    no separate flag round trip: one L2 round trip per stage boundary.
+//    Every poll is bounded in time.
+//  * Plain fp16 copies of every stage output are written to the workspace for
+//    inspection.
+#include "wq4_device.cuh"
+#include "wq4_host.h"
+#include "wq4.h"
+
+#include <cuda_runtime.h>
+
+#include <cmath>
+#include <cstring>
+#include <map>
+#include <mutex>
+#include <vector>
+
+namespace wq4 {
+namespace {
+
+constexpr int kNW = 8;                       // consumer warps
+constexpr int kChainThreads = (kNW + 1) * 32;
+constexpr int kChainMaxSlots = 32;
+constexpr int kChainHeader = 1024;           // mbarriers, reductions, scalars
+constexpr int kMaxChainBatch = 4;
+
+enum StageType { kQKV = 0, kO = 1, kGU = 2, kDOWN = 3, kLM = 4 };
+
+struct DevMat {
+    const uint32_t* W;
+    const uint16_t* s;
+};
+
+struct ChainParams {
+    const DevMat* mats;  // [4L + 1]: per layer qkv, o, gate_up, down; then lm_head
+    int L, H, F, Nqkv, V;
+    float eps;
+    const uint16_t* x;   // [B][H] token input
+    uint16_t* logits;    // [B][V]
+    uint32_t* seq;       // token counter (workspace header)
+    uint32_t* done;      // CTAs finished with this token
+    uint32_t* abort;     // epoch of a token whose waits gave up (stops the others early)
+    uint64_t* llA;       // [L][B][H/2]   query block of qkv (attention stand-in)
+    uint64_t* llX1;      // [L][B][H/2]   x + o
+    uint64_t* llM;       // [L][B][F/2]   silu(gate) * up
+    uint64_t* llX;       // [L+1][B][H/2] layer outputs (index 0 unused)
+    uint64_t* llV;       // [L][B][H/2]   RMS-normalised layer inputs (residual of O)
+    uint16_t* pV;        // [L+1][B][H]   RMS-normalised layer inputs; [L] feeds the LM head
+    uint16_t* pX2;       // [L][B][H]     layer outputs
+    uint16_t* pQKV;      // [L][B][Nqkv]
+    uint16_t* pO;        // [L][B][H]
+    uint16_t* pX1;       // [L][B][H]
+    uint16_t* pGU;       // [L][B][2F]
+    uint16_t* pM;        // [L][B][F]
+    uint16_t* pD;        // [L][B][H]
+    int nslots;
+    uint32_t slot_bytes;
+    uint32_t x_bytes;
+    uint32_t* err;
+};
+
+struct Stage {
+    int type, layer, N, K, rpi, items;
+    const uint32_t* W;
+    const uint16_t* s;
+};
+
+__device__ __forceinline__ Stage stage_at(const ChainParams& p, int st)
+{
+    Stage g;
+    if (st == 4 * p.L) {
+        g.type = kLM; g.layer = p.L; g.N = p.V; g.K = p.H; g.rpi = 2; g.items = (p.V + 1) / 2;
+    } else {
+        g.layer = st >> 2;
+        g.type = st & 3;
+        switch (g.type) {
+            case kQKV: g.N = p.Nqkv; g.K = p.H; g.rpi = 2; g.items = p.Nqkv / 2; break;
+            case kO: g.N = p.H; g.K = p.H; g.rpi = 2; g.items = p.H / 2; break;
+            case kGU: g.N = 2 * p.F; g.K = p.H; g.rpi = 4; g.items = p.F / 2; break;
+            default: g.N = p.H; g.K = p.F; g.rpi = 2; g.items = p.H / 2; break;
+        }
+    }
+    g.W = p.mats[st].W;
+    g.s = p.mats[st].s;
+    return g;
+}
+
+// Byte layout of one chunk (items [ia, ib) of a stage) inside a slot.
+struct ChunkLayout {
+    int nrows;          // rows in the chunk (both halves for gate_up)
+    int nh;             // rows per half (gate_up) / nrows otherwise
+    uint32_t codes_bytes, scale_bytes;
+};
+
+__device__ __forceinline__ ChunkLayout chunk_layout(const Stage& g, int ia, int ib)
+{
+    ChunkLayout c;
+    if (g.type == kGU) {
+        c.nh = 2 * (ib - ia);
+        c.nrows = 2 * c.nh;
+    } else {
+        const int r1 = min(2 * ib, g.N);
+        c.nrows = r1 - 2 * ia;
+        c.nh = c.nrows;
+    }
+    c.codes_bytes = static_cast<uint32_t>(c.nrows) * (g.K / 2);
+    c.scale_bytes = static_cast<uint32_t>(c.nrows) * (g.K / 16);
+    return c;
+}
+
+__device__ __forceinline__ void cta_items(int items, int* i0, int* i1)
+{
+    *i0 = static_cast<int>(static_cast<int64_t>(blockIdx.x) * items / gridDim.x);
+    *i1 = static_cast<int>(static_cast<int64_t>(blockIdx.x + 1) * items / gridDim.x);
+}
+
+__device__ __forceinline__ int items_per_slot(const ChainParams& p, const Stage& g)
+{
+    const uint32_t item_bytes = static_cast<uint32_t>(g.rpi) * (g.K / 2 + g.K / 16);
+    const int ips = static_cast<int>(p.slot_bytes / item_bytes);
+    return ips < 1 ? 1 : ips;
+}
+
+// ------------------------------------------------------- flagged words --
+
+__device__ __forceinline__ void ll_store(uint64_t* addr, uint32_t data, uint32_t epoch)
+{
+    const uint64_t v = (static_cast<uint64_t>(epoch) << 32) | data;
+    asm volatile("st.relaxed.gpu.global.b64 [%0], %1;" ::"l"(addr), "l"(v) : "memory");
+}
+
+__device__ __forceinline__ void ll_load2_raw(const uint64_t* addr, uint64_t& a, uint64_t& b)
+{
+    asm volatile("ld.relaxed.gpu.global.v2.b64 {%0, %1}, [%2];" : "=l"(a), "=l"(b) : "l"(addr) : "memory");
+}
+
+__device__ __forceinline__ uint64_t ll_load1_raw(const uint64_t* addr)
+{
+    uint64_t a;
+    asm volatile("ld.relaxed.gpu.global.b64 %0, [%1];" : "=l"(a) : "l"(addr) : "memory");
+    return a;
+}
+
+// A wait gives up after kWaitTimeoutNs, or at once when another CTA already
+// gave up on this token; the first to give up records the token in *abort.
+__device__ __forceinline__ bool gave_up(uint64_t t0, uint32_t epoch, uint32_t* abort)
+{
+    if (*reinterpret_cast<const volatile uint32_t*>(abort) == epoch) return true;
+    if (globaltimer_ns() - t0 > kWaitTimeoutNs) {
+        atomicExch(abort, epoch);
+        return true;
+    }
+    return false;
+}
+
+// Four consecutive flagged words (8 fp16 values) at a 32-byte aligned address;
+// polls until all four carry `epoch`.
+__device__ __forceinline__ uint4 ll_load4(const uint64_t* addr, uint32_t epoch, uint32_t* err, uint32_t* abort)
+{
+    uint64_t a, b, c, d;
+    ll_load2_raw(addr, a, b);
+    ll_load2_raw(addr + 2, c, d);
+    if (static_cast<uint32_t>(a >> 32) != epoch || static_cast<uint32_t>(b >> 32) != epoch ||
+        static_cast<uint32_t>(c >> 32) != epoch || static_cast<uint32_t>(d >> 32) != epoch) {
+        const uint64_t t0 = globaltimer_ns();
+        for (uint32_t it = 0;; ++it) {
+            ll_load2_raw(addr, a, b);
+            ll_load2_raw(addr + 2, c, d);
+            if (static_cast<uint32_t>(a >> 32) == epoch && static_cast<uint32_t>(b >> 32) == epoch &&
+                static_cast<uint32_t>(c >> 32) == epoch && static_cast<uint32_t>(d >> 32) == epoch)
+                break;
+            if ((it & 63) == 63 && gave_up(t0, epoch, abort)) {
+                atomicOr(err, kErrFlagTimeout);
+                break;
+            }
+        }
+    }
+    return make_uint4(static_cast<uint32_t>(a), static_cast<uint32_t>(b), static_cast<uint32_t>(c),
+                      static_cast<uint32_t>(d));
+}
+
+__device__ __forceinline__ uint32_t ll_load(const uint64_t* addr, uint32_t epoch, uint32_t* err, uint32_t* abort)
+{
+    uint64_t a = ll_load1_raw(addr);
+    if (static_cast<uint32_t>(a >> 32) != epoch) {
+        const uint64_t t0 = globaltimer_ns();
+        for (uint32_t it = 0;; ++it) {
+            a = ll_load1_raw(addr);
+            if (static_cast<uint32_t>(a >> 32) == epoch) break;
+            if ((it & 63) == 63 && gave_up(t0, epoch, abort)) {
+                atomicOr(err, kErrFlagTimeout);
+                break;
+            }
+        }
+    }
+    return static_cast<uint32_t>(a);
+}
+
+__device__ __forceinline__ float lo_f(uint32_t v) { return half_bits_to_float(static_cast<uint16_t>(v & 0xFFFFu)); }
+__device__ __forceinline__ float hi_f(uint32_t v) { return half_bits_to_float(static_cast<uint16_t>(v >> 16)); }
+__device__ __forceinline__ uint32_t pack2(uint16_t a, uint16_t b)
+{
+    return static_cast<uint32_t>(a) | (static_cast<uint32_t>(b) << 16);
+}
+// fp16(a + b): the fp32 sum of two fp16 values rounded to fp16 equals the
+// correctly rounded fp16 sum (fp32 carries more than 2 * 11 + 2 bits).
+__device__ __forceinline__ uint16_t add_h(float a, float b) { return float_to_half_bits(a + b); }
+
+// fp16(r * v_i) for the 8 fp16 values of a chunk
+__device__ __forceinline__ uint4 scale8(uint4 v, float r)
+{
+    uint32_t w[4] = {v.x, v.y, v.z, v.w};
+#pragma unroll
+    for (int i = 0; i < 4; ++i)
+        w[i] = pack2(float_to_half_bits(r * lo_f(w[i])), float_to_half_bits(r * hi_f(w[i])));
+    return make_uint4(w[0], w[1], w[2], w[3]);
+}
+
+__device__ __forceinline__ float sum8_sq(uint4 v)
+{
+    const uint32_t w[4] = {v.x, v.y, v.z, v.w};
+    float s = 0.f;
+#pragma unroll
+    for (int i = 0; i < 4; ++i) {
+        const float a = lo_f(w[i]), b = hi_f(w[i]);
+        s = fmaf(a, a, s);
+        s = fmaf(b, b, s);
+    }
+    return s;
+}
+
+// ---------------------------------------------------------- the kernel --
+
+template <int B>
+__global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const ChainParams p)
+{
+    extern __shared__ __align__(1024) uint8_t smem[];
+    uint64_t* full = reinterpret_cast<uint64_t*>(smem);
+    uint64_t* empty = full + kChainMaxSlots;
+    float* red = reinterpret_cast<float*>(smem + 2 * kChainMaxSlots * 8);   // [kNW][B]
+    uint32_t* epoch_sh = reinterpret_cast<uint32_t*>(smem + 2 * kChainMaxSlots * 8 + kNW * kMaxChainBatch * 4);
+    uint4* xs = reinterpret_cast<uint4*>(smem + kChainHeader);
+    uint8_t* slots = smem + kChainHeader + p.x_bytes;
+
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int nstages = 4 * p.L + 1;
+
+    if (threadIdx.x == 0) {
+        for (int i = 0; i < p.nslots; ++i) {
+            mbar_init(&full[i], 1);
+            mbar_init(&empty[i], kNW);
+        }
+        mbar_fence_init();
+        uint32_t s;
+        asm volatile("ld.relaxed.gpu.global.b32 %0, [%1];" : "=r"(s) : "l"(p.seq) : "memory");
+        *epoch_sh = s + 1u;
+    }
+    __syncthreads();
+    const uint32_t epoch = *epoch_sh;
+
+    if (warp == kNW) {
+        // ------------------------------------------------ producer warp
+        if (lane == 0) {
+            const uint64_t pol = l2_policy_evict_first();
+            int ord = 0;
+            for (int st = 0; st < nstages; ++st) {
+                const Stage g = stage_at(p, st);
+                int i0, i1;
+                cta_items(g.items, &i0, &i1);
+                const int ips = items_per_slot(p, g);
+                const int wpr = g.K >> 3, gpr = g.K >> 5;
+                for (int ia = i0; ia < i1; ia += ips, ++ord) {
+                    const int ib = min(i1, ia + ips);
+                    const int slot = ord % p.nslots, round = ord / p.nslots;
+                    if (round > 0) mbar_wait(&empty[slot], (round - 1) & 1, p.err);
+                    const ChunkLayout c = chunk_layout(g, ia, ib);
+                    uint8_t* dst = slots + static_cast<size_t>(slot) * p.slot_bytes;
+                    mbar_arrive_expect_tx(&full[slot], c.codes_bytes + c.scale_bytes);
+                    if (g.type == kGU) {
+                        const uint32_t hc = c.codes_bytes / 2, hs = c.scale_bytes / 2;
+                        const size_t up = static_cast<size_t>(p.F);
+                        bulk_g2s(dst, g.W + static_cast<size_t>(2 * ia) * wpr, hc, &full[slot], pol);
+                        bulk_g2s(dst + hc, g.W + (up + 2 * ia) * wpr, hc, &full[slot], pol);
+                        bulk_g2s(dst + c.codes_bytes, g.s + static_cast<size_t>(2 * ia) * gpr, hs, &full[slot], pol);
+                        bulk_g2s(dst + c.codes_bytes + hs, g.s + (up + 2 * ia) * gpr, hs, &full[slot], pol);
+                    } else {
+                        bulk_g2s(dst, g.W + static_cast<size_t>(2 * ia) * wpr, c.codes_bytes, &full[slot], pol);
+                        bulk_g2s(dst + c.codes_bytes, g.s + static_cast<size_t>(2 * ia) * gpr, c.scale_bytes,
+                                 &full[slot], pol);
+                    }
+                }
+            }
+            const int first = ord > p.nslots ? ord - p.nslots : 0;
+            for (int o = first; o < ord; ++o) mbar_wait(&full[o % p.nslots], (o / p.nslots) & 1, p.err);
+        }
+    } else {
+        // ------------------------------------------------ consumer warps
+        const int H = p.H, F = p.F;
+        int ord = 0;
+        for (int st = 0; st < nstages; ++st) {
+            const Stage g = stage_at(p, st);
+            int i0, i1;
+            cta_items(g.items, &i0, &i1);
+            if (i1 <= i0) continue;
+            const int l = g.layer;
+            const int K = g.K, gpr = K >> 5, cpr = K >> 3;
+
+            // -- stage the input vector (all consumer warps) and its RMS factor
+            named_barrier_sync(1, kNW * 32);   // every warp is done with the previous xs
+            {
+                const uint64_t* ll = nullptr;
+                const bool plain = (g.type == kQKV && l == 0);
+                if (g.type == kQKV) ll = p.llX + static_cast<size_t>(l) * B * (H / 2);
+                else if (g.type == kO) ll = p.llA + static_cast<size_t>(l) * B * (H / 2);
+                else if (g.type == kGU) ll = p.llX1 + static_cast<size_t>(l) * B * (H / 2);
+                else if (g.type == kDOWN) ll = p.llM + static_cast<size_t>(l) * B * (F / 2);
+                else ll = p.llX + static_cast<size_t>(p.L) * B * (H / 2);
+                float ss[B];
+#pragma unroll
+                for (int b = 0; b < B; ++b) ss[b] = 0.f;
+                for (int i = threadIdx.x; i < B * cpr; i += kNW * 32) {
+                    const int b = i / cpr, c = i - b * cpr;
+                    uint4 v;
+                    if (plain) {
+                        v = reinterpret_cast<const uint4*>(p.x)[i];
+                    } else {
+                        v = ll_load4(ll + static_cast<size_t>(b) * (K / 2) + 4 * c, epoch, p.err, p.abort);
+                    }
+                    xs[b * cpr + x_chunk(c >> 2, c & 3)] = v;
+#pragma unroll
+                    for (int bb = 0; bb < B; ++bb)
+                        if (bb == b) ss[bb] += sum8_sq(v);
+                }
+#pragma unroll
+                for (int b = 0; b < B; ++b) {
+                    const float v = warp_sum(ss[b]);
+                    if (lane == 0) red[warp * kMaxChainBatch + b] = v;
+                }
+            }
+            named_barrier_sync(1, kNW * 32);
+            float rf[B];
+#pragma unroll
+            for (int b = 0; b < B; ++b) {
+                float t = 0.f;
+                for (int w = 0; w < kNW; ++w) t += red[w * kMaxChainBatch + b];
+                rf[b] = (g.type == kDOWN) ? 1.f : 1.f / sqrtf(t / static_cast<float>(K) + p.eps);
+            }
+            if (g.type == kQKV || g.type == kLM) {
+                // re-feed after RMS normalisation: xs <- fp16(r * u), in place;
+                // each thread rescales the chunks it staged itself
+                const bool writer = (i0 == 0);   // first CTA that owns items
+                uint16_t* pv = p.pV + static_cast<size_t>(l) * B * H;
+                uint64_t* lv = p.llV + static_cast<size_t>(l) * B * (H / 2);
+                for (int i = threadIdx.x; i < B * cpr; i += kNW * 32) {
+                    const int b = i / cpr, c = i - b * cpr;
+                    uint4& cell = xs[b * cpr + x_chunk(c >> 2, c & 3)];
+                    float r = rf[0];
+#pragma unroll
+                    for (int bb = 1; bb < B; ++bb)
+                        if (bb == b) r = rf[bb];
+                    const uint4 v = scale8(cell, r);
+                    cell = v;
+                    if (writer) {
+                        reinterpret_cast<uint4*>(pv + static_cast<size_t>(b) * H)[c] = v;
+                        if (g.type == kQKV) {
+                            uint64_t* w = lv + static_cast<size_t>(b) * (H / 2) + 4 * c;
+                            ll_store(w + 0, v.x, epoch);
+                            ll_store(w + 1, v.y, epoch);
+                            ll_store(w + 2, v.z, epoch);
+                            ll_store(w + 3, v.w, epoch);
+                        }
+                    }
+                }
+                named_barrier_sync(1, kNW * 32);
+#pragma unroll
+                for (int b = 0; b < B; ++b) rf[b] = 1.f;
+            }
+
+            // -- stream the CTA's items of this stage
+            const int ips = items_per_slot(p, g);
+            for (int ia = i0; ia < i1; ia += ips, ++ord) {
+                const int ib = min(i1, ia + ips);
+                const int slot = ord % p.nslots;
+                mbar_wait(&full[slot], (ord / p.nslots) & 1, p.err);
+                const uint8_t* base = slots + static_cast<size_t>(slot) * p.slot_bytes;
+                const ChunkLayout c = chunk_layout(g, ia, ib);
+                const int first = ia + ((warp - (ia - i0) % kNW) + kNW) % kNW;
+                for (int it = first; it < ib; it += kNW) {
+                    const int ii = it - ia;
+                    constexpr int RMAX = 4;
+                    const uint4* crow[RMAX];
+                    const uint16_t* srow[RMAX];
+                    const int rpi = g.rpi;
+                    if (g.type == kGU) {
+#pragma unroll
+                        for (int r = 0; r < 4; ++r) {
+                            const int half = r >> 1, rr = 2 * ii + (r & 1);
+                            crow[r] = reinterpret_cast<const uint4*>(base + static_cast<size_t>(half) * (c.codes_bytes / 2) +
+                                                                     static_cast<size_t>(rr) * (K / 2));
+                            srow[r] = reinterpret_cast<const uint16_t*>(base + c.codes_bytes + half * (c.scale_bytes / 2) +
+                                                                        rr * (K / 16));
+                        }
+                    } else {
+                        const int nvalid = min(2, g.N - 2 * it);
+#pragma unroll
+                        for (int r = 0; r < 2; ++r) {
+                            const int rr = 2 * ii + (r < nvalid ? r : 0);
+                            crow[r] = reinterpret_cast<const uint4*>(base + static_cast<size_t>(rr) * (K / 2));
+                            srow[r] = reinterpret_cast<const uint16_t*>(base + c.codes_bytes + rr * (K / 16));
+                        }
+                        crow[2] = crow[3] = crow[0];
+                        srow[2] = srow[3] = srow[0];
+                    }
+                    float acc[RMAX][B];
+#pragma unroll
+                    for (int r = 0; r < RMAX; ++r)
+#pragma unroll
+                        for (int b = 0; b < B; ++b) acc[r][b] = 0.f;
+
+                    if (rpi == 4) {
+                        for (int gg = lane; gg < gpr; gg += 32) {
+#pragma unroll
+                            for (int r = 0; r < 4; ++r)
+                                group_dot_smem<B>(crow[r][gg], half_bits_to_float(srow[r][gg]), xs, cpr, gg, acc[r]);
+                        }
+                    } else {
+                        for (int gg = lane; gg < gpr; gg += 32) {
+#pragma unroll
+                            for (int r = 0; r < 2; ++r)
+                                group_dot_smem<B>(crow[r][gg], half_bits_to_float(srow[r][gg]), xs, cpr, gg, acc[r]);
+                        }
+                    }
+#pragma unroll
+                    for (int r = 0; r < RMAX; ++r)
+#pragma unroll
+                        for (int b = 0; b < B; ++b)
+                            if (r < rpi) acc[r][b] = warp_sum(acc[r][b]);
+
+                    // -- fused epilogue (one lane per batch row)
+#pragma unroll
+                    for (int b = 0; b < B; ++b) {
+                        if (lane != b) continue;
+                        const int n = 2 * it;
+                        if (g.type == kQKV) {
+                            const uint16_t y0 = float_to_half_bits(rf[b] * acc[0][b]);
+                            const uint16_t y1 = float_to_half_bits(rf[b] * acc[1][b]);
+                            const uint32_t w = pack2(y0, y1);
+                            *reinterpret_cast<uint32_t*>(p.pQKV + (static_cast<size_t>(l) * B + b) * p.Nqkv + n) = w;
+                            if (n < H) ll_store(p.llA + (static_cast<size_t>(l) * B + b) * (H / 2) + n / 2, w, epoch);
+                        } else if (g.type == kO) {
+                            const uint16_t o0 = float_to_half_bits(rf[b] * acc[0][b]);
+                            const uint16_t o1 = float_to_half_bits(rf[b] * acc[1][b]);
+                            const uint32_t xw =
+                                ll_load(p.llV + (static_cast<size_t>(l) * B + b) * (H / 2) + n / 2, epoch, p.err, p.abort);
+                            const uint32_t x1 = pack2(add_h(lo_f(xw), half_bits_to_float(o0)),
+                                                      add_h(hi_f(xw), half_bits_to_float(o1)));
+                            const size_t off = (static_cast<size_t>(l) * B + b) * H + n;
+                            *reinterpret_cast<uint32_t*>(p.pO + off) = pack2(o0, o1);
+                            *reinterpret_cast<uint32_t*>(p.pX1 + off) = x1;
+                            ll_store(p.llX1 + (static_cast<size_t>(l) * B + b) * (H / 2) + n / 2, x1, epoch);
+                        } else if (g.type == kGU) {
+                            const int j = n;  // pair index of gate/up rows j, j+1
+                            const uint16_t g0 = float_to_half_bits(rf[b] * acc[0][b]);
+                            const uint16_t g1 = float_to_half_bits(rf[b] * acc[1][b]);
+                            const uint16_t u0 = float_to_half_bits(rf[b] * acc[2][b]);
+                            const uint16_t u1 = float_to_half_bits(rf[b] * acc[3][b]);
+                            const float gf0 = half_bits_to_float(g0), gf1 = half_bits_to_float(g1);
+                            const uint16_t m0 = float_to_half_bits(gf0 / (1.f + expf(-gf0)) * half_bits_to_float(u0));
+                            const uint16_t m1 = float_to_half_bits(gf1 / (1.f + expf(-gf1)) * half_bits_to_float(u1));
+                            const size_t gu = (static_cast<size_t>(l) * B + b) * (2 * F);
+                            *reinterpret_cast<uint32_t*>(p.pGU + gu + j) = pack2(g0, g1);
+                            *reinterpret_cast<uint32_t*>(p.pGU + gu + F + j) = pack2(u0, u1);
+                            const uint32_t mw = pack2(m0, m1);
+                            *reinterpret_cast<uint32_t*>(p.pM + (static_cast<size_t>(l) * B + b) * F + j) = mw;
+                            ll_store(p.llM + (static_cast<size_t>(l) * B + b) * (F / 2) + j / 2, mw, epoch);
+                        } else if (g.type == kDOWN) {
+                            const uint16_t d0 = float_to_half_bits(acc[0][b]);
+                            const uint16_t d1 = float_to_half_bits(acc[1][b]);
+                            const uint32_t x1 =
+                                ll_load(p.llX1 + (static_cast<size_t>(l) * B + b) * (H / 2) + n / 2, epoch, p.err, p.abort);
+                            const uint32_t x2 = pack2(add_h(lo_f(x1), half_bits_to_float(d0)),
+                                                      add_h(hi_f(x1), half_bits_to_float(d1)));
+                            *reinterpret_cast<uint32_t*>(p.pD + (static_cast<size_t>(l) * B + b) * H + n) = pack2(d0, d1);
+                            *reinterpret_cast<uint32_t*>(p.pX2 + (static_cast<size_t>(l) * B + b) * H + n) = x2;
+                            ll_store(p.llX + (static_cast<size_t>(l + 1) * B + b) * (H / 2) + n / 2, x2, epoch);
+                        } else {
+                            uint16_t* out = p.logits + static_cast<size_t>(b) * p.V;
+                            out[n] = float_to_half_bits(rf[b] * acc[0][b]);
+                            if (n + 1 < p.V) out[n + 1] = float_to_half_bits(rf[b] * acc[1][b]);
+                        }
+                    }
+                }
+                __syncwarp();
+                if (lane == 0) mbar_arrive(&empty[slot]);
+            }
+        }
+    }
+
+    // ---------------------------------------------------- token epilogue
+    __syncthreads();
+    if (threadIdx.x == 0) {
+        __threadfence();
+        const uint32_t prev = atomicAdd(p.done, 1u);
+        if (prev == gridDim.x - 1) {
+            atomicExch(p.done, 0u);
+            __threadfence();
+            atomicExch(p.seq, epoch);
+        }
+    }
+}
+
+// ---------------------------------------------------------------- host --
+
+struct Layout {
+    size_t header, mats, llA, llX1, llM, llX, llV, pV, pX2, pQKV, pO, pX1, pGU, pM, pD, x_stage, logits_stage, total;
+    size_t ll_begin, ll_end;
+};
+
+struct Dims {
+    int L, H, F, Nqkv, V, B;
+};
+
+bool table_dims(const wq4_layer_table* t, Dims* d)
+{
+    if (!t) return false;
+    if (t->num_layers < 1 || t->num_layers > 4096) return false;
+    if (t->hidden < 256 || t->hidden % 256) return false;
+    if (t->ffn < 256 || t->ffn % 256) return false;
+    if (t->n_q_heads < 1 || t->n_kv_heads < 0 || t->head_dim < 1) return false;
+    if (static_cast<int64_t>(t->n_q_heads) * t->head_dim != t->hidden) return false;
+    const int64_t nqkv = static_cast<int64_t>(t->n_q_heads + 2 * t->n_kv_heads) * t->head_dim;
+    if (nqkv % 2 || nqkv > (1 << 24)) return false;
+    if (t->vocab < 1 || t->vocab > (1 << 24)) return false;
+    if (t->batch < 1 || t->batch > WQ4_MAX_BATCH) return false;
+    if (!(t->rms_eps > 0.f) || !std::isfinite(t->rms_eps)) return false;
+    if (!t->layers) return false;
+    d->L = t->num_layers;
+    d->H = t->hidden;
+    d->F = t->ffn;
+    d->Nqkv = static_cast<int>(nqkv);
+    d->V = t->vocab;
+    d->B = t->batch;
+    return true;
+}
+
+Layout make_layout(const Dims& d)
+{
+    Layout y;
+    size_t o = 0;
+    auto take = [&](size_t bytes) {
+        const size_t at = o;
+        o = align_up(o + bytes, 256);
+        return at;
+    };
+    const size_t B = d.B, L = d.L, H = d.H, F = d.F;
+    y.header = take(256);
+    y.mats = take(sizeof(DevMat) * (4 * L + 1));
+    y.ll_begin = o;
+    y.llA = take(8 * L * B * (H / 2));
+    y.llX1 = take(8 * L * B * (H / 2));
+    y.llM = take(8 * L * B * (F / 2));
+    y.llX = take(8 * (L + 1) * B * (H / 2));
+    y.llV = take(8 * L * B * (H / 2));
+    y.ll_end = o;
+    y.pV = take(2 * (L + 1) * B * H);
+    y.pX2 = take(2 * L * B * H);
+    y.pQKV = take(2 * L * B * d.Nqkv);
+    y.pO = take(2 * L * B * H);
+    y.pX1 = take(2 * L * B * H);
+    y.pGU = take(2 * L * B * 2 * F);
+    y.pM = take(2 * L * B * F);
+    y.pD = take(2 * L * B * H);
+    y.x_stage = take(2 * B * H);
+    y.logits_stage = take(2 * B * static_cast<size_t>(d.V));
+    y.total = o;
+    return y;
+}
+
+struct Plan {
+    wq4_layer_table table;
+    std::vector<wq4_layer> layers;
+    Dims dims;
+    Layout lay;
+    int device;
+    int grid;
+    int nslots;
+    uint32_t slot_bytes, x_bytes;
+    size_t smem;
+};
+
+std::mutex g_plan_mu;
+std::map<const wq4_layer_table*, Plan> g_plans;
+
+bool same_contents(const Plan& pl, const wq4_layer_table* t)
+{
+    if (std::memcmp(&pl.table, t, sizeof(*t)) != 0) return false;
+    return std::memcmp(pl.layers.data(), t->layers, sizeof(wq4_layer) * t->num_layers) == 0;
+}
+
+bool mat_ok(const wq4_mat& m)
+{
+    return m.W && m.s && aligned(m.W, 16) && aligned(m.s, 16);
+}
+
+template <int B>
+cudaError_t set_chain_attr(int smem)
+{
+    return cudaFuncSetAttribute(chain_kernel<B>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+}
+
+// Slot size: a multiple of 128 bytes holding at least one item of every
+// stage, chosen to waste the least ring space over the chain's byte mix.
+uint32_t choose_slot_bytes(const Dims& d)
+{
+    struct S { size_t item, bytes; };
+    const size_t rowH = static_cast<size_t>(d.H) / 2 + d.H / 16, rowF = static_cast<size_t>(d.F) / 2 + d.F / 16;
+    const S st[5] = {{2 * rowH, static_cast<size_t>(d.Nqkv) * rowH},
+                     {2 * rowH, static_cast<size_t>(d.H) * rowH},
+                     {4 * rowH, static_cast<size_t>(2) * d.F * rowH},
+                     {2 * rowF, static_cast<size_t>(d.H) * rowF},
+                     {2 * rowH, static_cast<size_t>(d.V) * rowH}};
+    size_t max_item = 0;
+    for (const S& s : st) max_item = s.item > max_item ? s.item : max_item;
+    size_t lo = align_up(max_item, 128);
+    if (lo < 16384) lo = 16384;
+    size_t best = lo;
+    double best_waste = 1e300;
+    for (size_t sb = lo; sb <= lo + 8192; sb += 128) {
+        double waste = 0;
+        for (const S& s : st) {
+            const size_t ips = sb / s.item;
+            waste += static_cast<double>(s.bytes) * (1.0 - static_cast<double>(ips * s.item) / sb);
+        }
+        if (waste < best_waste) {
+            best_waste = waste;
+            best = sb;
+        }
+    }
+    return static_cast<uint32_t>(best);
+}
+
+int build_plan(const wq4_layer_table* t, Plan* pl, cudaStream_t stream)
+{
+    Dims d;
+    if (!table_dims(t, &d)) return WQ4_ERR_INVALID;
+    if (d.B > kMaxChainBatch) return WQ4_ERR_UNSUPPORTED;
+    for (int l = 0; l < d.L; ++l) {
+        const wq4_layer& ly = t->layers[l];
+        if (!mat_ok(ly.qkv) || !mat_ok(ly.o) || !mat_ok(ly.gate_up) || !mat_ok(ly.down)) return WQ4_ERR_INVALID;
+    }
+    if (!mat_ok(t->lm_head)) return WQ4_ERR_INVALID;
+    const Layout lay = make_layout(d);
+    if (!t->workspace || !aligned(t->workspace, 256)) return WQ4_ERR_ALIGN;
+    if (t->workspace_bytes < lay.total) return WQ4_ERR_INVALID;
+    int dev = 0;
+    const DeviceInfo* di = current_device_info(&dev);
+    if (!di) return WQ4_ERR_CUDA;
+    if (!di->coop_launch) return WQ4_ERR_UNSUPPORTED;
+    const uint32_t x_bytes = static_cast<uint32_t>(align_up(static_cast<size_t>(d.B) * 2 * (d.H > d.F ? d.H : d.F), 128));
+    const uint32_t slot_bytes = choose_slot_bytes(d);
+    const long avail = static_cast<long>(di->smem_optin) - kChainHeader - static_cast<long>(x_bytes);
+    int nslots = avail > 0 ? static_cast<int>(avail / slot_bytes) : 0;
+    if (nslots < 2) return WQ4_ERR_UNSUPPORTED;
+    if (nslots > kChainMaxSlots) nslots = kChainMaxSlots;
+    const size_t smem = kChainHeader + x_bytes + static_cast<size_t>(nslots) * slot_bytes;
+    cudaError_t e = cudaSuccess;
+    switch (d.B) {
+        case 1: e = set_chain_attr<1>(static_cast<int>(smem)); break;
+        case 2: e = set_chain_attr<2>(static_cast<int>(smem)); break;
+        case 3: e = set_chain_attr<3>(static_cast<int>(smem)); break;
+        default: e = set_chain_attr<4>(static_cast<int>(smem)); break;
+    }
+    if (e != cudaSuccess) return WQ4_ERR_CUDA;
+
+    std::vector<DevMat> mats(4 * static_cast<size_t>(d.L) + 1);
+    for (int l = 0; l < d.L; ++l) {
+        const wq4_layer& ly = t->layers[l];
+        mats[4 * l + 0] = {ly.qkv.W, ly.qkv.s};
+        mats[4 * l + 1] = {ly.o.W, ly.o.s};
+        mats[4 * l + 2] = {ly.gate_up.W, ly.gate_up.s};
+        mats[4 * l + 3] = {ly.down.W, ly.down.s};
+    }
+    mats[4 * d.L] = {t->lm_head.W, t->lm_head.s};
+    uint8_t* ws = static_cast<uint8_t*>(t->workspace);
+    // header (token counter) and every flagged word start at zero: epoch 0 never matches
+    if (cudaMemsetAsync(ws + lay.header, 0, 256, stream) != cudaSuccess) return WQ4_ERR_CUDA;
+    if (cudaMemsetAsync(ws + lay.ll_begin, 0, lay.ll_end - lay.ll_begin, stream) != cudaSuccess) return WQ4_ERR_CUDA;
+    // pageable source: the call returns once the bytes are staged
+    if (cudaMemcpyAsync(ws + lay.mats, mats.data(), sizeof(DevMat) * mats.size(), cudaMemcpyHostToDevice, stream) !=
+        cudaSuccess)
+        return WQ4_ERR_CUDA;
+
+    pl->table = *t;
+    pl->layers.assign(t->layers, t->layers + d.L);
+    pl->dims = d;
+    pl->lay = lay;
+    pl->device = dev;
+    pl->grid = di->sm_count;
+    pl->nslots = nslots;
+    pl->slot_bytes = slot_bytes;
+    pl->x_bytes = x_bytes;
+    pl->smem = smem;
+    return WQ4_OK;
+}
+
+int launch_chain(const Plan& pl, const uint16_t* x, uint16_t* logits, cudaStream_t stream)
+{
+    uint8_t* ws = static_cast<uint8_t*>(pl.table.workspace);
+    const Layout& y = pl.lay;
+    ChainParams p;
+    p.mats = reinterpret_cast<const DevMat*>(ws + y.mats);
+    p.L = pl.dims.L;
+    p.H = pl.dims.H;
+    p.F = pl.dims.F;
+    p.Nqkv = pl.dims.Nqkv;
+    p.V = pl.dims.V;
+    p.eps = pl.table.rms_eps;
+    p.x = x;
+    p.logits = logits;
+    p.seq = reinterpret_cast<uint32_t*>(ws + y.header);
+    p.done = reinterpret_cast<uint32_t*>(ws + y.header) + 1;
+    p.abort = reinterpret_cast<uint32_t*>(ws + y.header) + 2;
+    p.llA = reinterpret_cast<uint64_t*>(ws + y.llA);
+    p.llX1 = reinterpret_cast<uint64_t*>(ws + y.llX1);
+    p.llM = reinterpret_cast<uint64_t*>(ws + y.llM);
+    p.llX = reinterpret_cast<uint64_t*>(ws + y.llX);
+    p.llV = reinterpret_cast<uint64_t*>(ws + y.llV);
+    p.pV = reinterpret_cast<uint16_t*>(ws + y.pV);
+    p.pX2 = reinterpret_cast<uint16_t*>(ws + y.pX2);
+    p.pQKV = reinterpret_cast<uint16_t*>(ws + y.pQKV);
+    p.pO = reinterpret_cast<uint16_t*>(ws + y.pO);
+    p.pX1 = reinterpret_cast<uint16_t*>(ws + y.pX1);
+    p.pGU = reinterpret_cast<uint16_t*>(ws + y.pGU);
+    p.pM = reinterpret_cast<uint16_t*>(ws + y.pM);
+    p.pD = reinterpret_cast<uint16_t*>(ws + y.pD);
+    p.nslots = pl.nslots;
+    p.slot_bytes = pl.slot_bytes;
+    p.x_bytes = pl.x_bytes;
+    p.err = status_word();
+    if (!p.err) return WQ4_ERR_CUDA;
+
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(pl.grid);
+    cfg.blockDim = dim3(kChainThreads);
+    cfg.dynamicSmemBytes = pl.smem;
+    cfg.stream = stream;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeCooperative;
+    attr[0].val.cooperative = 1;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    cudaError_t e;
+    switch (pl.dims.B) {
+        case 1: e = cudaLaunchKernelEx(&cfg, chain_kernel<1>, p); break;
+        case 2: e = cudaLaunchKernelEx(&cfg, chain_kernel<2>, p); break;
+        case 3: e = cudaLaunchKernelEx(&cfg, chain_kernel<3>, p); break;
+        default: e = cudaLaunchKernelEx(&cfg, chain_kernel<4>, p); break;
+    }
+    return e == cudaSuccess ? WQ4_OK : WQ4_ERR_CUDA;
+}
+
+// Finds (or builds) the plan of `t`; returns a copy to launch from.
+int get_plan(const wq4_layer_table* t, Plan* out, cudaStream_t stream)
+{
+    if (!t) return WQ4_ERR_INVALID;
+    Dims d;
+    if (!table_dims(t, &d)) return WQ4_ERR_INVALID;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return WQ4_ERR_CUDA;
+    std::lock_guard<std::mutex> lock(g_plan_mu);
+    auto it = g_plans.find(t);
+    if (it != g_plans.end() && it->second.device == dev && same_contents(it->second, t)) {
+        *out = it->second;
+        return WQ4_OK;
+    }
+    Plan pl;
+    const int rc = build_plan(t, &pl, stream);
+    if (rc != WQ4_OK) return rc;
+    g_plans[t] = pl;
+    *out = pl;
+    return WQ4_OK;
+}
+
+}  // namespace
+}  // namespace wq4
+
+using namespace wq4;
+
+extern "C" size_t wq4_chain_workspace_bytes(const wq4_layer_table* table)
+{
+    Dims d;
+    if (!table_dims(table, &d)) return 0;
+    return make_layout(d).total;
+}
+
+extern "C" int wq4_decode_chain(const wq4_layer_table* table, const uint16_t* x, uint16_t* logits, void* stream)
+{
+    if (!table || !x || !logits) return WQ4_ERR_INVALID;
+    if (!aligned(x, 16) || !aligned(logits, 2)) return WQ4_ERR_ALIGN;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    Plan pl;
+    const int rc = get_plan(table, &pl, st);
+    if (rc != WQ4_OK) return rc;
+    const size_t lb = static_cast<size_t>(pl.dims.B) * pl.dims.V * 2;
+    if (overlaps(logits, lb, x, static_cast<size_t>(pl.dims.B) * pl.dims.H * 2) ||
+        overlaps(logits, lb, table->workspace, pl.lay.logits_stage))
+        return WQ4_ERR_INVALID;
+    return launch_chain(pl, x, logits, st);
+}
+
+extern "C" int wq4_decode_chain_host(const wq4_layer_table* table, const uint16_t* x_host, uint16_t* logits_host,
+                                     void* stream)
+{
+    if (!table || !x_host || !logits_host) return WQ4_ERR_INVALID;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    Plan pl;
+    int rc = get_plan(table, &pl, st);
+    if (rc != WQ4_OK) return rc;
+    uint8_t* ws = static_cast<uint8_t*>(table->workspace);
+    uint16_t* xd = reinterpret_cast<uint16_t*>(ws + pl.lay.x_stage);
+    uint16_t* ld = reinterpret_cast<uint16_t*>(ws + pl.lay.logits_stage);
+    const size_t xb = static_cast<size_t>(pl.dims.B) * pl.dims.H * 2;
+    const size_t lb = static_cast<size_t>(pl.dims.B) * pl.dims.V * 2;
+    if (cudaMemcpyAsync(xd, x_host, xb, cudaMemcpyHostToDevice, st) != cudaSuccess) return WQ4_ERR_CUDA;
+    rc = launch_chain(pl, xd, ld, st);
+    if (rc != WQ4_OK) return rc;
+    if (cudaMemcpyAsync(logits_host, ld, lb, cudaMemcpyDeviceToHost, st) != cudaSuccess) return WQ4_ERR_CUDA;
+    return cudaStreamSynchronize(st) == cudaSuccess ? WQ4_OK : WQ4_ERR_CUDA;
+}
+
+extern "C" int wq4_chain_plan_destroy(const wq4_layer_table* table)
+{
+    std::lock_guard<std::mutex> lock(g_plan_mu);
+    return g_plans.erase(table) ? WQ4_OK : WQ4_ERR_INVALID;
+}
+
+extern "C" int wq4_chain_trace_offsets(const wq4_layer_table* table, int layer, wq4_chain_trace* out)
+{
+    Dims d;
+    if (!out || !table_dims(table, &d) || layer < 0 || layer > d.L) return WQ4_ERR_INVALID;
+    const Layout y = make_layout(d);
+    const size_t B = d.B, H = d.H, F = d.F, l = layer;
+    std::memset(out, 0, sizeof(*out));
+    out->x_in = y.pV + 2 * l * B * H;
+    if (layer == d.L) return WQ4_OK;
+    out->qkv = y.pQKV + 2 * l * B * d.Nqkv;
+    out->o = y.pO + 2 * l * B * H;
+    out->x_mid = y.pX1 + 2 * l * B * H;
+    out->gate_up = y.pGU + 2 * l * B * 2 * F;
+    out->act = y.pM + 2 * l * B * F;
+    out->down = y.pD + 2 * l * B * H;
+    out->x_out = y.pX2 + 2 * l * B * H;
+    return WQ4_OK;
+}

@@ -1,0 +1,139 @@
+"""Device-resident synthetic decoders and their layer tables.
+
+Shapes follow the 1-8B 4-bit models the paper decodes (Section 3, Table 1:
+Llama-3.1-8B; Section 1: a 4-bit 3B model).  Weights are drawn on the device
+by the seeded generator (wq4_synth_*), one stream per (layer, projection,
+codes|scales), so any row block can be regenerated on the host with
+``synth.matrix`` for checking.  torch provides the device memory; every
+computation goes through the C ABI.
+"""
+from __future__ import annotations
+
+from dataclasses import dataclass
+
+import numpy as np
+
+from . import synth
+from . import wq4 as _w
+
+
+@dataclass(frozen=True)
+class ModelShape:
+    name: str
+    num_layers: int
+    hidden: int
+    ffn: int
+    n_q_heads: int
+    n_kv_heads: int
+    head_dim: int
+    vocab: int
+
+    @property
+    def n_qkv(self) -> int:
+        return (self.n_q_heads + 2 * self.n_kv_heads) * self.head_dim
+
+    def mats(self, layer: int):
+        """(name, N, K, projection index) of one layer's projections."""
+        H, F = self.hidden, self.ffn
+        return [("qkv", self.n_qkv, H, synth.MAT_QKV), ("o", H, H, synth.MAT_O),
+                ("gate_up", 2 * F, H, synth.MAT_GATE_UP), ("down", H, F, synth.MAT_DOWN)]
+
+    def weight_count(self) -> int:
+        per_layer = sum(N * K for _, N, K, _ in self.mats(0))
+        return self.num_layers * per_layer + self.vocab * self.hidden
+
+    def weight_bytes(self) -> int:
+        """Packed codes (0.5 B) + fp16 scales (1/16 B) per weight."""
+        return self.weight_count() * 9 // 16
+
+
+# 3B-shaped: hidden 3072, 24 q + 8 kv heads of 128, FFN 8192, 28 layers.
+SHAPE_3B = ModelShape("3b", 28, 3072, 8192, 24, 8, 128, 128256)
+# 8B-shaped (Llama-3.1-8B): hidden 4096, 32 q + 8 kv heads, FFN 14336, 32 layers.
+SHAPE_8B = ModelShape("8b", 32, 4096, 14336, 32, 8, 128, 128256)
+SHAPES = {"3b": SHAPE_3B, "8b": SHAPE_8B}
+
+
+def fill_matrix(W, s, N: int, K: int, seed: int, layer: int, mat: int, stream=None) -> None:
+    _w.wq4_synth_codes(W, 0, N * K // 8, seed, synth.stream_id(synth.KIND_CODES, layer, mat), stream)
+    _w.wq4_synth_scales(s, 0, N * K // 32, seed, synth.stream_id(synth.KIND_SCALES, layer, mat),
+                        synth.SCALE_LO, synth.SCALE_HI, stream)
+
+
+class DecodeModel:
+    """A synthetic decoder resident in device memory plus its wq4 layer table."""
+
+    def __init__(self, shape: ModelShape, batch: int = 1, seed: int = 0, eps: float = 1e-5, device=None):
+        import torch
+        self.shape, self.batch, self.seed, self.eps = shape, batch, seed, eps
+        dev = torch.device("cuda") if device is None else torch.device(device)
+        self.weights = []          # per layer: dict name -> (W tensor, s tensor)
+        self._keep = []
+        layers = (_w.wq4_layer * shape.num_layers)()
+        for l in range(shape.num_layers):
+            d = {}
+            for name, N, K, mat in shape.mats(l):
+                W = torch.empty((N, K // 8), dtype=torch.int32, device=dev)
+                s = torch.empty((N, K // 32), dtype=torch.int16, device=dev)
+                fill_matrix(W, s, N, K, seed, l, mat)
+                d[name] = (W, s)
+                setattr(layers[l], name, _w.wq4_mat(W.data_ptr(), s.data_ptr()))
+            self.weights.append(d)
+        V, H = shape.vocab, shape.hidden
+        W = torch.empty((V, H // 8), dtype=torch.int32, device=dev)
+        s = torch.empty((V, H // 32), dtype=torch.int16, device=dev)
+        fill_matrix(W, s, V, H, seed, shape.num_layers, synth.MAT_LM_HEAD)
+        self.lm_head = (W, s)
+        self._layers = layers
+        t = _w.wq4_layer_table()
+        t.num_layers, t.hidden, t.ffn = shape.num_layers, shape.hidden, shape.ffn
+        t.n_q_heads, t.n_kv_heads, t.head_dim = shape.n_q_heads, shape.n_kv_heads, shape.head_dim
+        t.vocab, t.batch, t.rms_eps = shape.vocab, batch, eps
+        t.layers = layers
+        t.lm_head = _w.wq4_mat(W.data_ptr(), s.data_ptr())
+        nbytes = _w.wq4_chain_workspace_bytes(t)
+        if nbytes == 0:
+            raise ValueError(f"invalid chain shape {shape} batch {batch}")
+        self.workspace = torch.zeros(nbytes + 256, dtype=torch.uint8, device=dev)
+        base = self.workspace.data_ptr()
+        aligned = (base + 255) // 256 * 256
+        self._ws_offset = aligned - base
+        t.workspace = aligned
+        t.workspace_bytes = nbytes
+        self.table = t
+
+    # --- decoding -------------------------------------------------------
+    def decode(self, x, logits, stream=None, check=True) -> int:
+        return _w.wq4_decode_chain(self.table, x, logits, stream, check=check)
+
+    def decode_host(self, x_host: np.ndarray, logits_host: np.ndarray, stream=None) -> int:
+        return _w.wq4_decode_chain_host(self.table, x_host, logits_host, stream)
+
+    def destroy_plan(self) -> None:
+        _w.wq4_chain_plan_destroy(self.table)
+
+    # --- inspection -----------------------------------------------------
+    def trace(self, layer: int):
+        """fp16 bit arrays (numpy uint16 [batch][len]) of one layer's stages."""
+        off = _w.wq4_chain_trace_offsets(self.table, layer)
+        sh, B = self.shape, self.batch
+        lens = dict(x_in=sh.hidden, qkv=sh.n_qkv, o=sh.hidden, x_mid=sh.hidden,
+                    gate_up=2 * sh.ffn, act=sh.ffn, down=sh.hidden, x_out=sh.hidden)
+        out = {}
+        for name, n in lens.items():
+            o = getattr(off, name)
+            if layer == sh.num_layers and name != "x_in":
+                continue
+            o += self._ws_offset
+            buf = self.workspace[o:o + 2 * B * n]
+            out[name] = buf.cpu().numpy().view(np.uint16).reshape(B, n)
+        return out
+
+    def host_rows(self, layer: int, name: str, row_start: int, nrows: int):
+        """Rows of one projection regenerated on the host (uint32 W, uint16 s)."""
+        sh = self.shape
+        if name == "lm_head":
+            N, K, mat, lay = sh.vocab, sh.hidden, synth.MAT_LM_HEAD, sh.num_layers
+        else:
+            (N, K, mat), lay = [(N, K, m) for nm, N, K, m in sh.mats(layer) if nm == name][0], layer
+        return synth.matrix(self.seed, N, K, lay, mat, row_start, nrows)

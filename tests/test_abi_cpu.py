@@ -1,0 +1,136 @@
+"""The C ABI without a GPU: the library loads, exports every entry point its
+headers declare, and rejects bad arguments before touching the device."""
+import ctypes
+import os
+import re
+import subprocess
+
+import numpy as np
+import pytest
+
+import oracle
+from paper_2412_15803_gb300 import wq4
+
+ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
+
+
+def declared_functions():
+    names = set()
+    for h in ("wq4.h", "wq4_synth.h"):
+        text = open(os.path.join(ROOT, "include", h)).read()
+        text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
+        names |= set(re.findall(r"^[A-Za-z_][\w \*]*?\b(wq4_\w+)\s*\(", text, flags=re.M))
+    return names
+
+
+def test_exports_every_declared_symbol():
+    lib = wq4.load()
+    names = declared_functions()
+    assert len(names) >= 12
+    assert names == set(wq4.EXPORTED)
+    dyn = subprocess.run(["nm", "-D", "--defined-only", wq4.lib_path()], capture_output=True, text=True).stdout
+    for n in names:
+        assert hasattr(lib, n), n
+        assert re.search(rf"\bT {n}$", dyn, flags=re.M), n
+
+
+def test_status_strings():
+    assert wq4.wq4_status_string(0) == "ok"
+    assert "alignment" in wq4.wq4_status_string(-2) or "misaligned" in wq4.wq4_status_string(-2)
+    assert wq4.wq4_status_string(12345) == "unknown status"
+
+
+def test_pack_host_matches_oracle_and_rejects_bad_codes():
+    q = np.random.default_rng(0).integers(0, 16, size=(5, 64), dtype=np.uint8)
+    assert np.array_equal(wq4.wq4_pack_host(q), oracle.pack(q))
+    q[2, 3] = 16
+    with pytest.raises(wq4.Wq4Error):
+        wq4.wq4_pack_host(q)
+
+
+A16 = 1 << 20  # fake, 16-byte aligned "device" addresses: never dereferenced
+
+
+@pytest.mark.parametrize("args,expect", [
+    (dict(W=0), wq4.WQ4_ERR_INVALID),
+    (dict(x=0), wq4.WQ4_ERR_INVALID),
+    (dict(N=0), wq4.WQ4_ERR_INVALID),
+    (dict(K=48), wq4.WQ4_ERR_INVALID),
+    (dict(K=16), wq4.WQ4_ERR_INVALID),
+    (dict(batch=0), wq4.WQ4_ERR_INVALID),
+    (dict(batch=33), wq4.WQ4_ERR_INVALID),
+    (dict(W=A16 + 4), wq4.WQ4_ERR_ALIGN),
+    (dict(x=8 * A16 + 8), wq4.WQ4_ERR_ALIGN),
+    (dict(s=2 * A16 + 1), wq4.WQ4_ERR_ALIGN),
+    (dict(y=A16 + 64), wq4.WQ4_ERR_INVALID),   # y overlaps W
+])
+def test_gemv_rejects_bad_arguments(args, expect):
+    a = dict(W=A16, s=2 * A16, x=8 * A16, y=16 * A16, N=64, K=256, batch=1)
+    a.update(args)
+    rc = wq4.load().wq4_gemv(a["W"], a["s"], a["x"], a["y"], a["N"], a["K"], a["batch"], None)
+    assert rc == expect
+
+
+def test_unpack_debug_rejects_bad_arguments():
+    L = wq4.load()
+    assert L.wq4_unpack_debug(A16, 2 * A16, None, None, 4, 64, None) == wq4.WQ4_ERR_INVALID
+    assert L.wq4_unpack_debug(A16, 2 * A16, 4 * A16 + 2, None, 4, 64, None) == wq4.WQ4_ERR_ALIGN
+    assert L.wq4_unpack_debug(A16, 2 * A16, 4 * A16, None, 4, 40, None) == wq4.WQ4_ERR_INVALID
+
+
+def _table(**kw):
+    layers = (wq4.wq4_layer * 2)()
+    t = wq4.wq4_layer_table()
+    t.num_layers, t.hidden, t.ffn, t.n_q_heads, t.n_kv_heads, t.head_dim = 2, 256, 512, 2, 1, 128
+    t.vocab, t.batch, t.rms_eps = 1000, 1, 1e-5
+    t.layers = layers
+    for k, v in kw.items():
+        setattr(t, k, v)
+    return t, layers
+
+
+def test_chain_workspace_bytes_and_invalid_tables():
+    t, _ = _table()
+    n = wq4.wq4_chain_workspace_bytes(t)
+    assert n > 0 and n % 256 == 0
+    t4, _ = _table(batch=4)
+    assert wq4.wq4_chain_workspace_bytes(t4) > n
+    for bad in (dict(hidden=200), dict(ffn=100), dict(n_q_heads=3), dict(batch=0), dict(batch=33),
+                dict(vocab=0), dict(rms_eps=0.0), dict(num_layers=0)):
+        tb, _ = _table(**bad)
+        assert wq4.wq4_chain_workspace_bytes(tb) == 0, bad
+        assert wq4.load().wq4_decode_chain(ctypes.byref(tb), A16, 2 * A16, None) == wq4.WQ4_ERR_INVALID
+
+
+def test_chain_trace_offsets_are_disjoint_and_inside_workspace():
+    t, _ = _table(batch=2)
+    total = wq4.wq4_chain_workspace_bytes(t)
+    spans = []
+    lens = dict(x_in=256, qkv=512, o=256, x_mid=256, gate_up=1024, act=512, down=256, x_out=256)
+    for layer in range(2):
+        off = wq4.wq4_chain_trace_offsets(t, layer)
+        for name, n in lens.items():
+            o = getattr(off, name)
+            assert o % 2 == 0 and o + 2 * 2 * n <= total
+            spans.append((o, o + 4 * n))
+    spans.append((wq4.wq4_chain_trace_offsets(t, 2).x_in, wq4.wq4_chain_trace_offsets(t, 2).x_in + 4 * 256))
+    spans.sort()
+    for (a0, a1), (b0, b1) in zip(spans, spans[1:]):
+        assert a1 <= b0
+    with pytest.raises(wq4.Wq4Error):
+        wq4.wq4_chain_trace_offsets(t, 3)
+
+
+def test_chain_rejects_null_and_misaligned_io():
+    t, _ = _table()
+    L = wq4.load()
+    assert L.wq4_decode_chain(ctypes.byref(t), None, A16, None) == wq4.WQ4_ERR_INVALID
+    assert L.wq4_decode_chain(ctypes.byref(t), A16 + 8, 2 * A16, None) == wq4.WQ4_ERR_ALIGN
+    assert L.wq4_chain_plan_destroy(ctypes.byref(t)) == wq4.WQ4_ERR_INVALID
+
+
+def test_synth_rejects_bad_arguments():
+    L = wq4.load()
+    assert L.wq4_synth_codes(A16, 1, 4, 0, 0, None) == -1
+    assert L.wq4_synth_codes(A16, 0, 3, 0, 0, None) == -1
+    assert L.wq4_synth_scales(None, 0, 4, 0, 0, 0.005, 0.02, None) == -1

@@ -1,0 +1,186 @@
+"""GPU parity of the persistent decode chain, stage by stage.
+
+Each projection is compared with the oracle on the GPU's own fp16 input to
+that stage (read back from the workspace trace), with the GEMV tolerance;
+residual adds must be bit-exact; silu(gate) * up within one fp16 ulp of the
+fp64 value; the LM head like a projection.  End-to-end logits of the small
+model are compared with the oracle chain by relative L2 (information only).
+"""
+import numpy as np
+import pytest
+import torch
+
+import oracle
+from oracle import chain as ochain
+from paper_2412_15803_gb300 import synth
+from paper_2412_15803_gb300.model import SHAPE_3B, DecodeModel, ModelShape
+
+pytestmark = pytest.mark.gpu
+
+TINY = ModelShape("tiny", 3, 256, 512, 2, 1, 128, 1001)
+SMALL = ModelShape("small", 2, 1024, 2816 - 2816 % 256, 8, 2, 128, 4000)
+
+
+def within(gpu16, ref, A, what):
+    err = np.abs(oracle.half_to_double(gpu16) - ref)
+    tol = oracle.tolerance(ref, A)
+    bad = np.argwhere(~(err <= tol))
+    assert bad.size == 0, f"{what}: {len(bad)} out of tolerance, first {bad[:3]}"
+
+
+def run(model, x):
+    xd = torch.from_numpy(x.view(np.int16)).cuda()
+    logits = torch.empty((model.batch, model.shape.vocab), dtype=torch.int16, device="cuda")
+    model.decode(xd, logits)
+    torch.cuda.synchronize()
+    from paper_2412_15803_gb300 import wq4
+    assert wq4.wq4_device_status() == 0
+    return logits.cpu().numpy().view(np.uint16)
+
+
+def check_norm(v_gpu, u, eps, what):
+    """The re-fed input: fp16(r(u) u) with r in fp32 on the GPU, within one
+    fp16 ulp of the fp64 value."""
+    r = ochain.rms_factors(u, eps)
+    ref = r[:, None] * oracle.half_to_double(u)
+    err = np.abs(oracle.half_to_double(v_gpu) - ref)
+    assert np.all(err <= oracle.ulp16_array(np.abs(ref))), what
+
+
+def check_stages(model, layer, rows=None, u=None):
+    """Stage-wise parity of one layer; rows: None = all, else a dict name -> row
+    index array; u: the layer's raw input (None: the previous layer's output)."""
+    sh, eps = model.shape, model.eps
+    H, F = sh.hidden, sh.ffn
+    t = model.trace(layer)
+    if u is None:
+        u = model.trace(layer - 1)["x_out"]
+    check_norm(t["x_in"], u, eps, f"layer {layer} input normalisation")
+
+    def proj(name, inp, use_r, out, N):
+        r = ochain.rms_factors(inp, eps) if use_r else None
+        idx = np.arange(N) if rows is None else rows[name]
+        W, s = model.host_rows(layer, name, 0, N) if rows is None else _rows(model, layer, name, idx)
+        y, A, _ = oracle.gemv(W, s, inp, r)
+        within(out[:, idx], y, A, f"layer {layer} {name}")
+
+    proj("qkv", t["x_in"], False, t["qkv"], sh.n_qkv)
+    a = np.ascontiguousarray(t["qkv"][:, :H])
+    proj("o", a, True, t["o"], H)
+    assert np.array_equal(t["x_mid"], oracle.add_fp16(t["x_in"], t["o"]))
+    proj("gate_up", t["x_mid"], True, t["gate_up"], 2 * F)
+    m64, _ = oracle.silu_mul(np.ascontiguousarray(t["gate_up"][:, :F]), np.ascontiguousarray(t["gate_up"][:, F:]))
+    err = np.abs(oracle.half_to_double(t["act"]) - m64)
+    assert np.all(err <= oracle.ulp16_array(np.abs(m64))), f"layer {layer} act"
+    proj("down", t["act"], False, t["down"], H)
+    assert np.array_equal(t["x_out"], oracle.add_fp16(t["x_mid"], t["down"]))
+
+
+def _rows(model, layer, name, idx):
+    Ws, ss = [], []
+    for i in idx:
+        W, s = model.host_rows(layer, name, int(i), 1)
+        Ws.append(W)
+        ss.append(s)
+    return np.concatenate(Ws), np.concatenate(ss)
+
+
+def check_logits(model, logits, rows=None):
+    sh = model.shape
+    xin = model.trace(sh.num_layers)["x_in"]
+    check_norm(xin, model.trace(sh.num_layers - 1)["x_out"], model.eps, "LM head input normalisation")
+    r = None
+    if rows is None:
+        W, s = model.host_rows(sh.num_layers, "lm_head", 0, sh.vocab)
+        idx = np.arange(sh.vocab)
+    else:
+        idx = rows
+        W, s = _rows(model, sh.num_layers, "lm_head", idx)
+    y, A, _ = oracle.gemv(W, s, xin, r)
+    within(logits[:, idx], y, A, "lm_head")
+
+
+@pytest.mark.parametrize("batch", [1, 2, 3, 4])
+def test_tiny_chain_every_stage_every_element(batch):
+    model = DecodeModel(TINY, batch=batch, seed=batch)
+    x = synth.activations(100 + batch, batch, TINY.hidden)
+    logits = run(model, x)
+    for l in range(TINY.num_layers):
+        check_stages(model, l, u=x if l == 0 else None)
+    check_logits(model, logits)
+    # end to end against the oracle chain (information: fp16 stage roundings may differ)
+    layers = [{n: model.host_rows(l, n, 0, N) for n, N, _, _ in TINY.mats(l)} for l in range(TINY.num_layers)]
+    lm = model.host_rows(TINY.num_layers, "lm_head", 0, TINY.vocab)
+    ref16, ref, _ = ochain.token(x, layers, lm, TINY.hidden, TINY.ffn, model.eps)
+    g = oracle.half_to_double(logits)
+    rel = np.linalg.norm(g - ref) / np.linalg.norm(ref)
+    assert rel < 2e-2, rel
+
+
+def test_tiny_chain_repeat_and_host_variant():
+    model = DecodeModel(TINY, batch=2, seed=9)
+    x = synth.activations(7, 2, TINY.hidden)
+    a = run(model, x)
+    tr_a = model.trace(1)
+    b = run(model, x)
+    assert np.array_equal(a, b)
+    tr_b = model.trace(1)
+    for k in tr_a:
+        assert np.array_equal(tr_a[k], tr_b[k])
+    lh = np.zeros((2, TINY.vocab), np.uint16)
+    model.decode_host(np.ascontiguousarray(x), lh)
+    assert np.array_equal(lh, a)
+    # a new input after the plan exists
+    x2 = synth.activations(8, 2, TINY.hidden)
+    c = run(model, x2)
+    assert not np.array_equal(c, a)
+    for l in range(TINY.num_layers):
+        check_stages(model, l, u=x2 if l == 0 else None)
+
+
+def test_small_chain_ragged_items():
+    """Non-power-of-two FFN and a vocab that is not a multiple of the item size."""
+    model = DecodeModel(SMALL, batch=1, seed=4)
+    x = synth.activations(44, 1, SMALL.hidden)
+    logits = run(model, x)
+    for l in range(SMALL.num_layers):
+        check_stages(model, l, u=x if l == 0 else None)
+    check_logits(model, logits)
+
+
+def test_plan_rebuilds_when_table_changes():
+    model = DecodeModel(TINY, batch=1, seed=3)
+    x = synth.activations(1, 1, TINY.hidden)
+    a = run(model, x)
+    other = DecodeModel(TINY, batch=1, seed=12)
+    # point layer 1's down projection at another model's weights
+    model._layers[1].down = other._layers[1].down
+    model.weights[1]["down"] = other.weights[1]["down"]
+    b = run(model, x)
+    assert not np.array_equal(a, b)
+    t = model.trace(1)
+    W, s = other.host_rows(1, "down", 0, TINY.hidden)
+    y, A, _ = oracle.gemv(W, s, t["act"])
+    within(t["down"], y, A, "rebuilt plan down")
+    model.destroy_plan()
+
+
+def test_3b_chain_full_size_sampled():
+    """The 28-layer 3B-shaped chain at batch 1, as the benchmark runs it:
+    sampled rows of every projection of three layers, and of the LM head."""
+    model = DecodeModel(SHAPE_3B, batch=1, seed=0)
+    x = synth.activations(0, 1, SHAPE_3B.hidden)
+    logits = run(model, x)
+    rng = np.random.default_rng(0)
+    sh = SHAPE_3B
+
+    def pick(N):
+        return np.unique(np.concatenate([[0, 1, N - 2, N - 1], rng.integers(0, N, 24)]))
+
+    for l in (0, 13, 27):
+        rows = dict(qkv=pick(sh.n_qkv), o=pick(sh.hidden), gate_up=pick(2 * sh.ffn), down=pick(sh.hidden))
+        check_stages(model, l, rows, u=x if l == 0 else None)
+    check_logits(model, logits, rows=pick(sh.vocab))
+    # the whole output is finite and the chain is deterministic
+    assert np.all(np.isfinite(oracle.half_to_double(logits)))
+    assert np.array_equal(run(model, x), logits)

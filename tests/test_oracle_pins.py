@@ -270,7 +270,22 @@ def _identity_like(N, K, value_code=8, scale=0x3C00):
     return oracle.pack(q), np.full((N, K // 32), scale, np.uint16)
 
 
-def test_chain_all_sevens_is_residual_identity():
+def test_rms_normalize_closed_forms():
+    eps = 1e-5
+    c = np.full(64, 0x4200, np.uint16)                      # 3.0
+    v = oracle.rms_normalize(c, eps).view(np.float16).astype(np.float64)
+    assert np.all(v == np.float16(3.0 / math.sqrt(9.0 + eps)))
+    u = np.array([3.0, 4.0]).astype(np.float16).view(np.uint16)
+    v = oracle.rms_normalize(u, 0.0).view(np.float16).astype(np.float64)[0]
+    assert list(v) == [np.float16(3 / math.sqrt(12.5)), np.float16(4 / math.sqrt(12.5))]
+    assert np.all(oracle.rms_normalize(np.zeros(8, np.uint16), 1.0) == 0)
+    # rows are normalised independently
+    two = np.stack([c, np.full(64, 0x4400, np.uint16)])  # rows of 3.0 and 4.0
+    out = oracle.rms_normalize(two, 0.0).view(np.float16).astype(np.float64)
+    assert np.all(out == 1.0)
+
+
+def test_chain_all_sevens_passes_the_normalised_input_through():
     H, F, V, Nqkv, L, batch, eps = 64, 96, 80, 128, 3, 2, 1e-5
     rnd = lambda N, K: (oracle.pack(np.full((N, K), 7, np.uint8)),
                         synth.scales_fp16(2, N * K, 0, N * K // 32).reshape(N, K // 32))
@@ -279,8 +294,10 @@ def test_chain_all_sevens_is_residual_identity():
     x = synth.activations(7, batch, H)
     logits, y, tr = ochain.token(x, layers, rnd(V, H), H, F, eps)
     assert np.all(y == 0.0)
-    for t in tr:
-        assert np.array_equal(t["x2"], x)
+    assert np.array_equal(tr[0]["v"], oracle.rms_normalize(x, eps))
+    for t in tr[:-1]:
+        assert np.all(t["qkv"] & 0x7FFF == 0) and np.all(t["d"] & 0x7FFF == 0)
+        assert np.array_equal(t["x2"], t["v"])          # o = d = 0: output = layer input
 
 
 def test_chain_wiring_with_identity_projections():
@@ -288,13 +305,12 @@ def test_chain_wiring_with_identity_projections():
     values follow from the stage definitions with numpy fp16 rounding."""
     H, F, batch, eps = 64, 64, 1, 1e-5
     Nqkv = 2 * H
-    layers = [dict(qkv=_identity_like(Nqkv, H), o=_identity_like(H, H),
-                   gate_up=_identity_like(2 * F, H), down=_identity_like(H, F))]
-    # gate_up: rows [0, F) and [F, 2F) both copy the input
     qg = np.full((2 * F, H), 7, np.uint8)
-    qg[np.arange(F), np.arange(F)] = 8
-    qg[F + np.arange(F), np.arange(F)] = 8
-    layers[0]["gate_up"] = (oracle.pack(qg), np.full((2 * F, H // 32), 0x3C00, np.uint16))
+    qg[np.arange(F), np.arange(F)] = 8        # gate rows copy the input
+    qg[F + np.arange(F), np.arange(F)] = 8    # up rows copy it too
+    layers = [dict(qkv=_identity_like(Nqkv, H), o=_identity_like(H, H),
+                   gate_up=(oracle.pack(qg), np.full((2 * F, H // 32), 0x3C00, np.uint16)),
+                   down=_identity_like(H, F))]
     lm = _identity_like(H, H)
     x = synth.activations(11, batch, H)
     logits, y, tr = ochain.token(x, layers, lm, H, F, eps)
@@ -302,22 +318,22 @@ def test_chain_wiring_with_identity_projections():
     f16 = lambda v: np.asarray(v, np.float64).astype(np.float16).astype(np.float64)
     xv = x.view(np.float16).astype(np.float64)[0]
     r = lambda v: 1.0 / np.sqrt(np.mean(v * v) + eps)
-    qkv = f16(r(xv) * xv)                       # first H rows copy rms(x)
-    a = qkv
-    o = f16(r(a) * a)
-    x1 = f16(xv + o)
+    v = f16(r(xv) * xv)                         # layer input after normalisation
+    qkv = v                                     # first H rows copy v
+    o = f16(r(qkv) * qkv)
+    x1 = f16(v + o)
     g = f16(r(x1) * x1)
     m = f16(g / (1.0 + np.exp(-g)) * g)
-    d = f16(m)
-    x2 = f16(x1 + d)
+    x2 = f16(x1 + m)
     lg = f16(r(x2) * x2)
     t = tr[0]
     h64 = lambda b: b.view(np.float16).astype(np.float64)[0]
-    assert np.array_equal(h64(t["qkv"])[:H], qkv) and np.all(h64(t["qkv"])[H:] == 0)
-    assert np.array_equal(h64(t["o"]), o)
-    assert np.array_equal(h64(t["x1"]), x1)
-    assert np.array_equal(h64(t["gu"]), np.concatenate([g, g]))
-    assert np.allclose(h64(t["m"]), m, rtol=2.0 ** -10, atol=2.0 ** -24)
+    assert np.allclose(h64(t["v"]), v, rtol=2.0 ** -10, atol=0)
+    assert np.array_equal(h64(t["qkv"])[:H], h64(t["v"])) and np.all(h64(t["qkv"])[H:] == 0)
+    assert np.allclose(h64(t["o"]), o, rtol=2.0 ** -9, atol=2.0 ** -24)
+    assert np.array_equal(h64(t["x1"]), f16(h64(t["v"]) + h64(t["o"])))
+    assert np.allclose(h64(t["gu"]), np.concatenate([g, g]), rtol=2.0 ** -9, atol=2.0 ** -24)
+    assert np.allclose(h64(t["m"]), m, rtol=2.0 ** -8, atol=2.0 ** -24)
     assert np.array_equal(h64(t["d"]), h64(t["m"]))
-    assert np.allclose(h64(t["x2"]), x2, rtol=2.0 ** -9, atol=2.0 ** -20)
-    assert np.allclose(logits.view(np.float16).astype(np.float64)[0], lg, rtol=2.0 ** -9, atol=2.0 ** -20)
+    assert np.array_equal(h64(t["x2"]), f16(h64(t["x1"]) + h64(t["d"])))
+    assert np.allclose(logits.view(np.float16).astype(np.float64)[0], lg, rtol=2.0 ** -8, atol=2.0 ** -24)

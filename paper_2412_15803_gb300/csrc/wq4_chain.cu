@@ -687,12 +687,15 @@ int build_plan(const wq4_layer_table* t, Plan* pl, cudaStream_t stream)
     if (nslots < 2) return WQ4_ERR_UNSUPPORTED;
     if (nslots > kChainMaxSlots) nslots = kChainMaxSlots;
     const size_t smem = kChainHeader + x_bytes + static_cast<size_t>(nslots) * slot_bytes;
+    // The limit is a property of the kernel, shared by every plan: set it to
+    // the device maximum so that no plan's launch depends on which plan was
+    // built last.
     cudaError_t e = cudaSuccess;
     switch (d.B) {
-        case 1: e = set_chain_attr<1>(static_cast<int>(smem)); break;
-        case 2: e = set_chain_attr<2>(static_cast<int>(smem)); break;
-        case 3: e = set_chain_attr<3>(static_cast<int>(smem)); break;
-        default: e = set_chain_attr<4>(static_cast<int>(smem)); break;
+        case 1: e = set_chain_attr<1>(di->smem_optin); break;
+        case 2: e = set_chain_attr<2>(di->smem_optin); break;
+        case 3: e = set_chain_attr<3>(di->smem_optin); break;
+        default: e = set_chain_attr<4>(di->smem_optin); break;
     }
     if (e != cudaSuccess) return WQ4_ERR_CUDA;
 

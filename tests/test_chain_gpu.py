@@ -184,3 +184,17 @@ def test_3b_chain_full_size_sampled():
     # the whole output is finite and the chain is deterministic
     assert np.all(np.isfinite(oracle.half_to_double(logits)))
     assert np.array_equal(run(model, x), logits)
+
+
+def test_two_models_with_different_rings_alternate():
+    """Plans of different shapes (different shared-memory rings) stay valid
+    whichever plan was built last."""
+    a = DecodeModel(TINY, batch=1, seed=41)
+    b = DecodeModel(SMALL, batch=1, seed=42)
+    xa = synth.activations(71, 1, TINY.hidden)
+    xb = synth.activations(72, 1, SMALL.hidden)
+    la = run(a, xa)
+    lb = run(b, xb)
+    assert np.array_equal(run(a, xa), la)
+    assert np.array_equal(run(b, xb), lb)
+    check_logits(a, la)

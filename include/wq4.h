@@ -186,6 +186,38 @@ int wq4_decode_chain(const wq4_layer_table* table, const uint16_t* x,
 int wq4_decode_chain_host(const wq4_layer_table* table, const uint16_t* x_host,
                           uint16_t* logits_host, void* stream);
 
+/*
+ * Size of the device array wq4_decode_chain_noalloc uses as its workspace
+ * (16 MiB: the 3B-shaped chain at batch 1-2, the 8B-shaped one at batch 1).
+ */
+#define WQ4_NOALLOC_SCRATCH_BYTES (16u << 20)
+
+/*
+ * wq4_decode_chain without a caller-allocated workspace.  The paper has no
+ * counterpart: this is for callers that cannot call cudaMalloc -- a plug-in
+ * inside a host framework that owns all device memory through its own pool
+ * and permits no other allocation, or a latency-critical loop where
+ * cudaMalloc's implicit device synchronization is not acceptable.
+ *
+ * The workspace is a fixed device array of WQ4_NOALLOC_SCRATCH_BYTES inside
+ * this library: every GPU that loads the library holds it until the process
+ * exits.  table->workspace and table->workspace_bytes are ignored; everything
+ * else, x and logits are as for wq4_decode_chain.  The call allocates no
+ * device memory (no cudaMalloc, cudaFree or allocating library routine).
+ *   - The first call on a device looks up the array's device address
+ *     (cudaGetSymbolAddress, with that device current); make that first call
+ *     before any stream capture.
+ *   - All calls on a device share the one array, which keeps the last call's
+ *     contents; the first call for a table, or a call with a different table
+ *     than the previous one, clears the array's counters and flags again.
+ *     Calls that overlap on the GPU race on the array: serialize them.
+ *   - A table whose wq4_chain_workspace_bytes exceeds
+ *     WQ4_NOALLOC_SCRATCH_BYTES is rejected with WQ4_ERR_UNSUPPORTED before
+ *     anything is enqueued.
+ */
+int wq4_decode_chain_noalloc(const wq4_layer_table* table, const uint16_t* x,
+                             uint16_t* logits, void* stream);
+
 /* Releases the cached plan of `table` (host-side state only; the workspace
  * stays the caller's).  Returns WQ4_ERR_INVALID if no plan exists. */
 int wq4_chain_plan_destroy(const wq4_layer_table* table);

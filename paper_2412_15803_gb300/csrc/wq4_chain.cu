@@ -879,3 +879,66 @@ extern "C" int wq4_chain_trace_offsets(const wq4_layer_table* table, int layer, 
     out->x_out = y.pX2 + 2 * l * B * H;
     return WQ4_OK;
 }
+
+// ------------------------------------------------- allocation-free variant --
+//
+// wq4_decode_chain_noalloc: the same persistent chain kernel, with its
+// workspace in a fixed device array of this library instead of a buffer the
+// caller allocates.  For callers that cannot call cudaMalloc themselves.
+
+namespace wq4 {
+namespace {
+
+constexpr size_t kNoAllocScratchBytes = static_cast<size_t>(WQ4_NOALLOC_SCRATCH_BYTES);
+constexpr int kNoAllocMaxDevices = 64;
+
+// Every device that loads the library holds this array until the process
+// exits.  Host code may not use its name as an address: the address comes
+// from cudaGetSymbolAddress, once per device.
+static __device__ __align__(256) uint8_t g_noalloc_scratch[kNoAllocScratchBytes];
+
+struct NoAllocDevice {
+    bool ready = false;
+    void* scratch = nullptr;          // device address of g_noalloc_scratch
+    wq4_layer_table table = {};       // the caller's table, pointed at the scratch
+};
+
+NoAllocDevice g_noalloc[kNoAllocMaxDevices];
+std::mutex g_noalloc_mu;
+
+}  // namespace
+}  // namespace wq4
+
+extern "C" int wq4_decode_chain_noalloc(const wq4_layer_table* table, const uint16_t* x, uint16_t* logits,
+                                        void* stream)
+{
+    if (!table || !x || !logits) return WQ4_ERR_INVALID;
+    if (!aligned(x, 16) || !aligned(logits, 2)) return WQ4_ERR_ALIGN;
+    Dims d;
+    if (!table_dims(table, &d)) return WQ4_ERR_INVALID;
+    if (make_layout(d).total > kNoAllocScratchBytes) return WQ4_ERR_UNSUPPORTED;
+    int dev = 0;
+    if (cudaGetDevice(&dev) != cudaSuccess) return WQ4_ERR_CUDA;
+    if (dev < 0 || dev >= kNoAllocMaxDevices) return WQ4_ERR_UNSUPPORTED;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    std::lock_guard<std::mutex> lock(g_noalloc_mu);
+    NoAllocDevice& nd = g_noalloc[dev];
+    if (!nd.ready) {
+        void* p = nullptr;
+        if (cudaGetSymbolAddress(&p, g_noalloc_scratch) != cudaSuccess || p == nullptr) return WQ4_ERR_CUDA;
+        nd.scratch = p;
+        nd.ready = true;
+    }
+    // One table object per device stands for "whoever uses the array now":
+    // a call with another model changes its contents, so the cached plan is
+    // rebuilt and the array's flags and counters are cleared again.
+    nd.table = *table;
+    nd.table.workspace = nd.scratch;
+    nd.table.workspace_bytes = kNoAllocScratchBytes;
+    Plan pl;
+    const int rc = get_plan(&nd.table, &pl, st);
+    if (rc != WQ4_OK) return rc;
+    const size_t lb = static_cast<size_t>(pl.dims.B) * pl.dims.V * 2;
+    if (overlaps(logits, lb, x, static_cast<size_t>(pl.dims.B) * pl.dims.H * 2)) return WQ4_ERR_INVALID;
+    return launch_chain(pl, x, logits, st);
+}

@@ -82,6 +82,7 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
     L.wq4_chain_workspace_bytes.restype = _SZ
     L.wq4_decode_chain.argtypes = [ctypes.POINTER(wq4_layer_table), _P, _P, _P]
     L.wq4_decode_chain_host.argtypes = [ctypes.POINTER(wq4_layer_table), _P, _P, _P]
+    L.wq4_decode_chain_noalloc.argtypes = [ctypes.POINTER(wq4_layer_table), _P, _P, _P]
     L.wq4_chain_plan_destroy.argtypes = [ctypes.POINTER(wq4_layer_table)]
     L.wq4_chain_trace_offsets.argtypes = [ctypes.POINTER(wq4_layer_table), _I,
                                           ctypes.POINTER(wq4_chain_trace)]
@@ -94,7 +95,7 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
 # names every C entry point of include/*.h (checked by the tests)
 EXPORTED = ["wq4_gemv", "wq4_unpack_debug", "wq4_pack_host", "wq4_status_string",
             "wq4_device_status", "wq4_chain_workspace_bytes", "wq4_decode_chain",
-            "wq4_decode_chain_host", "wq4_chain_plan_destroy", "wq4_chain_trace_offsets",
+            "wq4_decode_chain_host", "wq4_decode_chain_noalloc", "wq4_chain_plan_destroy", "wq4_chain_trace_offsets",
             "wq4_synth_codes", "wq4_synth_scales"]
 
 
@@ -168,6 +169,11 @@ def wq4_decode_chain(table: wq4_layer_table, x, logits, stream=None, check: bool
 def wq4_decode_chain_host(table: wq4_layer_table, x_host, logits_host, stream=None, check: bool = True) -> int:
     rc = load().wq4_decode_chain_host(ctypes.byref(table), _ptr(x_host), _ptr(logits_host), _stream(stream))
     return _check("wq4_decode_chain_host", rc) if check else rc
+
+
+def wq4_decode_chain_noalloc(table: wq4_layer_table, x, logits, stream=None, check: bool = True) -> int:
+    rc = load().wq4_decode_chain_noalloc(ctypes.byref(table), _ptr(x), _ptr(logits), _stream(stream))
+    return _check("wq4_decode_chain_noalloc", rc) if check else rc
 
 
 def wq4_chain_plan_destroy(table: wq4_layer_table) -> int:

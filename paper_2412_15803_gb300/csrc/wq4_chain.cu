@@ -42,11 +42,23 @@
 namespace wq4 {
 namespace {
 
-constexpr int kNW = 8;                       // consumer warps
-constexpr int kChainThreads = (kNW + 1) * 32;
 constexpr int kChainMaxSlots = 32;
-constexpr int kChainHeader = 1024;           // mbarriers, reductions, scalars
 constexpr int kMaxChainBatch = 4;
+// Shared-memory header: mbarriers | RMS partial sums | epoch | the residual
+// words of the CTA's rows (O and down stages); then the staged input vector,
+// then the weight ring.
+constexpr int kHdrRed = 512;                 // float red[16][kMaxChainBatch]
+constexpr int kHdrEpoch = 768;
+constexpr int kHdrRes = 1024;                // uint32 res[kMaxResWords]: prefetched residual words
+constexpr int kMaxResWords = 1024;
+constexpr int kChainHeader = kHdrRes + 4 * kMaxResWords;
+
+// Consumer warps per CTA: with the producer warp, 16 warps (128 registers a
+// thread) for batch 1-2, 8 warps (255 registers) for batch 3-4.
+template <int B>
+struct ChainWarps {
+    static constexpr int NW = (B <= 2) ? 15 : 7;
+};
 
 enum StageType { kQKV = 0, kO = 1, kGU = 2, kDOWN = 3, kLM = 4 };
 
@@ -255,16 +267,137 @@ __device__ __forceinline__ float sum8_sq(uint4 v)
 
 // ---------------------------------------------------------- the kernel --
 
+// One group (32 codes) of every row of an item against the staged
+// activations.  crow/srow point at the lane's first group of each row, xl at
+// the lane's first group of activation row 0; `off` is the group offset
+// (a multiple of 32, so the lane's chunk swizzle `sw` does not change).  The
+// activations are loaded once and used for every row; each row's 32 products
+// go into two 16-long fp32 chains before the group's scale is applied.
+template <int B, int RPI>
+__device__ __forceinline__ void group_rows_dot(const uint4* const crow[4], const uint16_t* const srow[4],
+                                               const uint4* xl, int cpr, int sw, int off, float acc[4][B])
+{
+    uint4 xv[B][4];
+#pragma unroll
+    for (int b = 0; b < B; ++b)
+#pragma unroll
+        for (int j = 0; j < 4; ++j) xv[b][j] = xl[b * cpr + 4 * off + (j ^ sw)];
+#pragma unroll
+    for (int r = 0; r < RPI; ++r) {
+        const uint4 cw = crow[r][off];
+        const float sc = half_bits_to_float(srow[r][off]);
+        uint32_t q[16];
+        unpack_word(cw.x, q + 0);
+        unpack_word(cw.y, q + 4);
+        unpack_word(cw.z, q + 8);
+        unpack_word(cw.w, q + 12);
+#pragma unroll
+        for (int b = 0; b < B; ++b) {
+            const float a01 = fma8(q + 4, xv[b][1], fma8(q + 0, xv[b][0], 0.f));
+            const float a23 = fma8(q + 12, xv[b][3], fma8(q + 8, xv[b][2], 0.f));
+            acc[r][b] = fmaf(sc, a01 + a23, acc[r][b]);
+        }
+    }
+}
+
+// Every group of the item's rows: lane l takes groups l + 32 i.  Rows of 32,
+// 64, 96, 128 or 256 groups run fully unrolled (all loads of the item can be
+// issued ahead of its arithmetic); other lengths take a loop and a tail.
+template <int B, int RPI>
+__device__ __forceinline__ void item_dot(const uint4* const crow[4], const uint16_t* const srow[4],
+                                         const uint4* xl, int cpr, int gpr, int lane, float acc[4][B])
+{
+    const int sw = (lane >> 1) & 3;
+    switch (gpr) {
+        case 32: group_rows_dot<B, RPI>(crow, srow, xl, cpr, sw, 0, acc); return;
+        case 64:
+#pragma unroll
+            for (int i = 0; i < 2; ++i) group_rows_dot<B, RPI>(crow, srow, xl, cpr, sw, 32 * i, acc);
+            return;
+        case 96:
+#pragma unroll
+            for (int i = 0; i < 3; ++i) group_rows_dot<B, RPI>(crow, srow, xl, cpr, sw, 32 * i, acc);
+            return;
+        case 128:
+#pragma unroll
+            for (int i = 0; i < 4; ++i) group_rows_dot<B, RPI>(crow, srow, xl, cpr, sw, 32 * i, acc);
+            return;
+        case 256:
+#pragma unroll
+            for (int i = 0; i < 8; ++i) group_rows_dot<B, RPI>(crow, srow, xl, cpr, sw, 32 * i, acc);
+            return;
+        default: {
+            const int full = gpr >> 5;
+#pragma unroll 2
+            for (int i = 0; i < full; ++i) group_rows_dot<B, RPI>(crow, srow, xl, cpr, sw, 32 * i, acc);
+            if (lane < (gpr & 31)) group_rows_dot<B, RPI>(crow, srow, xl, cpr, sw, 32 * full, acc);
+        }
+    }
+}
+
+// Fused epilogue of one item for batch row b: v0..v3 are the item's row sums
+// (rows 2it, 2it+1; for gate_up gate 2it, 2it+1 then up 2it, 2it+1); resw is
+// the item's residual word (O: the normalised layer input, down: x + o).
 template <int B>
-__global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const ChainParams p)
+__device__ __forceinline__ void item_epilogue(const ChainParams& p, const Stage& g, int it, int b, float v0,
+                                              float v1, float v2, float v3, float rf, uint32_t resw, uint32_t epoch)
+{
+    const int H = p.H, F = p.F, l = g.layer;
+    const int n = 2 * it;
+    if (g.type == kQKV) {
+        const uint32_t w = pack2(float_to_half_bits(rf * v0), float_to_half_bits(rf * v1));
+        *reinterpret_cast<uint32_t*>(p.pQKV + (static_cast<size_t>(l) * B + b) * p.Nqkv + n) = w;
+        if (n < H) ll_store(p.llA + (static_cast<size_t>(l) * B + b) * (H / 2) + n / 2, w, epoch);
+    } else if (g.type == kO) {
+        const uint16_t o0 = float_to_half_bits(rf * v0);
+        const uint16_t o1 = float_to_half_bits(rf * v1);
+        const uint32_t x1 = pack2(add_h(lo_f(resw), half_bits_to_float(o0)), add_h(hi_f(resw), half_bits_to_float(o1)));
+        const size_t off = (static_cast<size_t>(l) * B + b) * H + n;
+        *reinterpret_cast<uint32_t*>(p.pO + off) = pack2(o0, o1);
+        *reinterpret_cast<uint32_t*>(p.pX1 + off) = x1;
+        ll_store(p.llX1 + (static_cast<size_t>(l) * B + b) * (H / 2) + n / 2, x1, epoch);
+    } else if (g.type == kGU) {
+        const int j = n;  // gate rows j, j+1 and up rows F+j, F+j+1
+        const uint16_t g0 = float_to_half_bits(rf * v0);
+        const uint16_t g1 = float_to_half_bits(rf * v1);
+        const uint16_t u0 = float_to_half_bits(rf * v2);
+        const uint16_t u1 = float_to_half_bits(rf * v3);
+        const float gf0 = half_bits_to_float(g0), gf1 = half_bits_to_float(g1);
+        const uint16_t m0 = float_to_half_bits(gf0 / (1.f + expf(-gf0)) * half_bits_to_float(u0));
+        const uint16_t m1 = float_to_half_bits(gf1 / (1.f + expf(-gf1)) * half_bits_to_float(u1));
+        const size_t gu = (static_cast<size_t>(l) * B + b) * (2 * F);
+        *reinterpret_cast<uint32_t*>(p.pGU + gu + j) = pack2(g0, g1);
+        *reinterpret_cast<uint32_t*>(p.pGU + gu + F + j) = pack2(u0, u1);
+        const uint32_t mw = pack2(m0, m1);
+        *reinterpret_cast<uint32_t*>(p.pM + (static_cast<size_t>(l) * B + b) * F + j) = mw;
+        ll_store(p.llM + (static_cast<size_t>(l) * B + b) * (F / 2) + j / 2, mw, epoch);
+    } else if (g.type == kDOWN) {
+        const uint16_t d0 = float_to_half_bits(v0);
+        const uint16_t d1 = float_to_half_bits(v1);
+        const uint32_t x2 = pack2(add_h(lo_f(resw), half_bits_to_float(d0)), add_h(hi_f(resw), half_bits_to_float(d1)));
+        *reinterpret_cast<uint32_t*>(p.pD + (static_cast<size_t>(l) * B + b) * H + n) = pack2(d0, d1);
+        *reinterpret_cast<uint32_t*>(p.pX2 + (static_cast<size_t>(l) * B + b) * H + n) = x2;
+        ll_store(p.llX + (static_cast<size_t>(l + 1) * B + b) * (H / 2) + n / 2, x2, epoch);
+    } else {
+        uint16_t* out = p.logits + static_cast<size_t>(b) * p.V;
+        out[n] = float_to_half_bits(rf * v0);
+        if (n + 1 < p.V) out[n + 1] = float_to_half_bits(rf * v1);
+    }
+}
+
+template <int B, int NW>
+__global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainParams p)
 {
     extern __shared__ __align__(1024) uint8_t smem[];
     uint64_t* full = reinterpret_cast<uint64_t*>(smem);
     uint64_t* empty = full + kChainMaxSlots;
-    float* red = reinterpret_cast<float*>(smem + 2 * kChainMaxSlots * 8);   // [kNW][B]
-    uint32_t* epoch_sh = reinterpret_cast<uint32_t*>(smem + 2 * kChainMaxSlots * 8 + kNW * kMaxChainBatch * 4);
+    float* red = reinterpret_cast<float*>(smem + kHdrRed);          // [NW][kMaxChainBatch]
+    uint32_t* epoch_sh = reinterpret_cast<uint32_t*>(smem + kHdrEpoch);
+    uint32_t* res = reinterpret_cast<uint32_t*>(smem + kHdrRes);    // [B][items of the CTA]
     uint4* xs = reinterpret_cast<uint4*>(smem + kChainHeader);
     uint8_t* slots = smem + kChainHeader + p.x_bytes;
+    constexpr int kConsumers = NW * 32;
+    constexpr int kPoll = 2;     // input chunks a thread has in flight at once
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nstages = 4 * p.L + 1;
@@ -272,7 +405,7 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const ChainPara
     if (threadIdx.x == 0) {
         for (int i = 0; i < p.nslots; ++i) {
             mbar_init(&full[i], 1);
-            mbar_init(&empty[i], kNW);
+            mbar_init(&empty[i], NW);
         }
         mbar_fence_init();
         uint32_t s;
@@ -282,7 +415,7 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const ChainPara
     __syncthreads();
     const uint32_t epoch = *epoch_sh;
 
-    if (warp == kNW) {
+    if (warp == NW) {
         // ------------------------------------------------ producer warp
         if (lane == 0) {
             const uint64_t pol = l2_policy_evict_first();
@@ -320,7 +453,8 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const ChainPara
     } else {
         // ------------------------------------------------ consumer warps
         const int H = p.H, F = p.F;
-        int ord = 0;
+        int cslot = 0;          // ring slot of the next chunk
+        uint32_t cpar = 0;      // phase parity of that slot's full barrier
         for (int st = 0; st < nstages; ++st) {
             const Stage g = stage_at(p, st);
             int i0, i1;
@@ -328,9 +462,11 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const ChainPara
             if (i1 <= i0) continue;
             const int l = g.layer;
             const int K = g.K, gpr = K >> 5, cpr = K >> 3;
+            const int nit = i1 - i0;
 
-            // -- stage the input vector (all consumer warps) and its RMS factor
-            named_barrier_sync(1, kNW * 32);   // every warp is done with the previous xs
+            // -- stage the input vector (all consumer warps), its RMS factor and
+            //    the residual words of the CTA's rows
+            named_barrier_sync(1, kConsumers);   // every warp is done with the previous xs and res
             {
                 const uint64_t* ll = nullptr;
                 const bool plain = (g.type == kQKV && l == 0);
@@ -339,21 +475,68 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const ChainPara
                 else if (g.type == kGU) ll = p.llX1 + static_cast<size_t>(l) * B * (H / 2);
                 else if (g.type == kDOWN) ll = p.llM + static_cast<size_t>(l) * B * (F / 2);
                 else ll = p.llX + static_cast<size_t>(p.L) * B * (H / 2);
+                const uint64_t* rl = nullptr;
+                if (g.type == kO) rl = p.llV + static_cast<size_t>(l) * B * (H / 2);
+                else if (g.type == kDOWN) rl = p.llX1 + static_cast<size_t>(l) * B * (H / 2);
+                if (rl) {
+                    for (int t = threadIdx.x; t < B * nit; t += kConsumers) {
+                        const int b = t / nit, k = t - b * nit;
+                        res[t] = ll_load(rl + static_cast<size_t>(b) * (H / 2) + i0 + k, epoch, p.err, p.abort);
+                    }
+                }
                 float ss[B];
 #pragma unroll
                 for (int b = 0; b < B; ++b) ss[b] = 0.f;
-                for (int i = threadIdx.x; i < B * cpr; i += kNW * 32) {
-                    const int b = i / cpr, c = i - b * cpr;
-                    uint4 v;
+                const int total = B * cpr;
+                for (int ib = threadIdx.x; ib < total; ib += kPoll * kConsumers) {
+                    uint4 v[kPoll];
                     if (plain) {
-                        v = reinterpret_cast<const uint4*>(p.x)[i];
-                    } else {
-                        v = ll_load4(ll + static_cast<size_t>(b) * (K / 2) + 4 * c, epoch, p.err, p.abort);
-                    }
-                    xs[b * cpr + x_chunk(c >> 2, c & 3)] = v;
 #pragma unroll
-                    for (int bb = 0; bb < B; ++bb)
-                        if (bb == b) ss[bb] += sum8_sq(v);
+                        for (int k = 0; k < kPoll; ++k) {
+                            const int i = ib + k * kConsumers;
+                            if (i < total) v[k] = reinterpret_cast<const uint4*>(p.x)[i];
+                        }
+                    } else {
+                        // issue every load first, then wait for the ones not yet published
+                        uint64_t w[kPoll][4];
+#pragma unroll
+                        for (int k = 0; k < kPoll; ++k) {
+                            const int i = ib + k * kConsumers;
+                            if (i < total) {
+                                const int b = i / cpr, c = i - b * cpr;
+                                const uint64_t* a = ll + static_cast<size_t>(b) * (K / 2) + 4 * c;
+                                ll_load2_raw(a, w[k][0], w[k][1]);
+                                ll_load2_raw(a + 2, w[k][2], w[k][3]);
+                            }
+                        }
+#pragma unroll
+                        for (int k = 0; k < kPoll; ++k) {
+                            const int i = ib + k * kConsumers;
+                            if (i < total) {
+                                bool ok = true;
+#pragma unroll
+                                for (int j = 0; j < 4; ++j) ok = ok && static_cast<uint32_t>(w[k][j] >> 32) == epoch;
+                                if (ok) {
+                                    v[k] = make_uint4(static_cast<uint32_t>(w[k][0]), static_cast<uint32_t>(w[k][1]),
+                                                      static_cast<uint32_t>(w[k][2]), static_cast<uint32_t>(w[k][3]));
+                                } else {
+                                    const int b = i / cpr, c = i - b * cpr;
+                                    v[k] = ll_load4(ll + static_cast<size_t>(b) * (K / 2) + 4 * c, epoch, p.err, p.abort);
+                                }
+                            }
+                        }
+                    }
+#pragma unroll
+                    for (int k = 0; k < kPoll; ++k) {
+                        const int i = ib + k * kConsumers;
+                        if (i < total) {
+                            const int b = i / cpr, c = i - b * cpr;
+                            xs[b * cpr + x_chunk(c >> 2, c & 3)] = v[k];
+#pragma unroll
+                            for (int bb = 0; bb < B; ++bb)
+                                if (bb == b) ss[bb] += sum8_sq(v[k]);
+                        }
+                    }
                 }
 #pragma unroll
                 for (int b = 0; b < B; ++b) {
@@ -361,12 +544,12 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const ChainPara
                     if (lane == 0) red[warp * kMaxChainBatch + b] = v;
                 }
             }
-            named_barrier_sync(1, kNW * 32);
+            named_barrier_sync(1, kConsumers);
             float rf[B];
 #pragma unroll
             for (int b = 0; b < B; ++b) {
-                float t = 0.f;
-                for (int w = 0; w < kNW; ++w) t += red[w * kMaxChainBatch + b];
+                // the same sum, in the same order, in every warp and every CTA
+                const float t = warp_sum(lane < NW ? red[lane * kMaxChainBatch + b] : 0.f);
                 rf[b] = (g.type == kDOWN) ? 1.f : 1.f / sqrtf(t / static_cast<float>(K) + p.eps);
             }
             if (g.type == kQKV || g.type == kLM) {
@@ -375,7 +558,7 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const ChainPara
                 const bool writer = (i0 == 0);   // first CTA that owns items
                 uint16_t* pv = p.pV + static_cast<size_t>(l) * B * H;
                 uint64_t* lv = p.llV + static_cast<size_t>(l) * B * (H / 2);
-                for (int i = threadIdx.x; i < B * cpr; i += kNW * 32) {
+                for (int i = threadIdx.x; i < B * cpr; i += kConsumers) {
                     const int b = i / cpr, c = i - b * cpr;
                     uint4& cell = xs[b * cpr + x_chunk(c >> 2, c & 3)];
                     float r = rf[0];
@@ -395,127 +578,68 @@ __global__ void __launch_bounds__(kChainThreads, 1) chain_kernel(const ChainPara
                         }
                     }
                 }
-                named_barrier_sync(1, kNW * 32);
+                named_barrier_sync(1, kConsumers);
 #pragma unroll
                 for (int b = 0; b < B; ++b) rf[b] = 1.f;
             }
 
-            // -- stream the CTA's items of this stage
+            // -- stream the CTA's items of this stage: item i0 + k goes to warp k % NW
             const int ips = items_per_slot(p, g);
-            for (int ia = i0; ia < i1; ia += ips, ++ord) {
+            const uint4* xl = xs + 4 * lane;
+            int it = i0 + warp;
+            for (int ia = i0; ia < i1; ia += ips) {
                 const int ib = min(i1, ia + ips);
-                const int slot = ord % p.nslots;
-                mbar_wait(&full[slot], (ord / p.nslots) & 1, p.err);
-                const uint8_t* base = slots + static_cast<size_t>(slot) * p.slot_bytes;
+                mbar_wait(&full[cslot], cpar, p.err);
+                const uint8_t* base = slots + static_cast<size_t>(cslot) * p.slot_bytes;
                 const ChunkLayout c = chunk_layout(g, ia, ib);
-                const int first = ia + ((warp - (ia - i0) % kNW) + kNW) % kNW;
-                for (int it = first; it < ib; it += kNW) {
-                    const int ii = it - ia;
-                    constexpr int RMAX = 4;
-                    const uint4* crow[RMAX];
-                    const uint16_t* srow[RMAX];
-                    const int rpi = g.rpi;
+                for (; it < ib; it += NW) {
+                    const int ii = it - ia;        // item within the chunk
+                    const uint4* crow[4];
+                    const uint16_t* srow[4];
                     if (g.type == kGU) {
 #pragma unroll
                         for (int r = 0; r < 4; ++r) {
                             const int half = r >> 1, rr = 2 * ii + (r & 1);
                             crow[r] = reinterpret_cast<const uint4*>(base + static_cast<size_t>(half) * (c.codes_bytes / 2) +
-                                                                     static_cast<size_t>(rr) * (K / 2));
+                                                                     static_cast<size_t>(rr) * (K / 2)) + lane;
                             srow[r] = reinterpret_cast<const uint16_t*>(base + c.codes_bytes + half * (c.scale_bytes / 2) +
-                                                                        rr * (K / 16));
+                                                                        rr * (K / 16)) + lane;
                         }
                     } else {
                         const int nvalid = min(2, g.N - 2 * it);
 #pragma unroll
                         for (int r = 0; r < 2; ++r) {
                             const int rr = 2 * ii + (r < nvalid ? r : 0);
-                            crow[r] = reinterpret_cast<const uint4*>(base + static_cast<size_t>(rr) * (K / 2));
-                            srow[r] = reinterpret_cast<const uint16_t*>(base + c.codes_bytes + rr * (K / 16));
+                            crow[r] = reinterpret_cast<const uint4*>(base + static_cast<size_t>(rr) * (K / 2)) + lane;
+                            srow[r] = reinterpret_cast<const uint16_t*>(base + c.codes_bytes + rr * (K / 16)) + lane;
                         }
                         crow[2] = crow[3] = crow[0];
                         srow[2] = srow[3] = srow[0];
                     }
-                    float acc[RMAX][B];
+                    float acc[4][B];
 #pragma unroll
-                    for (int r = 0; r < RMAX; ++r)
+                    for (int r = 0; r < 4; ++r)
 #pragma unroll
                         for (int b = 0; b < B; ++b) acc[r][b] = 0.f;
-
-                    if (rpi == 4) {
-                        for (int gg = lane; gg < gpr; gg += 32) {
+                    if (g.rpi == 4) item_dot<B, 4>(crow, srow, xl, cpr, gpr, lane, acc);
+                    else item_dot<B, 2>(crow, srow, xl, cpr, gpr, lane, acc);
 #pragma unroll
-                            for (int r = 0; r < 4; ++r)
-                                group_dot_smem<B>(crow[r][gg], half_bits_to_float(srow[r][gg]), xs, cpr, gg, acc[r]);
-                        }
-                    } else {
-                        for (int gg = lane; gg < gpr; gg += 32) {
-#pragma unroll
-                            for (int r = 0; r < 2; ++r)
-                                group_dot_smem<B>(crow[r][gg], half_bits_to_float(srow[r][gg]), xs, cpr, gg, acc[r]);
-                        }
-                    }
-#pragma unroll
-                    for (int r = 0; r < RMAX; ++r)
+                    for (int r = 0; r < 4; ++r)
 #pragma unroll
                         for (int b = 0; b < B; ++b)
-                            if (r < rpi) acc[r][b] = warp_sum(acc[r][b]);
-
-                    // -- fused epilogue (one lane per batch row)
+                            if (r < g.rpi) acc[r][b] = warp_sum(acc[r][b]);
 #pragma unroll
-                    for (int b = 0; b < B; ++b) {
-                        if (lane != b) continue;
-                        const int n = 2 * it;
-                        if (g.type == kQKV) {
-                            const uint16_t y0 = float_to_half_bits(rf[b] * acc[0][b]);
-                            const uint16_t y1 = float_to_half_bits(rf[b] * acc[1][b]);
-                            const uint32_t w = pack2(y0, y1);
-                            *reinterpret_cast<uint32_t*>(p.pQKV + (static_cast<size_t>(l) * B + b) * p.Nqkv + n) = w;
-                            if (n < H) ll_store(p.llA + (static_cast<size_t>(l) * B + b) * (H / 2) + n / 2, w, epoch);
-                        } else if (g.type == kO) {
-                            const uint16_t o0 = float_to_half_bits(rf[b] * acc[0][b]);
-                            const uint16_t o1 = float_to_half_bits(rf[b] * acc[1][b]);
-                            const uint32_t xw =
-                                ll_load(p.llV + (static_cast<size_t>(l) * B + b) * (H / 2) + n / 2, epoch, p.err, p.abort);
-                            const uint32_t x1 = pack2(add_h(lo_f(xw), half_bits_to_float(o0)),
-                                                      add_h(hi_f(xw), half_bits_to_float(o1)));
-                            const size_t off = (static_cast<size_t>(l) * B + b) * H + n;
-                            *reinterpret_cast<uint32_t*>(p.pO + off) = pack2(o0, o1);
-                            *reinterpret_cast<uint32_t*>(p.pX1 + off) = x1;
-                            ll_store(p.llX1 + (static_cast<size_t>(l) * B + b) * (H / 2) + n / 2, x1, epoch);
-                        } else if (g.type == kGU) {
-                            const int j = n;  // pair index of gate/up rows j, j+1
-                            const uint16_t g0 = float_to_half_bits(rf[b] * acc[0][b]);
-                            const uint16_t g1 = float_to_half_bits(rf[b] * acc[1][b]);
-                            const uint16_t u0 = float_to_half_bits(rf[b] * acc[2][b]);
-                            const uint16_t u1 = float_to_half_bits(rf[b] * acc[3][b]);
-                            const float gf0 = half_bits_to_float(g0), gf1 = half_bits_to_float(g1);
-                            const uint16_t m0 = float_to_half_bits(gf0 / (1.f + expf(-gf0)) * half_bits_to_float(u0));
-                            const uint16_t m1 = float_to_half_bits(gf1 / (1.f + expf(-gf1)) * half_bits_to_float(u1));
-                            const size_t gu = (static_cast<size_t>(l) * B + b) * (2 * F);
-                            *reinterpret_cast<uint32_t*>(p.pGU + gu + j) = pack2(g0, g1);
-                            *reinterpret_cast<uint32_t*>(p.pGU + gu + F + j) = pack2(u0, u1);
-                            const uint32_t mw = pack2(m0, m1);
-                            *reinterpret_cast<uint32_t*>(p.pM + (static_cast<size_t>(l) * B + b) * F + j) = mw;
-                            ll_store(p.llM + (static_cast<size_t>(l) * B + b) * (F / 2) + j / 2, mw, epoch);
-                        } else if (g.type == kDOWN) {
-                            const uint16_t d0 = float_to_half_bits(acc[0][b]);
-                            const uint16_t d1 = float_to_half_bits(acc[1][b]);
-                            const uint32_t x1 =
-                                ll_load(p.llX1 + (static_cast<size_t>(l) * B + b) * (H / 2) + n / 2, epoch, p.err, p.abort);
-                            const uint32_t x2 = pack2(add_h(lo_f(x1), half_bits_to_float(d0)),
-                                                      add_h(hi_f(x1), half_bits_to_float(d1)));
-                            *reinterpret_cast<uint32_t*>(p.pD + (static_cast<size_t>(l) * B + b) * H + n) = pack2(d0, d1);
-                            *reinterpret_cast<uint32_t*>(p.pX2 + (static_cast<size_t>(l) * B + b) * H + n) = x2;
-                            ll_store(p.llX + (static_cast<size_t>(l + 1) * B + b) * (H / 2) + n / 2, x2, epoch);
-                        } else {
-                            uint16_t* out = p.logits + static_cast<size_t>(b) * p.V;
-                            out[n] = float_to_half_bits(rf[b] * acc[0][b]);
-                            if (n + 1 < p.V) out[n + 1] = float_to_half_bits(rf[b] * acc[1][b]);
-                        }
-                    }
+                    for (int b = 0; b < B; ++b)
+                        if (lane == b)
+                            item_epilogue<B>(p, g, it, b, acc[0][b], acc[1][b], acc[2][b], acc[3][b], rf[b],
+                                             res[b * nit + (it - i0)], epoch);
                 }
                 __syncwarp();
-                if (lane == 0) mbar_arrive(&empty[slot]);
+                if (lane == 0) mbar_arrive(&empty[cslot]);
+                if (++cslot == p.nslots) {
+                    cslot = 0;
+                    cpar ^= 1u;
+                }
             }
         }
     }
@@ -610,6 +734,7 @@ struct Plan {
     int nslots;
     uint32_t slot_bytes, x_bytes;
     size_t smem;
+    int nw;
 };
 
 std::mutex g_plan_mu;
@@ -629,8 +754,19 @@ bool mat_ok(const wq4_mat& m)
 template <int B>
 cudaError_t set_chain_attr(int smem)
 {
-    return cudaFuncSetAttribute(chain_kernel<B>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    return cudaFuncSetAttribute(chain_kernel<B, ChainWarps<B>::NW>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
 }
+
+int chain_warps(int B)
+{
+    switch (B) {
+        case 1: return ChainWarps<1>::NW;
+        case 2: return ChainWarps<2>::NW;
+        case 3: return ChainWarps<3>::NW;
+        default: return ChainWarps<4>::NW;
+    }
+}
+
 
 // Slot size: a multiple of 128 bytes holding at least one item of every
 // stage, chosen to waste the least ring space over the chain's byte mix.
@@ -727,6 +863,9 @@ int build_plan(const wq4_layer_table* t, Plan* pl, cudaStream_t stream)
     pl->slot_bytes = slot_bytes;
     pl->x_bytes = x_bytes;
     pl->smem = smem;
+    pl->nw = chain_warps(d.B);
+    // the residual words of a CTA's rows must fit in shared memory
+    if (static_cast<long>((d.H / 2 + pl->grid - 1) / pl->grid) * d.B > kMaxResWords) return WQ4_ERR_UNSUPPORTED;
     return WQ4_OK;
 }
 
@@ -768,7 +907,7 @@ int launch_chain(const Plan& pl, const uint16_t* x, uint16_t* logits, cudaStream
 
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(pl.grid);
-    cfg.blockDim = dim3(kChainThreads);
+    cfg.blockDim = dim3((pl.nw + 1) * 32);
     cfg.dynamicSmemBytes = pl.smem;
     cfg.stream = stream;
     cudaLaunchAttribute attr[1];
@@ -778,10 +917,10 @@ int launch_chain(const Plan& pl, const uint16_t* x, uint16_t* logits, cudaStream
     cfg.numAttrs = 1;
     cudaError_t e;
     switch (pl.dims.B) {
-        case 1: e = cudaLaunchKernelEx(&cfg, chain_kernel<1>, p); break;
-        case 2: e = cudaLaunchKernelEx(&cfg, chain_kernel<2>, p); break;
-        case 3: e = cudaLaunchKernelEx(&cfg, chain_kernel<3>, p); break;
-        default: e = cudaLaunchKernelEx(&cfg, chain_kernel<4>, p); break;
+        case 1: e = cudaLaunchKernelEx(&cfg, chain_kernel<1, ChainWarps<1>::NW>, p); break;
+        case 2: e = cudaLaunchKernelEx(&cfg, chain_kernel<2, ChainWarps<2>::NW>, p); break;
+        case 3: e = cudaLaunchKernelEx(&cfg, chain_kernel<3, ChainWarps<3>::NW>, p); break;
+        default: e = cudaLaunchKernelEx(&cfg, chain_kernel<4, ChainWarps<4>::NW>, p); break;
     }
     return e == cudaSuccess ? WQ4_OK : WQ4_ERR_CUDA;
 }

@@ -44,6 +44,10 @@ namespace {
 
 constexpr int kChainMaxSlots = 32;
 constexpr int kMaxChainBatch = 4;
+// A ring slot is released after kSlotRelease arrivals: one per item consumed
+// from it, plus (kSlotRelease - items) from the warp that consumed its first
+// item.  Only warps that own items of a chunk touch its barriers.
+constexpr uint32_t kSlotRelease = 1024;
 // Shared-memory header: mbarriers | RMS partial sums | epoch | the residual
 // words of the CTA's rows (O and down stages); then the staged input vector,
 // then the weight ring.
@@ -300,20 +304,16 @@ __device__ __forceinline__ void group_rows_dot(const uint4* const crow[4], const
     }
 }
 
-// Every group of the item's rows: lane l takes groups l + 32 i.  Rows of 32,
-// 64, 96, 128 or 256 groups run fully unrolled (all loads of the item can be
-// issued ahead of its arithmetic); other lengths take a loop and a tail.
+// Every group of the item's rows: lane l takes groups l + 32 i.  Rows of 96,
+// 128 or 256 groups (K = 3072, 4096, 8192) run fully unrolled (all loads of
+// the item can be issued ahead of its arithmetic); other lengths take a loop
+// and a tail.
 template <int B, int RPI>
 __device__ __forceinline__ void item_dot(const uint4* const crow[4], const uint16_t* const srow[4],
                                          const uint4* xl, int cpr, int gpr, int lane, float acc[4][B])
 {
     const int sw = (lane >> 1) & 3;
     switch (gpr) {
-        case 32: group_rows_dot<B, RPI>(crow, srow, xl, cpr, sw, 0, acc); return;
-        case 64:
-#pragma unroll
-            for (int i = 0; i < 2; ++i) group_rows_dot<B, RPI>(crow, srow, xl, cpr, sw, 32 * i, acc);
-            return;
         case 96:
 #pragma unroll
             for (int i = 0; i < 3; ++i) group_rows_dot<B, RPI>(crow, srow, xl, cpr, sw, 32 * i, acc);
@@ -405,7 +405,7 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
     if (threadIdx.x == 0) {
         for (int i = 0; i < p.nslots; ++i) {
             mbar_init(&full[i], 1);
-            mbar_init(&empty[i], NW);
+            mbar_init(&empty[i], kSlotRelease);
         }
         mbar_fence_init();
         uint32_t s;
@@ -453,8 +453,7 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
     } else {
         // ------------------------------------------------ consumer warps
         const int H = p.H, F = p.F;
-        int cslot = 0;          // ring slot of the next chunk
-        uint32_t cpar = 0;      // phase parity of that slot's full barrier
+        int cbase = 0;          // ring ordinal of the stage's first chunk
         for (int st = 0; st < nstages; ++st) {
             const Stage g = stage_at(p, st);
             int i0, i1;
@@ -583,16 +582,22 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
                 for (int b = 0; b < B; ++b) rf[b] = 1.f;
             }
 
-            // -- stream the CTA's items of this stage: item i0 + k goes to warp k % NW
+            // -- stream the CTA's items of this stage: item i0 + k goes to warp
+            //    k % NW; a warp visits only the chunks that hold its items
             const int ips = items_per_slot(p, g);
+            const int nchunks = (nit + ips - 1) / ips;
             const uint4* xl = xs + 4 * lane;
-            int it = i0 + warp;
-            for (int ia = i0; ia < i1; ia += ips) {
-                const int ib = min(i1, ia + ips);
-                mbar_wait(&full[cslot], cpar, p.err);
-                const uint8_t* base = slots + static_cast<size_t>(cslot) * p.slot_bytes;
+            for (int it = i0 + warp; it < i1;) {
+                const int ch = (it - i0) / ips;            // chunk of this item
+                const int ia = i0 + ch * ips, ib = min(i1, ia + ips);
+                const int o = cbase + ch;                   // ring ordinal of the chunk
+                const int slot = o % p.nslots;
+                mbar_wait(&full[slot], (o / p.nslots) & 1, p.err);
+                const uint8_t* base = slots + static_cast<size_t>(slot) * p.slot_bytes;
                 const ChunkLayout c = chunk_layout(g, ia, ib);
+                uint32_t arrivals = (it == ia) ? kSlotRelease - static_cast<uint32_t>(ib - ia) : 0u;
                 for (; it < ib; it += NW) {
+                    ++arrivals;
                     const int ii = it - ia;        // item within the chunk
                     const uint4* crow[4];
                     const uint16_t* srow[4];
@@ -635,12 +640,9 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
                                              res[b * nit + (it - i0)], epoch);
                 }
                 __syncwarp();
-                if (lane == 0) mbar_arrive(&empty[cslot]);
-                if (++cslot == p.nslots) {
-                    cslot = 0;
-                    cpar ^= 1u;
-                }
+                if (lane == 0) mbar_arrive_count(&empty[slot], arrivals);
             }
+            cbase += nchunks;
         }
     }
 

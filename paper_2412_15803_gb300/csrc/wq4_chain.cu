@@ -55,7 +55,10 @@ constexpr int kHdrRed = 512;                 // float red[16][kMaxChainBatch]
 constexpr int kHdrEpoch = 768;
 constexpr int kHdrRes = 1024;                // uint32 res[kMaxResWords]: prefetched residual words
 constexpr int kMaxResWords = 1024;
-constexpr int kChainHeader = kHdrRes + 4 * kMaxResWords;
+__host__ __device__ constexpr int chain_header_bytes(int, int)
+{
+    return kHdrRes + 4 * kMaxResWords;
+}
 
 // Consumer warps per CTA: with the producer warp, 16 warps (128 registers a
 // thread) for batch 1-2, 8 warps (255 registers) for batch 3-4.
@@ -109,7 +112,7 @@ __device__ __forceinline__ Stage stage_at(const ChainParams& p, int st)
 {
     Stage g;
     if (st == 4 * p.L) {
-        g.type = kLM; g.layer = p.L; g.N = p.V; g.K = p.H; g.rpi = 2; g.items = (p.V + 1) / 2;
+        g.type = kLM; g.layer = p.L; g.N = p.V; g.K = p.H; g.rpi = 4; g.items = (p.V + 3) / 4;
     } else {
         g.layer = st >> 2;
         g.type = st & 3;
@@ -139,8 +142,8 @@ __device__ __forceinline__ ChunkLayout chunk_layout(const Stage& g, int ia, int 
         c.nh = 2 * (ib - ia);
         c.nrows = 2 * c.nh;
     } else {
-        const int r1 = min(2 * ib, g.N);
-        c.nrows = r1 - 2 * ia;
+        const int r1 = min(g.rpi * ib, g.N);
+        c.nrows = r1 - g.rpi * ia;
         c.nh = c.nrows;
     }
     c.codes_bytes = static_cast<uint32_t>(c.nrows) * (g.K / 2);
@@ -336,7 +339,8 @@ __device__ __forceinline__ void item_dot(const uint4* const crow[4], const uint1
 }
 
 // Fused epilogue of one item for batch row b: v0..v3 are the item's row sums
-// (rows 2it, 2it+1; for gate_up gate 2it, 2it+1 then up 2it, 2it+1); resw is
+// (rows 2it, 2it+1; gate_up: gate 2it, 2it+1 then up 2it, 2it+1; LM head:
+// rows 4it .. 4it+3); resw is
 // the item's residual word (O: the normalised layer input, down: x + o).
 template <int B>
 __device__ __forceinline__ void item_epilogue(const ChainParams& p, const Stage& g, int it, int b, float v0,
@@ -379,9 +383,13 @@ __device__ __forceinline__ void item_epilogue(const ChainParams& p, const Stage&
         *reinterpret_cast<uint32_t*>(p.pX2 + (static_cast<size_t>(l) * B + b) * H + n) = x2;
         ll_store(p.llX + (static_cast<size_t>(l + 1) * B + b) * (H / 2) + n / 2, x2, epoch);
     } else {
-        uint16_t* out = p.logits + static_cast<size_t>(b) * p.V;
-        out[n] = float_to_half_bits(rf * v0);
-        if (n + 1 < p.V) out[n + 1] = float_to_half_bits(rf * v1);
+        const int n4 = 4 * it;   // the LM head's items are 4 rows
+        uint16_t* out = p.logits + static_cast<size_t>(b) * p.V + n4;
+        const int nv = p.V - n4;
+        out[0] = float_to_half_bits(rf * v0);
+        if (nv > 1) out[1] = float_to_half_bits(rf * v1);
+        if (nv > 2) out[2] = float_to_half_bits(rf * v2);
+        if (nv > 3) out[3] = float_to_half_bits(rf * v3);
     }
 }
 
@@ -394,8 +402,9 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
     float* red = reinterpret_cast<float*>(smem + kHdrRed);          // [NW][kMaxChainBatch]
     uint32_t* epoch_sh = reinterpret_cast<uint32_t*>(smem + kHdrEpoch);
     uint32_t* res = reinterpret_cast<uint32_t*>(smem + kHdrRes);    // [B][items of the CTA]
-    uint4* xs = reinterpret_cast<uint4*>(smem + kChainHeader);
-    uint8_t* slots = smem + kChainHeader + p.x_bytes;
+    constexpr int kHeader = chain_header_bytes(NW, B);
+    uint4* xs = reinterpret_cast<uint4*>(smem + kHeader);
+    uint8_t* slots = smem + kHeader + p.x_bytes;
     constexpr int kConsumers = NW * 32;
     constexpr int kPoll = 2;     // input chunks a thread has in flight at once
 
@@ -441,8 +450,8 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
                         bulk_g2s(dst + c.codes_bytes, g.s + static_cast<size_t>(2 * ia) * gpr, hs, &full[slot], pol);
                         bulk_g2s(dst + c.codes_bytes + hs, g.s + (up + 2 * ia) * gpr, hs, &full[slot], pol);
                     } else {
-                        bulk_g2s(dst, g.W + static_cast<size_t>(2 * ia) * wpr, c.codes_bytes, &full[slot], pol);
-                        bulk_g2s(dst + c.codes_bytes, g.s + static_cast<size_t>(2 * ia) * gpr, c.scale_bytes,
+                        bulk_g2s(dst, g.W + static_cast<size_t>(g.rpi * ia) * wpr, c.codes_bytes, &full[slot], pol);
+                        bulk_g2s(dst + c.codes_bytes, g.s + static_cast<size_t>(g.rpi * ia) * gpr, c.scale_bytes,
                                  &full[slot], pol);
                     }
                 }
@@ -587,60 +596,69 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
             const int ips = items_per_slot(p, g);
             const int nchunks = (nit + ips - 1) / ips;
             const uint4* xl = xs + 4 * lane;
-            for (int it = i0 + warp; it < i1;) {
-                const int ch = (it - i0) / ips;            // chunk of this item
-                const int ia = i0 + ch * ips, ib = min(i1, ia + ips);
-                const int o = cbase + ch;                   // ring ordinal of the chunk
-                const int slot = o % p.nslots;
-                mbar_wait(&full[slot], (o / p.nslots) & 1, p.err);
-                const uint8_t* base = slots + static_cast<size_t>(slot) * p.slot_bytes;
-                const ChunkLayout c = chunk_layout(g, ia, ib);
-                uint32_t arrivals = (it == ia) ? kSlotRelease - static_cast<uint32_t>(ib - ia) : 0u;
-                for (; it < ib; it += NW) {
-                    ++arrivals;
-                    const int ii = it - ia;        // item within the chunk
-                    const uint4* crow[4];
-                    const uint16_t* srow[4];
-                    if (g.type == kGU) {
-#pragma unroll
-                        for (int r = 0; r < 4; ++r) {
-                            const int half = r >> 1, rr = 2 * ii + (r & 1);
-                            crow[r] = reinterpret_cast<const uint4*>(base + static_cast<size_t>(half) * (c.codes_bytes / 2) +
-                                                                     static_cast<size_t>(rr) * (K / 2)) + lane;
-                            srow[r] = reinterpret_cast<const uint16_t*>(base + c.codes_bytes + half * (c.scale_bytes / 2) +
-                                                                        rr * (K / 16)) + lane;
+            int it = i0 + warp;
+            if (it < i1) {
+                int ia = i0 + (warp / ips) * ips, ib = min(i1, ia + ips);
+                int slot = (cbase + warp / ips) % p.nslots;
+                uint32_t par = ((cbase + warp / ips) / p.nslots) & 1u;
+                while (it < i1) {
+                    while (it >= ib) {                      // next chunk
+                        ia += ips;
+                        ib = min(i1, ia + ips);
+                        if (++slot == p.nslots) {
+                            slot = 0;
+                            par ^= 1u;
                         }
-                    } else {
-                        const int nvalid = min(2, g.N - 2 * it);
-#pragma unroll
-                        for (int r = 0; r < 2; ++r) {
-                            const int rr = 2 * ii + (r < nvalid ? r : 0);
-                            crow[r] = reinterpret_cast<const uint4*>(base + static_cast<size_t>(rr) * (K / 2)) + lane;
-                            srow[r] = reinterpret_cast<const uint16_t*>(base + c.codes_bytes + rr * (K / 16)) + lane;
-                        }
-                        crow[2] = crow[3] = crow[0];
-                        srow[2] = srow[3] = srow[0];
                     }
-                    float acc[4][B];
+                    mbar_wait(&full[slot], par, p.err);
+                    const uint8_t* base = slots + static_cast<size_t>(slot) * p.slot_bytes;
+                    const ChunkLayout c = chunk_layout(g, ia, ib);
+                    uint32_t arrivals = (it == ia) ? kSlotRelease - static_cast<uint32_t>(ib - ia) : 0u;
+                    for (; it < ib; it += NW) {
+                        ++arrivals;
+                        const int ii = it - ia;        // item within the chunk
+                        const uint4* crow[4];
+                        const uint16_t* srow[4];
+                        if (g.type == kGU) {
 #pragma unroll
-                    for (int r = 0; r < 4; ++r)
+                            for (int r = 0; r < 4; ++r) {
+                                const int half = r >> 1, rr = 2 * ii + (r & 1);
+                                crow[r] = reinterpret_cast<const uint4*>(base + static_cast<size_t>(half) * (c.codes_bytes / 2) +
+                                                                         static_cast<size_t>(rr) * (K / 2)) + lane;
+                                srow[r] = reinterpret_cast<const uint16_t*>(base + c.codes_bytes + half * (c.scale_bytes / 2) +
+                                                                            rr * (K / 16)) + lane;
+                            }
+                        } else {
+                            // rows rpi*it .. rpi*it + rpi - 1; rows past N repeat the first
+                            const int nvalid = min(g.rpi, g.N - g.rpi * it);
 #pragma unroll
-                        for (int b = 0; b < B; ++b) acc[r][b] = 0.f;
-                    if (g.rpi == 4) item_dot<B, 4>(crow, srow, xl, cpr, gpr, lane, acc);
-                    else item_dot<B, 2>(crow, srow, xl, cpr, gpr, lane, acc);
+                            for (int r = 0; r < 4; ++r) {
+                                const int rr = g.rpi * ii + (r < nvalid ? r : 0);
+                                crow[r] = reinterpret_cast<const uint4*>(base + static_cast<size_t>(rr) * (K / 2)) + lane;
+                                srow[r] = reinterpret_cast<const uint16_t*>(base + c.codes_bytes + rr * (K / 16)) + lane;
+                            }
+                        }
+                        float acc[4][B];
 #pragma unroll
-                    for (int r = 0; r < 4; ++r)
+                        for (int r = 0; r < 4; ++r)
+#pragma unroll
+                            for (int b = 0; b < B; ++b) acc[r][b] = 0.f;
+                        if (g.rpi == 4) item_dot<B, 4>(crow, srow, xl, cpr, gpr, lane, acc);
+                        else item_dot<B, 2>(crow, srow, xl, cpr, gpr, lane, acc);
+#pragma unroll
+                        for (int r = 0; r < 4; ++r)
+#pragma unroll
+                            for (int b = 0; b < B; ++b)
+                                if (r < g.rpi) acc[r][b] = warp_sum(acc[r][b]);
 #pragma unroll
                         for (int b = 0; b < B; ++b)
-                            if (r < g.rpi) acc[r][b] = warp_sum(acc[r][b]);
-#pragma unroll
-                    for (int b = 0; b < B; ++b)
-                        if (lane == b)
-                            item_epilogue<B>(p, g, it, b, acc[0][b], acc[1][b], acc[2][b], acc[3][b], rf[b],
-                                             res[b * nit + (it - i0)], epoch);
+                            if (lane == b)
+                                item_epilogue<B>(p, g, it, b, acc[0][b], acc[1][b], acc[2][b], acc[3][b], rf[b],
+                                                 res[b * nit + (it - i0)], epoch);
+                    }
+                    __syncwarp();
+                    if (lane == 0) mbar_arrive_count(&empty[slot], arrivals);
                 }
-                __syncwarp();
-                if (lane == 0) mbar_arrive_count(&empty[slot], arrivals);
             }
             cbase += nchunks;
         }
@@ -780,7 +798,7 @@ uint32_t choose_slot_bytes(const Dims& d)
                      {2 * rowH, static_cast<size_t>(d.H) * rowH},
                      {4 * rowH, static_cast<size_t>(2) * d.F * rowH},
                      {2 * rowF, static_cast<size_t>(d.H) * rowF},
-                     {2 * rowH, static_cast<size_t>(d.V) * rowH}};
+                     {4 * rowH, static_cast<size_t>(d.V) * rowH}};
     size_t max_item = 0;
     for (const S& s : st) max_item = s.item > max_item ? s.item : max_item;
     size_t lo = align_up(max_item, 128);
@@ -820,11 +838,12 @@ int build_plan(const wq4_layer_table* t, Plan* pl, cudaStream_t stream)
     if (!di->coop_launch) return WQ4_ERR_UNSUPPORTED;
     const uint32_t x_bytes = static_cast<uint32_t>(align_up(static_cast<size_t>(d.B) * 2 * (d.H > d.F ? d.H : d.F), 128));
     const uint32_t slot_bytes = choose_slot_bytes(d);
-    const long avail = static_cast<long>(di->smem_optin) - kChainHeader - static_cast<long>(x_bytes);
+    const int header = chain_header_bytes(chain_warps(d.B), d.B);
+    const long avail = static_cast<long>(di->smem_optin) - header - static_cast<long>(x_bytes);
     int nslots = avail > 0 ? static_cast<int>(avail / slot_bytes) : 0;
     if (nslots < 2) return WQ4_ERR_UNSUPPORTED;
     if (nslots > kChainMaxSlots) nslots = kChainMaxSlots;
-    const size_t smem = kChainHeader + x_bytes + static_cast<size_t>(nslots) * slot_bytes;
+    const size_t smem = header + x_bytes + static_cast<size_t>(nslots) * slot_bytes;
     // The limit is a property of the kernel, shared by every plan: set it to
     // the device maximum so that no plan's launch depends on which plan was
     // built last.

@@ -157,15 +157,16 @@ size_t wq4_chain_workspace_bytes(const wq4_layer_table* table);
  * layer's output), re-feeds it after RMS normalisation, and rounds every
  * stage output to fp16:
  *   v   = r(u) * u                     r(t) = 1/sqrt(mean(t^2) + rms_eps)
- *   qkv = W_qkv . v
+ *   qkv = r(u)  * W_qkv . u
  *   o   = r(a)  * W_o   . a            a = qkv[:, :hidden] (stands in for
  *   x1  = v + o                            attention, which is not in the chain)
  *   gu  = r(x1) * W_gu  . x1
  *   m   = silu(gu[:, :ffn]) * gu[:, ffn:]
  *   x2  = x1 + W_down . m              (the layer output, next layer's u)
- * then logits = W_lm . (r(xL) * xL).  RMS normalisation has no learned gain;
- * before O and gate_up it enters as a per-row factor of the projection
- * (Section 2.3 "kernel fusion").
+ * then logits = r(xL) * W_lm . xL.  RMS normalisation has no learned gain and
+ * enters every projection as a per-row factor (r(t) W.t = W.(r(t) t); Section
+ * 2.3 "kernel fusion"); the normalised v is materialised only in the
+ * residual stream.
  *   x      : fp16 [batch][hidden] device, 16-byte aligned
  *   logits : fp16 [batch][vocab]  device, 2-byte aligned
  * The first call for a table (or after its contents changed) validates it and

@@ -12,8 +12,8 @@ Layer l takes u (fp16 [batch][H]: the token input for l = 0, else the previous
 layer's output) and re-feeds it after RMS normalisation; every stage output
 is rounded to fp16:
 
-    v   = fp16( r(u) * u )                       layer input, RMS-normalised
-    qkv = fp16(          W_qkv  . v  )          [batch][Nqkv]
+    v   = fp16( r(u) * u )                       the normalised layer input
+    qkv = fp16( r(u)   * W_qkv  . u  )          [batch][Nqkv]
     a   = qkv[:, :H]                             (stands in for attention)
     o   = fp16( r(a)   * W_o    . a  )          [batch][H]
     x1  = fp16( v + o )
@@ -22,12 +22,13 @@ is rounded to fp16:
     d   = fp16(          W_down . m  )          [batch][H]
     x2  = fp16( x1 + d )                         layer output
 
-and after the last layer: logits = fp16( W_lm . fp16(r(xL) * xL) ).
+and after the last layer: logits = fp16( r(xL) * W_lm . xL ).
 
 r(v) = 1 / sqrt(mean(v^2) + eps) is RMS normalisation without a learned gain.
-Where it precedes a projection of an unnormalised vector (O, gate_up) it is
-applied as a per-row factor of the projection (r(v) W.v = W.(r(v) v) in real
-arithmetic), so that projection's input stays the fp16 vector.
+Before every projection it is applied as a per-row factor of the projection
+(r(v) W.v = W.(r(v) v) in real arithmetic), so the projection's input is the
+fp16 vector itself; the normalised vector v is rounded to fp16 only where it
+is kept, in the residual stream (x1 = v + o).
 
 Each step calls the primitives of ``oracle`` and nothing else.
 """
@@ -49,10 +50,11 @@ def layer(u, w, H: int, F: int, eps: float):
     Returns (x2, trace) where trace holds every stage's fp16 output and the
     fp64 values with their magnitudes A for the projections."""
     t = {"u": u}
+    r1 = rms_factors(u, eps)
     v = rms_normalize(u, eps)
     t["v"] = v
-    y, A, qkv = gemv(*w["qkv"], v)
-    t.update(qkv=qkv, qkv_ref=y, qkv_A=A)
+    y, A, qkv = gemv(*w["qkv"], u, r1)
+    t.update(r_u=r1, qkv=qkv, qkv_ref=y, qkv_A=A)
     a = np.ascontiguousarray(qkv[:, :H])
     r2 = rms_factors(a, eps)
     y, A, o = gemv(*w["o"], a, r2)
@@ -79,7 +81,7 @@ def token(x, layers, lm_head, H: int, F: int, eps: float):
     for w in layers:
         x, t = layer(x, w, H, F, eps)
         traces.append(t)
-    v = rms_normalize(x, eps)
-    y, A, logits = gemv(*lm_head, v)
-    traces.append({"u": x, "v": v, "logits_ref": y, "logits_A": A})
+    rf = rms_factors(x, eps)
+    y, A, logits = gemv(*lm_head, x, rf)
+    traces.append({"u": x, "v": rms_normalize(x, eps), "logits_ref": y, "logits_A": A})
     return logits, y, traces

@@ -12,10 +12,10 @@
 //    copies (TMA) and mbarriers.  Weights do not depend on activations, so the
 //    stream runs ahead across stage boundaries and HBM keeps working while the
 //    consumers wait for the next activation vector.
-//  * Each layer re-feeds its input after RMS normalisation: the QKV stage (and
-//    the LM head) normalise the staged vector in shared memory; every CTA
-//    computes the same factor in the same order, so all CTAs hold identical
-//    bits, and the first CTA publishes them for the O stage's residual add.
+//  * Each layer re-feeds its input after RMS normalisation.  Every CTA
+//    computes the same factor in the same order (identical bits everywhere),
+//    applies it as a row factor of its projection, and publishes its slice of
+//    the normalised vector for the O stage's residual add.
 //  * Consumer warps stage each stage's input vector in shared memory, take
 //    two-row items (four rows for gate_up: gate j, j+1 and up j, j+1)
 //    round-robin, unpack in registers, accumulate in fp32, and apply the
@@ -561,34 +561,25 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
                 rf[b] = (g.type == kDOWN) ? 1.f : 1.f / sqrtf(t / static_cast<float>(K) + p.eps);
             }
             if (g.type == kQKV || g.type == kLM) {
-                // re-feed after RMS normalisation: xs <- fp16(r * u), in place;
-                // each thread rescales the chunks it staged itself
-                const bool writer = (i0 == 0);   // first CTA that owns items
-                uint16_t* pv = p.pV + static_cast<size_t>(l) * B * H;
-                uint64_t* lv = p.llV + static_cast<size_t>(l) * B * (H / 2);
-                for (int i = threadIdx.x; i < B * cpr; i += kConsumers) {
-                    const int b = i / cpr, c = i - b * cpr;
-                    uint4& cell = xs[b * cpr + x_chunk(c >> 2, c & 3)];
+                // the normalised layer input v = fp16(r * u) is kept for the
+                // residual stream (and the trace): every CTA publishes its
+                // slice of it; the projections below use r as a row factor
+                const int nw = H / 2;                       // words of v per batch row
+                const int w0 = static_cast<int>(static_cast<int64_t>(blockIdx.x) * nw / gridDim.x);
+                const int w1 = static_cast<int>(static_cast<int64_t>(blockIdx.x + 1) * nw / gridDim.x);
+                const uint32_t* xw = reinterpret_cast<const uint32_t*>(xs);
+                for (int t = threadIdx.x; t < B * (w1 - w0); t += kConsumers) {
+                    const int b = t / (w1 - w0), w = w0 + (t - b * (w1 - w0));
+                    const int c = w >> 2;                   // chunk of the word
+                    const uint32_t u = xw[4 * (b * cpr + x_chunk(c >> 2, c & 3)) + (w & 3)];
                     float r = rf[0];
 #pragma unroll
                     for (int bb = 1; bb < B; ++bb)
                         if (bb == b) r = rf[bb];
-                    const uint4 v = scale8(cell, r);
-                    cell = v;
-                    if (writer) {
-                        reinterpret_cast<uint4*>(pv + static_cast<size_t>(b) * H)[c] = v;
-                        if (g.type == kQKV) {
-                            uint64_t* w = lv + static_cast<size_t>(b) * (H / 2) + 4 * c;
-                            ll_store(w + 0, v.x, epoch);
-                            ll_store(w + 1, v.y, epoch);
-                            ll_store(w + 2, v.z, epoch);
-                            ll_store(w + 3, v.w, epoch);
-                        }
-                    }
+                    const uint32_t v = pack2(float_to_half_bits(r * lo_f(u)), float_to_half_bits(r * hi_f(u)));
+                    reinterpret_cast<uint32_t*>(p.pV + (static_cast<size_t>(l) * B + b) * H)[w] = v;
+                    if (g.type == kQKV) ll_store(p.llV + (static_cast<size_t>(l) * B + b) * (H / 2) + w, v, epoch);
                 }
-                named_barrier_sync(1, kConsumers);
-#pragma unroll
-                for (int b = 0; b < B; ++b) rf[b] = 1.f;
             }
 
             // -- stream the CTA's items of this stage: item i0 + k goes to warp

@@ -64,7 +64,7 @@ def check_stages(model, layer, rows=None, u=None):
         y, A, _ = oracle.gemv(W, s, inp, r)
         within(out[:, idx], y, A, f"layer {layer} {name}")
 
-    proj("qkv", t["x_in"], False, t["qkv"], sh.n_qkv)
+    proj("qkv", np.ascontiguousarray(u), True, t["qkv"], sh.n_qkv)
     a = np.ascontiguousarray(t["qkv"][:, :H])
     proj("o", a, True, t["o"], H)
     assert np.array_equal(t["x_mid"], oracle.add_fp16(t["x_in"], t["o"]))
@@ -87,9 +87,10 @@ def _rows(model, layer, name, idx):
 
 def check_logits(model, logits, rows=None):
     sh = model.shape
-    xin = model.trace(sh.num_layers)["x_in"]
-    check_norm(xin, model.trace(sh.num_layers - 1)["x_out"], model.eps, "LM head input normalisation")
-    r = None
+    xL = model.trace(sh.num_layers - 1)["x_out"]
+    check_norm(model.trace(sh.num_layers)["x_in"], xL, model.eps, "LM head input normalisation")
+    xin = xL
+    r = ochain.rms_factors(xL, model.eps)
     if rows is None:
         W, s = model.host_rows(sh.num_layers, "lm_head", 0, sh.vocab)
         idx = np.arange(sh.vocab)

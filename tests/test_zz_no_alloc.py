@@ -28,7 +28,7 @@ def _logits_pair(model, x):
     wq4.wq4_decode_chain(model.table, xd, ref)
     torch.cuda.synchronize()
     ref_np = ref.cpu().numpy().view(np.uint16)
-    lm_in = model.trace(model.shape.num_layers)["x_in"]     # from the allocated workspace
+    lm_in = model.trace(model.shape.num_layers - 1)["x_out"]   # from the allocated workspace
     outs = []
     for _ in range(2):                                       # two calls in a row
         out = torch.full((model.batch, model.shape.vocab), -1, dtype=torch.int16, device="cuda")
@@ -43,7 +43,8 @@ def _within(got, ref16, model, lm_in):
     """|got - ref| within the GEMV tolerance 1e-3 * sum|w x| + ulp16(|ref|)."""
     sh = model.shape
     W, s = model.host_rows(sh.num_layers, "lm_head", 0, sh.vocab)
-    _, A, _ = oracle.gemv(W, s, lm_in)
+    from oracle import chain as ochain
+    _, A, _ = oracle.gemv(W, s, lm_in, ochain.rms_factors(lm_in, model.eps))
     ref = oracle.half_to_double(ref16)
     err = np.abs(oracle.half_to_double(got) - ref)
     assert np.all(err <= oracle.tolerance(ref, A))

@@ -217,6 +217,23 @@ def run_reference(args, rank, world):
 
 # ------------------------------------------------------------------- ours --
 
+def aggregate_replicas(total_ms: float, e2e_s_per_step: float, batch: int, steps: int, device="cpu"):
+    """Whole-job numbers over the ranks of the default process group (if any).
+
+    Every rank decodes its own replica for the same number of steps, so the
+    job time is the slowest rank's: returns (tokens/s, e2e tokens/s, job ms)
+    computed from the MAX over ranks of the timed region and of the e2e time
+    per step.  Works with any backend (nccl on GPUs, gloo on CPU)."""
+    import torch
+    import torch.distributed as dist
+    world = dist.get_world_size() if dist.is_available() and dist.is_initialized() else 1
+    t = torch.tensor([total_ms, e2e_s_per_step], dtype=torch.float64, device=device)
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    job_ms, e2e_step = float(t[0].item()), float(t[1].item())
+    return world * batch * steps / (job_ms / 1e3), world * batch / e2e_step, job_ms
+
+
 def run_ours(args, rank, world, local):
     import torch
     import torch.distributed as dist
@@ -270,11 +287,6 @@ def run_ours(args, rank, world, local):
     if wq4.wq4_device_status(stream) != 0:
         raise RuntimeError("device wait timed out during the timed region")
 
-    t = torch.tensor([total_ms], dtype=torch.float64, device="cuda")
-    if world > 1:
-        dist.all_reduce(t, op=dist.ReduceOp.MAX)
-    total_ms_max = float(t.item())
-
     # end to end through the host-buffer entry point: x H2D, chain, logits D2H
     x_host = torch.from_numpy(x_np.view(np.int16)).pin_memory()
     l_host = torch.empty((B, shape.vocab), dtype=torch.int16).pin_memory()
@@ -285,15 +297,10 @@ def run_ours(args, rank, world, local):
     for _ in range(e2e_steps):
         model.decode_host(x_host.numpy(), l_host.numpy(), stream)
     e2e_s = time.perf_counter() - t0
-    e2e_val = B * e2e_steps / e2e_s
-    if world > 1:
-        te = torch.tensor([e2e_s / e2e_steps], dtype=torch.float64, device="cuda")
-        dist.all_reduce(te, op=dist.ReduceOp.MAX)
-        e2e_val = world * B / float(te.item())
+    tokens_per_s, e2e_val, total_ms_max = aggregate_replicas(total_ms, e2e_s / e2e_steps, B, args.steps, "cuda")
 
     if rank == 0:
         ms = total_ms_max / args.steps
-        tokens_per_s = world * B * args.steps / (total_ms_max / 1e3)
         avg_launch_ms = statistics.mean(launch_ms)
         peak, peak_src = measured_peak()
         achieved = step_bytes / (avg_launch_ms * 1e-3) / 1e9

@@ -157,7 +157,7 @@ def oracle_sample(shape, batch: int, fraction: float, seed: int = 0):
     total_t, total_w = 0.0, 0
     for N, K, l, mat in blocks:
         n = max(1, int(np.ceil(fraction * N)))
-        W, s = synth.matrix(seed, N, K, l, mat, 0, n)
+        W, s = synth.matrix(seed, N, K, l, mat, 0, n, symmetric=True)
         t0 = time.perf_counter()
         oracle.gemv(W, s, x[K])
         total_t += time.perf_counter() - t0

@@ -132,8 +132,7 @@ typedef struct {
  *   is the stand-in attention output, see wq4_decode_chain).
  *   workspace  : device buffer of at least wq4_chain_workspace_bytes(table)
  *                bytes, 256-byte aligned, used only by this table's chain.
- *   All dimensions must be multiples of 256 except vocab (any >= 1); batch
- *   1..4 (WQ4_ERR_UNSUPPORTED above).
+ *   hidden and ffn must be multiples of 256, vocab any >= 1, batch 1..32.
  */
 typedef struct {
     int num_layers, hidden, ffn, n_q_heads, n_kv_heads, head_dim, vocab, batch;
@@ -169,9 +168,16 @@ size_t wq4_chain_workspace_bytes(const wq4_layer_table* table);
  * residual stream.
  *   x      : fp16 [batch][hidden] device, 16-byte aligned
  *   logits : fp16 [batch][vocab]  device, 2-byte aligned
+ * Batch 1-4 runs as the persistent kernel above.  Batch 5-32 runs as a CUDA
+ * graph of stage kernels (RMS factors, a CUDA-core stage GEMV with the row
+ * factor and the residual add fused, SiLU * up), captured once per table;
+ * each call copies x into the workspace, replays the graph and copies the
+ * logits out (all on `stream`).
  * The first call for a table (or after its contents changed) validates it and
  * uploads its pointer table into the workspace (cudaMemcpyAsync on `stream`);
- * later calls only launch.  Calls on one table must not overlap on the GPU.
+ * later calls only launch.  Rebuilding the plan of a batch 5-32 table
+ * synchronizes `stream` before freeing the old graph.  Calls on one table must
+ * not overlap on the GPU.
  * Returns WQ4_OK, WQ4_ERR_INVALID, WQ4_ERR_ALIGN, WQ4_ERR_UNSUPPORTED or
  * WQ4_ERR_CUDA (including a GPU that cannot co-schedule the persistent grid).
  */

@@ -21,10 +21,15 @@ extern "C" {
 
 /* Words [word_start, word_start + nwords) of a packed-code stream:
  * word 2m = low 32 bits of u64(key, m), word 2m+1 = high 32 bits.
+ * symmetric = 0: every code uniform on 0..15 (covers the whole format).
+ * symmetric != 0: then every code equal to 15 becomes 7, so codes lie in
+ * 0..14 with mean 7, the range of symmetric 4-bit quantisation (|q - 7| <= 7)
+ * and zero-mean weights, as trained models have; used for whole synthetic
+ * models, whose activations would otherwise drift out of fp16 range.
  * W: device uint32 buffer of nwords entries; word_start and nwords even.
  * Returns 0, -1 on bad arguments, -4 on a CUDA launch failure. */
 int wq4_synth_codes(uint32_t* W, int64_t word_start, int64_t nwords,
-                    uint64_t seed, uint64_t sid, void* stream);
+                    uint64_t seed, uint64_t sid, int symmetric, void* stream);
 
 /* Scales [start, start + n): fp16_RNE(lo + (hi - lo) * u),
  * u = (u64(key, i) >> 11) * 2^-53, one fp64 multiply then one fp64 add,

@@ -42,16 +42,26 @@
 namespace wq4 {
 namespace {
 
-constexpr int kChainMaxSlots = 32;
+constexpr int kChainMaxSlots = 16;
+// Chunk c of the ring lives in slot c % nslots and lands on full barrier
+// c % nbars, nbars = (kFullBars / nslots) * nslots.  A parity wait only tells
+// the wanted phase from the one before it, so a warp may wait on chunk c only
+// once chunk c - nbars has landed; consumer warps skip the chunks without
+// their items, and the plan keeps nslots + ceil(NW / items per slot) <= nbars
+// for every stage, which bounds how far ahead of the oldest unconsumed chunk
+// a warp can be (nslots - 1 + ceil(NW / items per slot) chunks).
+constexpr int kFullBars = 48;
 constexpr int kMaxChainBatch = 4;
 // A ring slot is released after kSlotRelease arrivals: one per item consumed
 // from it, plus (kSlotRelease - items) from the warp that consumed its first
 // item.  Only warps that own items of a chunk touch its barriers.
 constexpr uint32_t kSlotRelease = 1024;
-// Shared-memory header: mbarriers | RMS partial sums | epoch | the residual
+// Shared-memory header: mbarriers (kFullBars full, kChainMaxSlots empty) |
+// RMS partial sums | epoch | the residual
 // words of the CTA's rows (O and down stages); then the staged input vector,
 // then the weight ring.
 constexpr int kHdrRed = 512;                 // float red[16][kMaxChainBatch]
+static_assert(8 * (kFullBars + kChainMaxSlots) <= kHdrRed, "mbarriers overlap the header");
 constexpr int kHdrEpoch = 768;
 constexpr int kHdrRes = 1024;                // uint32 res[kMaxResWords]: prefetched residual words
 constexpr int kMaxResWords = 1024;
@@ -97,6 +107,7 @@ struct ChainParams {
     uint16_t* pM;        // [L][B][F]
     uint16_t* pD;        // [L][B][H]
     int nslots;
+    int nbars;           // full barriers: a multiple of nslots
     uint32_t slot_bytes;
     uint32_t x_bytes;
     uint32_t* err;
@@ -398,7 +409,7 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
 {
     extern __shared__ __align__(1024) uint8_t smem[];
     uint64_t* full = reinterpret_cast<uint64_t*>(smem);
-    uint64_t* empty = full + kChainMaxSlots;
+    uint64_t* empty = full + kFullBars;
     float* red = reinterpret_cast<float*>(smem + kHdrRed);          // [NW][kMaxChainBatch]
     uint32_t* epoch_sh = reinterpret_cast<uint32_t*>(smem + kHdrEpoch);
     uint32_t* res = reinterpret_cast<uint32_t*>(smem + kHdrRes);    // [B][items of the CTA]
@@ -412,10 +423,8 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
     const int nstages = 4 * p.L + 1;
 
     if (threadIdx.x == 0) {
-        for (int i = 0; i < p.nslots; ++i) {
-            mbar_init(&full[i], 1);
-            mbar_init(&empty[i], kSlotRelease);
-        }
+        for (int i = 0; i < p.nbars; ++i) mbar_init(&full[i], 1);
+        for (int i = 0; i < p.nslots; ++i) mbar_init(&empty[i], kSlotRelease);
         mbar_fence_init();
         uint32_t s;
         asm volatile("ld.relaxed.gpu.global.b32 %0, [%1];" : "=r"(s) : "l"(p.seq) : "memory");
@@ -441,23 +450,26 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
                     if (round > 0) mbar_wait(&empty[slot], (round - 1) & 1, p.err);
                     const ChunkLayout c = chunk_layout(g, ia, ib);
                     uint8_t* dst = slots + static_cast<size_t>(slot) * p.slot_bytes;
-                    mbar_arrive_expect_tx(&full[slot], c.codes_bytes + c.scale_bytes);
+                    uint64_t* fb = &full[ord % p.nbars];
+                    mbar_arrive_expect_tx(fb, c.codes_bytes + c.scale_bytes);
                     if (g.type == kGU) {
                         const uint32_t hc = c.codes_bytes / 2, hs = c.scale_bytes / 2;
                         const size_t up = static_cast<size_t>(p.F);
-                        bulk_g2s(dst, g.W + static_cast<size_t>(2 * ia) * wpr, hc, &full[slot], pol);
-                        bulk_g2s(dst + hc, g.W + (up + 2 * ia) * wpr, hc, &full[slot], pol);
-                        bulk_g2s(dst + c.codes_bytes, g.s + static_cast<size_t>(2 * ia) * gpr, hs, &full[slot], pol);
-                        bulk_g2s(dst + c.codes_bytes + hs, g.s + (up + 2 * ia) * gpr, hs, &full[slot], pol);
+                        bulk_g2s(dst, g.W + static_cast<size_t>(2 * ia) * wpr, hc, fb, pol);
+                        bulk_g2s(dst + hc, g.W + (up + 2 * ia) * wpr, hc, fb, pol);
+                        bulk_g2s(dst + c.codes_bytes, g.s + static_cast<size_t>(2 * ia) * gpr, hs, fb, pol);
+                        bulk_g2s(dst + c.codes_bytes + hs, g.s + (up + 2 * ia) * gpr, hs, fb, pol);
                     } else {
-                        bulk_g2s(dst, g.W + static_cast<size_t>(g.rpi * ia) * wpr, c.codes_bytes, &full[slot], pol);
+                        bulk_g2s(dst, g.W + static_cast<size_t>(g.rpi * ia) * wpr, c.codes_bytes, fb, pol);
                         bulk_g2s(dst + c.codes_bytes, g.s + static_cast<size_t>(g.rpi * ia) * gpr, c.scale_bytes,
-                                 &full[slot], pol);
+                                 fb, pol);
                     }
                 }
             }
+            // every chunk before the last nslots was consumed, so has landed:
+            // wait for the rest before the CTA's shared memory goes away
             const int first = ord > p.nslots ? ord - p.nslots : 0;
-            for (int o = first; o < ord; ++o) mbar_wait(&full[o % p.nslots], (o / p.nslots) & 1, p.err);
+            for (int o = first; o < ord; ++o) mbar_wait(&full[o % p.nbars], (o / p.nbars) & 1, p.err);
         }
     } else {
         // ------------------------------------------------ consumer warps
@@ -590,18 +602,20 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
             int it = i0 + warp;
             if (it < i1) {
                 int ia = i0 + (warp / ips) * ips, ib = min(i1, ia + ips);
-                int slot = (cbase + warp / ips) % p.nslots;
-                uint32_t par = ((cbase + warp / ips) / p.nslots) & 1u;
+                const int o0 = cbase + warp / ips;          // ring ordinal of the first chunk
+                int slot = o0 % p.nslots, bar = o0 % p.nbars;
+                uint32_t par = (o0 / p.nbars) & 1u;
                 while (it < i1) {
                     while (it >= ib) {                      // next chunk
                         ia += ips;
                         ib = min(i1, ia + ips);
-                        if (++slot == p.nslots) {
-                            slot = 0;
+                        if (++slot == p.nslots) slot = 0;
+                        if (++bar == p.nbars) {
+                            bar = 0;
                             par ^= 1u;
                         }
                     }
-                    mbar_wait(&full[slot], par, p.err);
+                    mbar_wait(&full[bar], par, p.err);
                     const uint8_t* base = slots + static_cast<size_t>(slot) * p.slot_bytes;
                     const ChunkLayout c = chunk_layout(g, ia, ib);
                     uint32_t arrivals = (it == ia) ? kSlotRelease - static_cast<uint32_t>(ib - ia) : 0u;
@@ -668,10 +682,113 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
     }
 }
 
+// ------------------------------------------------- graph path (batch 5-32) --
+//
+// For batches beyond what the persistent kernel stages in shared memory, the
+// token runs as a CUDA graph of stage kernels (captured once per plan): RMS
+// factors, a CUDA-core stage GEMV with the row factor, a strided input and a
+// fused residual add, and SiLU(gate) * up.  They write the same workspace
+// traces as the persistent kernel.
+
+// r[b] = 1/sqrt(mean(u[b]^2) + eps) over K fp16 values (row stride ld), one
+// CTA per batch row, summed in a fixed order; optionally v[b] = fp16(r[b] u[b]).
+__global__ void __launch_bounds__(256) rms_rows_kernel(const uint16_t* __restrict__ u, int ld, int K, float eps,
+                                                       float* __restrict__ r, uint16_t* __restrict__ v, int ldv)
+{
+    __shared__ float red[8];
+    const int b = blockIdx.x;
+    const uint16_t* ub = u + static_cast<size_t>(b) * ld;
+    float ss = 0.f;
+    for (int k = threadIdx.x; k < K; k += blockDim.x) {
+        const float t = half_bits_to_float(ub[k]);
+        ss = fmaf(t, t, ss);
+    }
+    ss = warp_sum(ss);
+    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
+    __syncthreads();
+    float tot = 0.f;
+#pragma unroll
+    for (int w = 0; w < 8; ++w) tot += red[w];
+    const float rb = 1.f / sqrtf(tot / static_cast<float>(K) + eps);
+    if (threadIdx.x == 0) r[b] = rb;
+    if (v) {
+        uint16_t* vb = v + static_cast<size_t>(b) * ldv;
+        for (int k = threadIdx.x; k < K; k += blockDim.x) vb[k] = float_to_half_bits(rb * half_bits_to_float(ub[k]));
+    }
+}
+
+// y[b][n] = fp16(r[b] * sum_k (q - 7) s x[b][k]) for a warp per row n, batch
+// in tiles of BT; x rows at stride ldx; with `res`, also y2 = fp16(res + y).
+template <int BT>
+__global__ void __launch_bounds__(256) stage_gemv_kernel(const uint32_t* __restrict__ W, const uint16_t* __restrict__ s,
+                                                         int N, int K, const uint16_t* __restrict__ x, int ldx, int B,
+                                                         const float* __restrict__ r, uint16_t* __restrict__ y, int ldy,
+                                                         const uint16_t* __restrict__ res, int ldres,
+                                                         uint16_t* __restrict__ y2, int ldy2)
+{
+    const int lane = threadIdx.x & 31;
+    const int gw = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
+    const int nw = gridDim.x * (blockDim.x >> 5);
+    const int gpr = K >> 5;
+    for (int n = gw; n < N; n += nw) {
+        const uint4* crow = reinterpret_cast<const uint4*>(W + static_cast<size_t>(n) * (K >> 3));
+        const uint16_t* srow = s + static_cast<size_t>(n) * gpr;
+        for (int b0 = 0; b0 < B; b0 += BT) {
+            float acc[BT];
+#pragma unroll
+            for (int b = 0; b < BT; ++b) acc[b] = 0.f;
+            for (int g = lane; g < gpr; g += 32) {
+                const uint4 cw = __ldg(crow + g);
+                const float sc = half_bits_to_float(__ldg(srow + g));
+                uint32_t q[16];
+                unpack_word(cw.x, q + 0);
+                unpack_word(cw.y, q + 4);
+                unpack_word(cw.z, q + 8);
+                unpack_word(cw.w, q + 12);
+#pragma unroll
+                for (int b = 0; b < BT; ++b) {
+                    if (b0 + b < B) {
+                        const uint4* xb = reinterpret_cast<const uint4*>(x + static_cast<size_t>(b0 + b) * ldx) + 4 * g;
+                        const float a01 = fma8(q + 4, __ldg(xb + 1), fma8(q + 0, __ldg(xb + 0), 0.f));
+                        const float a23 = fma8(q + 12, __ldg(xb + 3), fma8(q + 8, __ldg(xb + 2), 0.f));
+                        acc[b] = fmaf(sc, a01 + a23, acc[b]);
+                    }
+                }
+            }
+#pragma unroll
+            for (int b = 0; b < BT; ++b) {
+                const float v = warp_sum(acc[b]);
+                const int bb = b0 + b;
+                if (lane == b && bb < B) {
+                    const uint16_t yv = float_to_half_bits(r ? r[bb] * v : v);
+                    y[static_cast<size_t>(bb) * ldy + n] = yv;
+                    if (res)
+                        y2[static_cast<size_t>(bb) * ldy2 + n] =
+                            add_h(half_bits_to_float(res[static_cast<size_t>(bb) * ldres + n]), half_bits_to_float(yv));
+                }
+            }
+        }
+    }
+}
+
+// m[b][j] = fp16(silu(g) * u) with g = gu[b][j], u = gu[b][F + j].
+__global__ void __launch_bounds__(256) silu_mul_kernel(const uint16_t* __restrict__ gu, int F, int B,
+                                                       uint16_t* __restrict__ m)
+{
+    const int total = B * F;
+    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x) {
+        const int b = i / F, j = i - b * F;
+        const float gf = half_bits_to_float(gu[static_cast<size_t>(b) * 2 * F + j]);
+        const float uf = half_bits_to_float(gu[static_cast<size_t>(b) * 2 * F + F + j]);
+        m[i] = float_to_half_bits(gf / (1.f + expf(-gf)) * uf);
+    }
+}
+
 // ---------------------------------------------------------------- host --
 
 struct Layout {
-    size_t header, mats, llA, llX1, llM, llX, llV, pV, pX2, pQKV, pO, pX1, pGU, pM, pD, x_stage, logits_stage, total;
+    size_t header, mats, llA, llX1, llM, llX, llV, pV, pX2, pQKV, pO, pX1, pGU, pM, pD, x_stage, logits_stage, rfac,
+        total;
     size_t ll_begin, ll_end;
 };
 
@@ -731,6 +848,7 @@ Layout make_layout(const Dims& d)
     y.pD = take(2 * L * B * H);
     y.x_stage = take(2 * B * H);
     y.logits_stage = take(2 * B * static_cast<size_t>(d.V));
+    y.rfac = take(4 * (3 * L + 1) * B);   // RMS factors of the graph path: [L][3][B] + [B]
     y.total = o;
     return y;
 }
@@ -742,10 +860,11 @@ struct Plan {
     Layout lay;
     int device;
     int grid;
-    int nslots;
+    int nslots, nbars;
     uint32_t slot_bytes, x_bytes;
     size_t smem;
     int nw;
+    cudaGraphExec_t graph;   // graph path (batch > kMaxChainBatch), else null
 };
 
 std::mutex g_plan_mu;
@@ -810,11 +929,106 @@ uint32_t choose_slot_bytes(const Dims& d)
     return static_cast<uint32_t>(best);
 }
 
+int full_bars(int nslots)
+{
+    return (kFullBars / nslots) * nslots;
+}
+
+// True when no consumer wait on the ring can alias: for every stage,
+// nslots + ceil(NW / items per slot) <= the number of full barriers.
+bool ring_ok(const Dims& d, int nslots, uint32_t slot_bytes, int nw)
+{
+    const size_t rowH = static_cast<size_t>(d.H) / 2 + d.H / 16, rowF = static_cast<size_t>(d.F) / 2 + d.F / 16;
+    const size_t items[5] = {2 * rowH, 2 * rowH, 4 * rowH, 2 * rowF, 4 * rowH};
+    for (size_t item : items) {
+        size_t ips = slot_bytes / item;
+        if (ips < 1) ips = 1;
+        if (static_cast<size_t>(nslots) + (nw + ips - 1) / ips > static_cast<size_t>(full_bars(nslots))) return false;
+    }
+    return true;
+}
+
+// Records one token of the graph path on `cs`: every stage kernel of every
+// layer, reading the token input from the workspace staging area and writing
+// the logits to the workspace logits area.
+void record_graph_token(const wq4_layer_table* t, const Dims& d, const Layout& y, int sms, cudaStream_t cs)
+{
+    uint8_t* ws = static_cast<uint8_t*>(t->workspace);
+    const int B = d.B, H = d.H, F = d.F, L = d.L;
+    auto U16 = [&](size_t off) { return reinterpret_cast<uint16_t*>(ws + off); };
+    float* rf = reinterpret_cast<float*>(ws + y.rfac);
+    const size_t LH = static_cast<size_t>(B) * H;
+    auto gemv = [&](const wq4_mat& m, int N, int K, const uint16_t* x, int ldx, const float* r, uint16_t* out, int ldy,
+                    const uint16_t* res, uint16_t* out2) {
+        int grid = (N + 7) / 8;
+        if (grid > sms * 8) grid = sms * 8;
+        stage_gemv_kernel<8><<<grid, 256, 0, cs>>>(m.W, m.s, N, K, x, ldx, B, r, out, ldy, res, H, out2, H);
+    };
+    for (int l = 0; l < L; ++l) {
+        const wq4_layer& ly = t->layers[l];
+        const uint16_t* u = (l == 0) ? U16(y.x_stage) : U16(y.pX2) + static_cast<size_t>(l - 1) * LH;
+        float* r = rf + static_cast<size_t>(3 * l) * B;
+        uint16_t* v = U16(y.pV) + static_cast<size_t>(l) * LH;
+        uint16_t* qkv = U16(y.pQKV) + static_cast<size_t>(l) * B * d.Nqkv;
+        uint16_t* o = U16(y.pO) + static_cast<size_t>(l) * LH;
+        uint16_t* x1 = U16(y.pX1) + static_cast<size_t>(l) * LH;
+        uint16_t* gu = U16(y.pGU) + static_cast<size_t>(l) * B * 2 * F;
+        uint16_t* m = U16(y.pM) + static_cast<size_t>(l) * B * F;
+        uint16_t* dn = U16(y.pD) + static_cast<size_t>(l) * LH;
+        uint16_t* x2 = U16(y.pX2) + static_cast<size_t>(l) * LH;
+        rms_rows_kernel<<<B, 256, 0, cs>>>(u, H, H, t->rms_eps, r, v, H);
+        gemv(ly.qkv, d.Nqkv, H, u, H, r, qkv, d.Nqkv, nullptr, nullptr);
+        rms_rows_kernel<<<B, 256, 0, cs>>>(qkv, d.Nqkv, H, t->rms_eps, r + B, nullptr, 0);
+        gemv(ly.o, H, H, qkv, d.Nqkv, r + B, o, H, v, x1);
+        rms_rows_kernel<<<B, 256, 0, cs>>>(x1, H, H, t->rms_eps, r + 2 * B, nullptr, 0);
+        gemv(ly.gate_up, 2 * F, H, x1, H, r + 2 * B, gu, 2 * F, nullptr, nullptr);
+        silu_mul_kernel<<<sms * 4, 256, 0, cs>>>(gu, F, B, m);
+        gemv(ly.down, H, F, m, F, nullptr, dn, H, x1, x2);
+    }
+    const uint16_t* xl = U16(y.pX2) + static_cast<size_t>(L - 1) * LH;
+    float* r = rf + static_cast<size_t>(3 * L) * B;
+    rms_rows_kernel<<<B, 256, 0, cs>>>(xl, H, H, t->rms_eps, r, U16(y.pV) + static_cast<size_t>(L) * LH, H);
+    gemv(t->lm_head, d.V, H, xl, H, r, U16(y.logits_stage), d.V, nullptr, nullptr);
+}
+
+int build_graph_plan(const wq4_layer_table* t, const Dims& d, const Layout& lay, int dev, const DeviceInfo* di,
+                     Plan* pl)
+{
+    cudaStream_t cs = nullptr;
+    if (cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking) != cudaSuccess) return WQ4_ERR_CUDA;
+    cudaGraph_t graph = nullptr;
+    cudaGraphExec_t exec = nullptr;
+    int rc = WQ4_ERR_CUDA;
+    if (cudaStreamBeginCapture(cs, cudaStreamCaptureModeThreadLocal) == cudaSuccess) {
+        record_graph_token(t, d, lay, di->sm_count, cs);
+        if (cudaStreamEndCapture(cs, &graph) == cudaSuccess && graph &&
+            cudaGraphInstantiate(&exec, graph, 0) == cudaSuccess)
+            rc = WQ4_OK;
+    }
+    if (graph) cudaGraphDestroy(graph);
+    cudaStreamDestroy(cs);
+    if (rc != WQ4_OK) return rc;
+    pl->table = *t;
+    pl->layers.assign(t->layers, t->layers + d.L);
+    pl->dims = d;
+    pl->lay = lay;
+    pl->device = dev;
+    pl->grid = di->sm_count;
+    pl->nslots = 0;
+    pl->nbars = 0;
+    pl->slot_bytes = 0;
+    pl->x_bytes = 0;
+    pl->smem = 0;
+    pl->nw = 0;
+    pl->graph = exec;
+    return WQ4_OK;
+}
+
 int build_plan(const wq4_layer_table* t, Plan* pl, cudaStream_t stream)
 {
     Dims d;
     if (!table_dims(t, &d)) return WQ4_ERR_INVALID;
-    if (d.B > kMaxChainBatch) return WQ4_ERR_UNSUPPORTED;
+    pl->graph = nullptr;
     for (int l = 0; l < d.L; ++l) {
         const wq4_layer& ly = t->layers[l];
         if (!mat_ok(ly.qkv) || !mat_ok(ly.o) || !mat_ok(ly.gate_up) || !mat_ok(ly.down)) return WQ4_ERR_INVALID;
@@ -826,14 +1040,21 @@ int build_plan(const wq4_layer_table* t, Plan* pl, cudaStream_t stream)
     int dev = 0;
     const DeviceInfo* di = current_device_info(&dev);
     if (!di) return WQ4_ERR_CUDA;
+    if (d.B > kMaxChainBatch) {
+        if (d.Nqkv % 8) return WQ4_ERR_UNSUPPORTED;   // the O stage reads qkv rows with 16-byte loads
+        return build_graph_plan(t, d, lay, dev, di, pl);
+    }
     if (!di->coop_launch) return WQ4_ERR_UNSUPPORTED;
     const uint32_t x_bytes = static_cast<uint32_t>(align_up(static_cast<size_t>(d.B) * 2 * (d.H > d.F ? d.H : d.F), 128));
     const uint32_t slot_bytes = choose_slot_bytes(d);
     const int header = chain_header_bytes(chain_warps(d.B), d.B);
     const long avail = static_cast<long>(di->smem_optin) - header - static_cast<long>(x_bytes);
     int nslots = avail > 0 ? static_cast<int>(avail / slot_bytes) : 0;
-    if (nslots < 2) return WQ4_ERR_UNSUPPORTED;
     if (nslots > kChainMaxSlots) nslots = kChainMaxSlots;
+    // fewer slots give more full barriers per slot: take the deepest ring
+    // whose barriers cannot alias
+    while (nslots >= 2 && !ring_ok(d, nslots, slot_bytes, chain_warps(d.B))) --nslots;
+    if (nslots < 2) return WQ4_ERR_UNSUPPORTED;
     const size_t smem = header + x_bytes + static_cast<size_t>(nslots) * slot_bytes;
     // The limit is a property of the kernel, shared by every plan: set it to
     // the device maximum so that no plan's launch depends on which plan was
@@ -872,6 +1093,7 @@ int build_plan(const wq4_layer_table* t, Plan* pl, cudaStream_t stream)
     pl->device = dev;
     pl->grid = di->sm_count;
     pl->nslots = nslots;
+    pl->nbars = full_bars(nslots);
     pl->slot_bytes = slot_bytes;
     pl->x_bytes = x_bytes;
     pl->smem = smem;
@@ -885,6 +1107,18 @@ int launch_chain(const Plan& pl, const uint16_t* x, uint16_t* logits, cudaStream
 {
     uint8_t* ws = static_cast<uint8_t*>(pl.table.workspace);
     const Layout& y = pl.lay;
+    if (pl.graph) {
+        // the graph reads the token from and writes the logits to the workspace
+        uint16_t* xs = reinterpret_cast<uint16_t*>(ws + y.x_stage);
+        uint16_t* ls = reinterpret_cast<uint16_t*>(ws + y.logits_stage);
+        const size_t xb = static_cast<size_t>(pl.dims.B) * pl.dims.H * 2;
+        const size_t lb = static_cast<size_t>(pl.dims.B) * pl.dims.V * 2;
+        if (x != xs && cudaMemcpyAsync(xs, x, xb, cudaMemcpyDeviceToDevice, stream) != cudaSuccess) return WQ4_ERR_CUDA;
+        if (cudaGraphLaunch(pl.graph, stream) != cudaSuccess) return WQ4_ERR_CUDA;
+        if (logits != ls && cudaMemcpyAsync(logits, ls, lb, cudaMemcpyDeviceToDevice, stream) != cudaSuccess)
+            return WQ4_ERR_CUDA;
+        return WQ4_OK;
+    }
     ChainParams p;
     p.mats = reinterpret_cast<const DevMat*>(ws + y.mats);
     p.L = pl.dims.L;
@@ -912,6 +1146,7 @@ int launch_chain(const Plan& pl, const uint16_t* x, uint16_t* logits, cudaStream
     p.pM = reinterpret_cast<uint16_t*>(ws + y.pM);
     p.pD = reinterpret_cast<uint16_t*>(ws + y.pD);
     p.nslots = pl.nslots;
+    p.nbars = pl.nbars;
     p.slot_bytes = pl.slot_bytes;
     p.x_bytes = pl.x_bytes;
     p.err = status_word();
@@ -954,6 +1189,11 @@ int get_plan(const wq4_layer_table* t, Plan* out, cudaStream_t stream)
     Plan pl;
     const int rc = build_plan(t, &pl, stream);
     if (rc != WQ4_OK) return rc;
+    if (it != g_plans.end() && it->second.graph) {
+        // a replaced graph may still run on the GPU: free it once it is done
+        cudaStreamSynchronize(stream);
+        cudaGraphExecDestroy(it->second.graph);
+    }
     g_plans[t] = pl;
     *out = pl;
     return WQ4_OK;
@@ -1009,7 +1249,11 @@ extern "C" int wq4_decode_chain_host(const wq4_layer_table* table, const uint16_
 extern "C" int wq4_chain_plan_destroy(const wq4_layer_table* table)
 {
     std::lock_guard<std::mutex> lock(g_plan_mu);
-    return g_plans.erase(table) ? WQ4_OK : WQ4_ERR_INVALID;
+    auto it = g_plans.find(table);
+    if (it == g_plans.end()) return WQ4_ERR_INVALID;
+    if (it->second.graph) cudaGraphExecDestroy(it->second.graph);
+    g_plans.erase(it);
+    return WQ4_OK;
 }
 
 extern "C" int wq4_chain_trace_offsets(const wq4_layer_table* table, int layer, wq4_chain_trace* out)

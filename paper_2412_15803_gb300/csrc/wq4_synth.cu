@@ -27,12 +27,26 @@ uint64_t stream_key(uint64_t seed, uint64_t sid)
     return mix64(seed * kGamma + sid * kSidMul);
 }
 
-__global__ void codes_kernel(uint32_t* __restrict__ W, int64_t pair_start, int64_t npairs, uint64_t key)
+// Every 4-bit field equal to 15 becomes 7 (bit 3 cleared where all four bits
+// are set): codes 0..14 with mean 7.
+__device__ __forceinline__ uint32_t fold15(uint32_t w)
+{
+    const uint32_t m = w & (w >> 1) & (w >> 2) & (w >> 3) & 0x11111111u;
+    return w ^ (m << 3);
+}
+
+__global__ void codes_kernel(uint32_t* __restrict__ W, int64_t pair_start, int64_t npairs, uint64_t key,
+                             int symmetric)
 {
     for (int64_t t = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < npairs;
          t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
         const uint64_t v = mix64(key + static_cast<uint64_t>(pair_start + t + 1) * kGamma);
-        reinterpret_cast<uint2*>(W)[t] = make_uint2(static_cast<uint32_t>(v), static_cast<uint32_t>(v >> 32));
+        uint32_t lo = static_cast<uint32_t>(v), hi = static_cast<uint32_t>(v >> 32);
+        if (symmetric) {
+            lo = fold15(lo);
+            hi = fold15(hi);
+        }
+        reinterpret_cast<uint2*>(W)[t] = make_uint2(lo, hi);
     }
 }
 
@@ -60,14 +74,14 @@ int grid_for(int64_t n)
 }  // namespace
 
 extern "C" int wq4_synth_codes(uint32_t* W, int64_t word_start, int64_t nwords, uint64_t seed, uint64_t sid,
-                               void* stream)
+                               int symmetric, void* stream)
 {
     if (!W || word_start < 0 || nwords < 0 || (word_start % 2) || (nwords % 2)) return -1;
     if (reinterpret_cast<uintptr_t>(W) % 8) return -1;
     if (nwords == 0) return 0;
     const int64_t npairs = nwords / 2;
     codes_kernel<<<grid_for(npairs), 256, 0, static_cast<cudaStream_t>(stream)>>>(W, word_start / 2, npairs,
-                                                                                  stream_key(seed, sid));
+                                                                                  stream_key(seed, sid), symmetric);
     return cudaGetLastError() == cudaSuccess ? 0 : -4;
 }
 

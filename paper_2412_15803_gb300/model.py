@@ -54,8 +54,9 @@ SHAPE_8B = ModelShape("8b", 32, 4096, 14336, 32, 8, 128, 128256)
 SHAPES = {"3b": SHAPE_3B, "8b": SHAPE_8B}
 
 
-def fill_matrix(W, s, N: int, K: int, seed: int, layer: int, mat: int, stream=None) -> None:
-    _w.wq4_synth_codes(W, 0, N * K // 8, seed, synth.stream_id(synth.KIND_CODES, layer, mat), stream)
+def fill_matrix(W, s, N: int, K: int, seed: int, layer: int, mat: int, symmetric: bool = False,
+                stream=None) -> None:
+    _w.wq4_synth_codes(W, 0, N * K // 8, seed, synth.stream_id(synth.KIND_CODES, layer, mat), symmetric, stream)
     _w.wq4_synth_scales(s, 0, N * K // 32, seed, synth.stream_id(synth.KIND_SCALES, layer, mat),
                         synth.SCALE_LO, synth.SCALE_HI, stream)
 
@@ -75,14 +76,14 @@ class DecodeModel:
             for name, N, K, mat in shape.mats(l):
                 W = torch.empty((N, K // 8), dtype=torch.int32, device=dev)
                 s = torch.empty((N, K // 32), dtype=torch.int16, device=dev)
-                fill_matrix(W, s, N, K, seed, l, mat)
+                fill_matrix(W, s, N, K, seed, l, mat, symmetric=True)
                 d[name] = (W, s)
                 setattr(layers[l], name, _w.wq4_mat(W.data_ptr(), s.data_ptr()))
             self.weights.append(d)
         V, H = shape.vocab, shape.hidden
         W = torch.empty((V, H // 8), dtype=torch.int32, device=dev)
         s = torch.empty((V, H // 32), dtype=torch.int16, device=dev)
-        fill_matrix(W, s, V, H, seed, shape.num_layers, synth.MAT_LM_HEAD)
+        fill_matrix(W, s, V, H, seed, shape.num_layers, synth.MAT_LM_HEAD, symmetric=True)
         self.lm_head = (W, s)
         self._layers = layers
         t = _w.wq4_layer_table()
@@ -136,4 +137,4 @@ class DecodeModel:
             N, K, mat, lay = sh.vocab, sh.hidden, synth.MAT_LM_HEAD, sh.num_layers
         else:
             (N, K, mat), lay = [(N, K, m) for nm, N, K, m in sh.mats(layer) if nm == name][0], layer
-        return synth.matrix(self.seed, N, K, lay, mat, row_start, nrows)
+        return synth.matrix(self.seed, N, K, lay, mat, row_start, nrows, symmetric=True)

@@ -18,7 +18,12 @@ Streams (sid) name one tensor each; see ``stream_id``.
 
 Drawn tensors (the distributions of the 1-8B 4-bit decode workloads):
   * packed codes: uint32 words; word 2m is the low half and word 2m+1 the high
-    half of u64(m), so every 4-bit code is uniform on 0..15;
+    half of u64(m), so every 4-bit code is uniform on 0..15.  The symmetric
+    draw then turns every code 15 into 7: codes 0..14 with mean 7, the range
+    of symmetric 4-bit quantisation (|q - 7| <= 7) and zero-mean weights as in
+    trained models.  Whole synthetic models use it (with codes uniform on
+    0..15, q - 7 has mean 1/2 and the fp16 activations of a deep chain
+    overflow); single-matrix tests use the full range;
   * scales: fp16_RNE(lo + (hi - lo) * u), u = (u64(i) >> 11) * 2^-53,
     evaluated in fp64 as one multiply then one add, lo = 0.005, hi = 0.02;
   * activations: fp16_RNE(sqrt(-2 ln u1) * cos(2 pi u2)) (Box-Muller) with
@@ -85,14 +90,23 @@ def u64(k: int, start: int, count: int) -> np.ndarray:
     return _mix64(z)
 
 
-def codes_words(seed: int, sid: int, word_start: int, nwords: int) -> np.ndarray:
+def fold15(words: np.ndarray) -> np.ndarray:
+    """Every 4-bit field equal to 15 becomes 7 (bit 3 cleared where all four
+    bits are set)."""
+    w = words.astype(np.uint32)
+    m = w & (w >> np.uint32(1)) & (w >> np.uint32(2)) & (w >> np.uint32(3)) & np.uint32(0x11111111)
+    return w ^ (m << np.uint32(3))
+
+
+def codes_words(seed: int, sid: int, word_start: int, nwords: int, symmetric: bool = False) -> np.ndarray:
     """Packed-code words [word_start, word_start + nwords) of a stream (uint32).
 
     word_start and nwords must be even (two words per 64-bit draw)."""
     if word_start % 2 or nwords % 2:
         raise ValueError("codes are drawn two words at a time")
     v = u64(key(seed, sid), word_start // 2, nwords // 2)
-    return v.view(np.uint32).copy()  # little endian: low half first
+    w = v.view(np.uint32).copy()  # little endian: low half first
+    return fold15(w) if symmetric else w
 
 
 def scales_fp16(seed: int, sid: int, start: int, count: int,
@@ -114,7 +128,7 @@ def normal_fp16(seed: int, sid: int, count: int) -> np.ndarray:
 
 
 def matrix(seed: int, N: int, K: int, layer: int = 0, mat: int = 0,
-           row_start: int = 0, nrows: int | None = None):
+           row_start: int = 0, nrows: int | None = None, symmetric: bool = False):
     """Rows [row_start, row_start + nrows) of one N x K packed matrix.
 
     Returns (W uint32 [nrows][K/8], s uint16 [nrows][K/32]).  Row blocks of
@@ -123,7 +137,7 @@ def matrix(seed: int, N: int, K: int, layer: int = 0, mat: int = 0,
     if nrows is None:
         nrows = N - row_start
     wpr, gpr = K // 8, K // 32
-    W = codes_words(seed, stream_id(KIND_CODES, layer, mat), row_start * wpr, nrows * wpr)
+    W = codes_words(seed, stream_id(KIND_CODES, layer, mat), row_start * wpr, nrows * wpr, symmetric)
     s = scales_fp16(seed, stream_id(KIND_SCALES, layer, mat), row_start * gpr, nrows * gpr)
     return W.reshape(nrows, wpr), s.reshape(nrows, gpr)
 

@@ -86,7 +86,7 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
     L.wq4_chain_plan_destroy.argtypes = [ctypes.POINTER(wq4_layer_table)]
     L.wq4_chain_trace_offsets.argtypes = [ctypes.POINTER(wq4_layer_table), _I,
                                           ctypes.POINTER(wq4_chain_trace)]
-    L.wq4_synth_codes.argtypes = [_P, _I64, _I64, _U64, _U64, _P]
+    L.wq4_synth_codes.argtypes = [_P, _I64, _I64, _U64, _U64, _I, _P]
     L.wq4_synth_scales.argtypes = [_P, _I64, _I64, _U64, _U64, ctypes.c_double, ctypes.c_double, _P]
     _lib = L
     return L
@@ -186,8 +186,9 @@ def wq4_chain_trace_offsets(table: wq4_layer_table, layer: int) -> wq4_chain_tra
     return out
 
 
-def wq4_synth_codes(W, word_start: int, nwords: int, seed: int, sid: int, stream=None) -> None:
-    rc = load().wq4_synth_codes(_ptr(W), word_start, nwords, seed, sid, _stream(stream))
+def wq4_synth_codes(W, word_start: int, nwords: int, seed: int, sid: int, symmetric: bool = False,
+                    stream=None) -> None:
+    rc = load().wq4_synth_codes(_ptr(W), word_start, nwords, seed, sid, int(bool(symmetric)), _stream(stream))
     if rc != 0:
         raise Wq4Error("wq4_synth_codes", rc)
 

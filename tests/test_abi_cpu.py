@@ -131,6 +131,6 @@ def test_chain_rejects_null_and_misaligned_io():
 
 def test_synth_rejects_bad_arguments():
     L = wq4.load()
-    assert L.wq4_synth_codes(A16, 1, 4, 0, 0, None) == -1
-    assert L.wq4_synth_codes(A16, 0, 3, 0, 0, None) == -1
+    assert L.wq4_synth_codes(A16, 1, 4, 0, 0, 0, None) == -1
+    assert L.wq4_synth_codes(A16, 0, 3, 0, 0, 1, None) == -1
     assert L.wq4_synth_scales(None, 0, 4, 0, 0, 0.005, 0.02, None) == -1

@@ -13,7 +13,7 @@ import torch
 import oracle
 from oracle import chain as ochain
 from paper_2412_15803_gb300 import synth
-from paper_2412_15803_gb300.model import SHAPE_3B, DecodeModel, ModelShape
+from paper_2412_15803_gb300.model import SHAPE_3B, SHAPE_8B, DecodeModel, ModelShape
 
 pytestmark = pytest.mark.gpu
 
@@ -101,8 +101,9 @@ def check_logits(model, logits, rows=None):
     within(logits[:, idx], y, A, "lm_head")
 
 
-@pytest.mark.parametrize("batch", [1, 2, 3, 4])
+@pytest.mark.parametrize("batch", [1, 2, 3, 4, 5, 8, 32])
 def test_tiny_chain_every_stage_every_element(batch):
+    """Batch 1-4: the persistent kernel; 5-32: the graph of stage kernels."""
     model = DecodeModel(TINY, batch=batch, seed=batch)
     x = synth.activations(100 + batch, batch, TINY.hidden)
     logits = run(model, x)
@@ -187,6 +188,28 @@ def test_3b_chain_full_size_sampled():
     assert np.array_equal(run(model, x), logits)
 
 
+def test_8b_chain_batch4_full_size_sampled():
+    """The 32-layer 8B-shaped chain at batch 4: the shallowest weight ring
+    (six slots for seven consumer warps, one down-projection item per slot),
+    so consumer warps run furthest ahead of the producer.  Sampled rows of
+    three layers and of the LM head, and twenty tokens with identical bits."""
+    sh = SHAPE_8B
+    model = DecodeModel(sh, batch=4, seed=3)
+    x = synth.activations(5, 4, sh.hidden)
+    logits = run(model, x)
+    rng = np.random.default_rng(1)
+
+    def pick(N):
+        return np.unique(np.concatenate([[0, 1, N - 2, N - 1], rng.integers(0, N, 16)]))
+
+    for l in (0, 17, 31):
+        rows = dict(qkv=pick(sh.n_qkv), o=pick(sh.hidden), gate_up=pick(2 * sh.ffn), down=pick(sh.hidden))
+        check_stages(model, l, rows, u=x if l == 0 else None)
+    check_logits(model, logits, rows=pick(sh.vocab))
+    for _ in range(20):
+        assert np.array_equal(run(model, x), logits)
+
+
 def test_two_models_with_different_rings_alternate():
     """Plans of different shapes (different shared-memory rings) stay valid
     whichever plan was built last."""
@@ -199,3 +222,19 @@ def test_two_models_with_different_rings_alternate():
     assert np.array_equal(run(a, xa), la)
     assert np.array_equal(run(b, xb), lb)
     check_logits(a, la)
+
+
+@pytest.mark.parametrize("batch", [6, 16])
+def test_small_chain_graph_path_repeat_and_rebuild(batch):
+    model = DecodeModel(SMALL, batch=batch, seed=60 + batch)
+    x = synth.activations(61, batch, SMALL.hidden)
+    a = run(model, x)
+    assert np.array_equal(run(model, x), a)          # graph replays are deterministic
+    for l in range(SMALL.num_layers):
+        check_stages(model, l, u=x if l == 0 else None)
+    check_logits(model, a)
+    lh = np.zeros((batch, SMALL.vocab), np.uint16)
+    model.decode_host(np.ascontiguousarray(x), lh)
+    assert np.array_equal(lh, a)
+    model.destroy_plan()
+    assert np.array_equal(run(model, x), a)          # a new plan and graph give the same bits

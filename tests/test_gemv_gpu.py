@@ -185,6 +185,11 @@ def test_device_generator_matches_host_bit_exact():
     W, s = synth.matrix(77, N, K, 3, synth.MAT_DOWN)
     assert np.array_equal(Wd.cpu().numpy().view(np.uint32), W)
     assert np.array_equal(sd.cpu().numpy().view(np.uint16), s)
+    # the symmetric draw of whole models, over an offset block of words
+    Wsym = torch.empty(4096, dtype=torch.int32, device="cuda")
+    wq4.wq4_synth_codes(Wsym, 2 * 777, 4096, 77, 9, symmetric=True)
+    torch.cuda.synchronize()
+    assert np.array_equal(Wsym.cpu().numpy().view(np.uint32), synth.codes_words(77, 9, 2 * 777, 4096, symmetric=True))
     # an offset block through the C ABI directly
     part = torch.empty(1000, dtype=torch.int16, device="cuda")
     wq4.wq4_synth_scales(part, 123457, 1000, 77, 5, 0.005, 0.02)

@@ -36,6 +36,23 @@ def test_draw_distributions():
     assert abs(x.mean()) < 0.03 and abs(x.std() - 1.0) < 0.02
 
 
+def test_symmetric_code_draw():
+    # fold15 on patterns with every field value: only fields equal to 15 change, to 7
+    w = np.array([0xFFFFFFFF, 0xF0F0F0F0, 0xEDCBA987, 0x76543210, 0x8F7F0FEF], np.uint32)
+    assert [int(v) for v in synth.fold15(w)] == [0x77777777, 0x70707070, 0xEDCBA987, 0x76543210, 0x877707E7]
+    # the draw: the full-range words with fields 15 folded; codes 0..14 with
+    # P(7) = 2/16, the others 1/16, so the mean of q - 7 is 0
+    full = synth.codes_words(4, 11, 0, 1 << 18)
+    sym = synth.codes_words(4, 11, 0, 1 << 18, symmetric=True)
+    assert np.array_equal(sym, synth.fold15(full))
+    nib = np.stack([(sym >> np.uint32(4 * i)) & np.uint32(0xF) for i in range(8)], -1).ravel().astype(np.int64)
+    counts = np.bincount(nib, minlength=16) / nib.size
+    assert counts[15] == 0
+    assert abs(counts[7] - 2 / 16) < 0.002
+    assert np.all(np.abs(np.delete(counts[:15], 7) - 1 / 16) < 0.002)
+    assert abs((nib - 7).mean()) < 0.01
+
+
 def test_oracle_matches_stored_fixtures():
     lines = [l.split() for l in open(GOLDEN) if l.strip() and not l.startswith("#")]
     i = 0

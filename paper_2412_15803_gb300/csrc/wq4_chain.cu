@@ -62,7 +62,9 @@ constexpr uint32_t kSlotRelease = 1024;
 // then the weight ring.
 constexpr int kHdrRed = 512;                 // float red[16][kMaxChainBatch]
 static_assert(8 * (kFullBars + kChainMaxSlots) <= kHdrRed, "mbarriers overlap the header");
-constexpr int kHdrEpoch = 768;
+constexpr int kHdrEpoch = 768;               // uint32 epoch, then int vw0, vw1 (the CTA's slice of v)
+constexpr int kHdrInfo = 784;                // StageInfo info[5], one per stage type
+constexpr int kHdrWofs = 944;                // uint8 wofs[5][16]: a warp's first chunk within a stage
 constexpr int kHdrRes = 1024;                // uint32 res[kMaxResWords]: prefetched residual words
 constexpr int kMaxResWords = 1024;
 __host__ __device__ constexpr int chain_header_bytes(int, int)
@@ -162,6 +164,16 @@ __device__ __forceinline__ ChunkLayout chunk_layout(const Stage& g, int ia, int 
     return c;
 }
 
+// What one CTA does in every stage of one type, computed once per launch so
+// that no stage pays for integer divisions: items [i0, i1), items per ring
+// slot, the number of chunks, and that number modulo the slot and barrier
+// counts (flip: parity changes of the barrier ring beyond the wrap).
+struct StageInfo {
+    int i0, i1, ips, nchunks, nmod_slots, nmod_bars, flip, pad;
+};
+static_assert(kHdrInfo + 5 * sizeof(StageInfo) <= kHdrWofs, "stage table overlaps the header");
+static_assert(kHdrWofs + 5 * 16 <= kHdrRes, "warp table overlaps the header");
+
 __device__ __forceinline__ void cta_items(int items, int* i0, int* i1)
 {
     *i0 = static_cast<int>(static_cast<int64_t>(blockIdx.x) * items / gridDim.x);
@@ -173,6 +185,12 @@ __device__ __forceinline__ int items_per_slot(const ChainParams& p, const Stage&
     const uint32_t item_bytes = static_cast<uint32_t>(g.rpi) * (g.K / 2 + g.K / 16);
     const int ips = static_cast<int>(p.slot_bytes / item_bytes);
     return ips < 1 ? 1 : ips;
+}
+
+// A representative stage of each type (layer 0, or the LM head).
+__device__ __forceinline__ int stage_of_type(const ChainParams& p, int t)
+{
+    return t == kLM ? 4 * p.L : t;
 }
 
 // ------------------------------------------------------- flagged words --
@@ -413,6 +431,8 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
     float* red = reinterpret_cast<float*>(smem + kHdrRed);          // [NW][kMaxChainBatch]
     uint32_t* epoch_sh = reinterpret_cast<uint32_t*>(smem + kHdrEpoch);
     uint32_t* res = reinterpret_cast<uint32_t*>(smem + kHdrRes);    // [B][items of the CTA]
+    StageInfo* info = reinterpret_cast<StageInfo*>(smem + kHdrInfo);
+    uint8_t* wofs_tab = smem + kHdrWofs;
     constexpr int kHeader = chain_header_bytes(NW, B);
     uint4* xs = reinterpret_cast<uint4*>(smem + kHeader);
     uint8_t* slots = smem + kHeader + p.x_bytes;
@@ -429,6 +449,27 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
         uint32_t s;
         asm volatile("ld.relaxed.gpu.global.b32 %0, [%1];" : "=r"(s) : "l"(p.seq) : "memory");
         *epoch_sh = s + 1u;
+        // the CTA's slice of the normalised input v that it publishes
+        const int nw = p.H / 2;
+        epoch_sh[1] = static_cast<int>(static_cast<int64_t>(blockIdx.x) * nw / gridDim.x);
+        epoch_sh[2] = static_cast<int>(static_cast<int64_t>(blockIdx.x + 1) * nw / gridDim.x);
+    }
+    if (threadIdx.x >= 32 && threadIdx.x < 32 + 5) {
+        const int t = threadIdx.x - 32;
+        const Stage g = stage_at(p, stage_of_type(p, t));
+        StageInfo in;
+        cta_items(g.items, &in.i0, &in.i1);
+        in.ips = items_per_slot(p, g);
+        in.nchunks = (in.i1 - in.i0 + in.ips - 1) / in.ips;
+        in.nmod_slots = in.nchunks % p.nslots;
+        in.nmod_bars = in.nchunks % p.nbars;
+        in.flip = (in.nchunks / p.nbars) & 1;
+        in.pad = 0;
+        info[t] = in;
+    }
+    if (threadIdx.x >= 64 && threadIdx.x < 64 + 5 * 16) {
+        const int t = (threadIdx.x - 64) >> 4, w = (threadIdx.x - 64) & 15;
+        wofs_tab[t * 16 + w] = static_cast<uint8_t>(w / items_per_slot(p, stage_at(p, stage_of_type(p, t))));
     }
     __syncthreads();
     const uint32_t epoch = *epoch_sh;
@@ -437,20 +478,25 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
         // ------------------------------------------------ producer warp
         if (lane == 0) {
             const uint64_t pol = l2_policy_evict_first();
-            int ord = 0;
+            int ord = 0;                // ring ordinal of the next chunk
+            int slot = 0, round = 0;    // its slot and the slot's use count
+            int fbi = 0;                // its full barrier
             for (int st = 0; st < nstages; ++st) {
                 const Stage g = stage_at(p, st);
-                int i0, i1;
-                cta_items(g.items, &i0, &i1);
-                const int ips = items_per_slot(p, g);
+                const StageInfo in = info[g.type];
+                const int i0 = in.i0, i1 = in.i1, ips = in.ips;
                 const int wpr = g.K >> 3, gpr = g.K >> 5;
                 for (int ia = i0; ia < i1; ia += ips, ++ord) {
                     const int ib = min(i1, ia + ips);
-                    const int slot = ord % p.nslots, round = ord / p.nslots;
                     if (round > 0) mbar_wait(&empty[slot], (round - 1) & 1, p.err);
                     const ChunkLayout c = chunk_layout(g, ia, ib);
                     uint8_t* dst = slots + static_cast<size_t>(slot) * p.slot_bytes;
-                    uint64_t* fb = &full[ord % p.nbars];
+                    uint64_t* fb = &full[fbi];
+                    if (++slot == p.nslots) {
+                        slot = 0;
+                        ++round;
+                    }
+                    if (++fbi == p.nbars) fbi = 0;
                     mbar_arrive_expect_tx(fb, c.codes_bytes + c.scale_bytes);
                     if (g.type == kGU) {
                         const uint32_t hc = c.codes_bytes / 2, hs = c.scale_bytes / 2;
@@ -474,11 +520,13 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
     } else {
         // ------------------------------------------------ consumer warps
         const int H = p.H, F = p.F;
-        int cbase = 0;          // ring ordinal of the stage's first chunk
+        // slot, full barrier and barrier parity of the stage's first chunk
+        int cslot = 0, cbar = 0;
+        uint32_t cpar = 0;
         for (int st = 0; st < nstages; ++st) {
             const Stage g = stage_at(p, st);
-            int i0, i1;
-            cta_items(g.items, &i0, &i1);
+            const StageInfo& in = info[g.type];
+            const int i0 = in.i0, i1 = in.i1;
             if (i1 <= i0) continue;
             const int l = g.layer;
             const int K = g.K, gpr = K >> 5, cpr = K >> 3;
@@ -499,10 +547,10 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
                 if (g.type == kO) rl = p.llV + static_cast<size_t>(l) * B * (H / 2);
                 else if (g.type == kDOWN) rl = p.llX1 + static_cast<size_t>(l) * B * (H / 2);
                 if (rl) {
-                    for (int t = threadIdx.x; t < B * nit; t += kConsumers) {
-                        const int b = t / nit, k = t - b * nit;
-                        res[t] = ll_load(rl + static_cast<size_t>(b) * (H / 2) + i0 + k, epoch, p.err, p.abort);
-                    }
+#pragma unroll
+                    for (int b = 0; b < B; ++b)
+                        for (int k = threadIdx.x; k < nit; k += kConsumers)
+                            res[b * nit + k] = ll_load(rl + static_cast<size_t>(b) * (H / 2) + i0 + k, epoch, p.err, p.abort);
                 }
                 float ss[B];
 #pragma unroll
@@ -570,41 +618,43 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
             for (int b = 0; b < B; ++b) {
                 // the same sum, in the same order, in every warp and every CTA
                 const float t = warp_sum(lane < NW ? red[lane * kMaxChainBatch + b] : 0.f);
-                rf[b] = (g.type == kDOWN) ? 1.f : 1.f / sqrtf(t / static_cast<float>(K) + p.eps);
+                rf[b] = (g.type == kDOWN) ? 1.f : rsqrtf(t / static_cast<float>(K) + p.eps);
             }
             if (g.type == kQKV || g.type == kLM) {
                 // the normalised layer input v = fp16(r * u) is kept for the
                 // residual stream (and the trace): every CTA publishes its
                 // slice of it; the projections below use r as a row factor
-                const int nw = H / 2;                       // words of v per batch row
-                const int w0 = static_cast<int>(static_cast<int64_t>(blockIdx.x) * nw / gridDim.x);
-                const int w1 = static_cast<int>(static_cast<int64_t>(blockIdx.x + 1) * nw / gridDim.x);
+                const int w0 = static_cast<int>(epoch_sh[1]), w1 = static_cast<int>(epoch_sh[2]);
                 const uint32_t* xw = reinterpret_cast<const uint32_t*>(xs);
-                for (int t = threadIdx.x; t < B * (w1 - w0); t += kConsumers) {
-                    const int b = t / (w1 - w0), w = w0 + (t - b * (w1 - w0));
-                    const int c = w >> 2;                   // chunk of the word
-                    const uint32_t u = xw[4 * (b * cpr + x_chunk(c >> 2, c & 3)) + (w & 3)];
-                    float r = rf[0];
 #pragma unroll
-                    for (int bb = 1; bb < B; ++bb)
-                        if (bb == b) r = rf[bb];
-                    const uint32_t v = pack2(float_to_half_bits(r * lo_f(u)), float_to_half_bits(r * hi_f(u)));
-                    reinterpret_cast<uint32_t*>(p.pV + (static_cast<size_t>(l) * B + b) * H)[w] = v;
-                    if (g.type == kQKV) ll_store(p.llV + (static_cast<size_t>(l) * B + b) * (H / 2) + w, v, epoch);
+                for (int b = 0; b < B; ++b) {
+                    for (int w = w0 + threadIdx.x; w < w1; w += kConsumers) {
+                        const int c = w >> 2;               // chunk of the word
+                        const uint32_t u = xw[4 * (b * cpr + x_chunk(c >> 2, c & 3)) + (w & 3)];
+                        const uint32_t v = pack2(float_to_half_bits(rf[b] * lo_f(u)), float_to_half_bits(rf[b] * hi_f(u)));
+                        reinterpret_cast<uint32_t*>(p.pV + (static_cast<size_t>(l) * B + b) * H)[w] = v;
+                        if (g.type == kQKV) ll_store(p.llV + (static_cast<size_t>(l) * B + b) * (H / 2) + w, v, epoch);
+                    }
                 }
             }
 
             // -- stream the CTA's items of this stage: item i0 + k goes to warp
             //    k % NW; a warp visits only the chunks that hold its items
-            const int ips = items_per_slot(p, g);
-            const int nchunks = (nit + ips - 1) / ips;
+            const int ips = in.ips;
             const uint4* xl = xs + 4 * lane;
             int it = i0 + warp;
             if (it < i1) {
-                int ia = i0 + (warp / ips) * ips, ib = min(i1, ia + ips);
-                const int o0 = cbase + warp / ips;          // ring ordinal of the first chunk
-                int slot = o0 % p.nslots, bar = o0 % p.nbars;
-                uint32_t par = (o0 / p.nbars) & 1u;
+                // the warp's first chunk: wofs chunks after the stage's first
+                const int wofs = wofs_tab[g.type * 16 + warp];
+                int ia = i0 + wofs * ips, ib = min(i1, ia + ips);
+                int slot = cslot + wofs;
+                while (slot >= p.nslots) slot -= p.nslots;
+                int bar = cbar + wofs;                      // wofs < nbars
+                uint32_t par = cpar;
+                if (bar >= p.nbars) {
+                    bar -= p.nbars;
+                    par ^= 1u;
+                }
                 while (it < i1) {
                     while (it >= ib) {                      // next chunk
                         ia += ips;
@@ -665,7 +715,14 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
                     if (lane == 0) mbar_arrive_count(&empty[slot], arrivals);
                 }
             }
-            cbase += nchunks;
+            cslot += in.nmod_slots;
+            if (cslot >= p.nslots) cslot -= p.nslots;
+            cbar += in.nmod_bars;
+            cpar ^= static_cast<uint32_t>(in.flip);
+            if (cbar >= p.nbars) {
+                cbar -= p.nbars;
+                cpar ^= 1u;
+            }
         }
     }
 

@@ -60,7 +60,7 @@ constexpr uint32_t kSlotRelease = 1024;
 // RMS partial sums | epoch | the residual
 // words of the CTA's rows (O and down stages); then the staged input vector,
 // then the weight ring.
-constexpr int kHdrRed = 512;                 // float red[16][kMaxChainBatch]
+constexpr int kHdrRed = 512;                 // float red[kMaxChainBatch][16]: per-warp sums of squares
 static_assert(8 * (kFullBars + kChainMaxSlots) <= kHdrRed, "mbarriers overlap the header");
 constexpr int kHdrEpoch = 768;               // uint32 epoch, then int vw0, vw1 (the CTA's slice of v)
 constexpr int kHdrInfo = 784;                // StageInfo info[5], one per stage type
@@ -454,6 +454,7 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
         epoch_sh[1] = static_cast<int>(static_cast<int64_t>(blockIdx.x) * nw / gridDim.x);
         epoch_sh[2] = static_cast<int>(static_cast<int64_t>(blockIdx.x + 1) * nw / gridDim.x);
     }
+    if (threadIdx.x < kMaxChainBatch * 16) red[threadIdx.x] = 0.f;   // warps >= NW stay zero
     if (threadIdx.x >= 32 && threadIdx.x < 32 + 5) {
         const int t = threadIdx.x - 32;
         const Stage g = stage_at(p, stage_of_type(p, t));
@@ -609,7 +610,7 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
 #pragma unroll
                 for (int b = 0; b < B; ++b) {
                     const float v = warp_sum(ss[b]);
-                    if (lane == 0) red[warp * kMaxChainBatch + b] = v;
+                    if (lane == 0) red[b * 16 + warp] = v;
                 }
             }
             named_barrier_sync(1, kConsumers);
@@ -617,8 +618,11 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
 #pragma unroll
             for (int b = 0; b < B; ++b) {
                 // the same sum, in the same order, in every warp and every CTA
-                const float t = warp_sum(lane < NW ? red[lane * kMaxChainBatch + b] : 0.f);
-                rf[b] = (g.type == kDOWN) ? 1.f : rsqrtf(t / static_cast<float>(K) + p.eps);
+                const float4* r4 = reinterpret_cast<const float4*>(red + b * 16);
+                const float4 a = r4[0], c = r4[1], d = r4[2], e = r4[3];
+                const float t = (((a.x + a.y) + (a.z + a.w)) + ((c.x + c.y) + (c.z + c.w))) +
+                                (((d.x + d.y) + (d.z + d.w)) + ((e.x + e.y) + (e.z + e.w)));
+                rf[b] = (g.type == kDOWN) ? 1.f : rsqrtf(t * (1.f / static_cast<float>(K)) + p.eps);
             }
             if (g.type == kQKV || g.type == kLM) {
                 // the normalised layer input v = fp16(r * u) is kept for the

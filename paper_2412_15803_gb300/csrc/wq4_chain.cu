@@ -713,7 +713,8 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
                         for (int b = 0; b < B; ++b)
                             if (lane == b)
                                 item_epilogue<B>(p, g, it, b, acc[0][b], acc[1][b], acc[2][b], acc[3][b], rf[b],
-                                                 res[b * nit + (it - i0)], epoch);
+                                                 (g.type == kO || g.type == kDOWN) ? res[b * nit + (it - i0)] : 0u,
+                                                 epoch);
                     }
                     __syncwarp();
                     if (lane == 0) mbar_arrive_count(&empty[slot], arrivals);

@@ -29,6 +29,7 @@
 //    inspection.
 #include "wq4_device.cuh"
 #include "wq4_host.h"
+#include "wq4_tc_host.h"
 #include "wq4.h"
 
 #include <cuda_runtime.h>
@@ -747,110 +748,15 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
 // ------------------------------------------------- graph path (batch 5-32) --
 //
 // For batches beyond what the persistent kernel stages in shared memory, the
-// token runs as a CUDA graph of stage kernels (captured once per plan): RMS
-// factors, a CUDA-core stage GEMV with the row factor, a strided input and a
-// fused residual add, and SiLU(gate) * up.  They write the same workspace
+// token runs as a CUDA graph (captured once per plan) of tensor-core stage
+// kernels and per-stage epilogues (wq4_tc.cu); they write the same workspace
 // traces as the persistent kernel.
-
-// r[b] = 1/sqrt(mean(u[b]^2) + eps) over K fp16 values (row stride ld), one
-// CTA per batch row, summed in a fixed order; optionally v[b] = fp16(r[b] u[b]).
-__global__ void __launch_bounds__(256) rms_rows_kernel(const uint16_t* __restrict__ u, int ld, int K, float eps,
-                                                       float* __restrict__ r, uint16_t* __restrict__ v, int ldv)
-{
-    __shared__ float red[8];
-    const int b = blockIdx.x;
-    const uint16_t* ub = u + static_cast<size_t>(b) * ld;
-    float ss = 0.f;
-    for (int k = threadIdx.x; k < K; k += blockDim.x) {
-        const float t = half_bits_to_float(ub[k]);
-        ss = fmaf(t, t, ss);
-    }
-    ss = warp_sum(ss);
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = ss;
-    __syncthreads();
-    float tot = 0.f;
-#pragma unroll
-    for (int w = 0; w < 8; ++w) tot += red[w];
-    const float rb = 1.f / sqrtf(tot / static_cast<float>(K) + eps);
-    if (threadIdx.x == 0) r[b] = rb;
-    if (v) {
-        uint16_t* vb = v + static_cast<size_t>(b) * ldv;
-        for (int k = threadIdx.x; k < K; k += blockDim.x) vb[k] = float_to_half_bits(rb * half_bits_to_float(ub[k]));
-    }
-}
-
-// y[b][n] = fp16(r[b] * sum_k (q - 7) s x[b][k]) for a warp per row n, batch
-// in tiles of BT; x rows at stride ldx; with `res`, also y2 = fp16(res + y).
-template <int BT>
-__global__ void __launch_bounds__(256) stage_gemv_kernel(const uint32_t* __restrict__ W, const uint16_t* __restrict__ s,
-                                                         int N, int K, const uint16_t* __restrict__ x, int ldx, int B,
-                                                         const float* __restrict__ r, uint16_t* __restrict__ y, int ldy,
-                                                         const uint16_t* __restrict__ res, int ldres,
-                                                         uint16_t* __restrict__ y2, int ldy2)
-{
-    const int lane = threadIdx.x & 31;
-    const int gw = blockIdx.x * (blockDim.x >> 5) + (threadIdx.x >> 5);
-    const int nw = gridDim.x * (blockDim.x >> 5);
-    const int gpr = K >> 5;
-    for (int n = gw; n < N; n += nw) {
-        const uint4* crow = reinterpret_cast<const uint4*>(W + static_cast<size_t>(n) * (K >> 3));
-        const uint16_t* srow = s + static_cast<size_t>(n) * gpr;
-        for (int b0 = 0; b0 < B; b0 += BT) {
-            float acc[BT];
-#pragma unroll
-            for (int b = 0; b < BT; ++b) acc[b] = 0.f;
-            for (int g = lane; g < gpr; g += 32) {
-                const uint4 cw = __ldg(crow + g);
-                const float sc = half_bits_to_float(__ldg(srow + g));
-                uint32_t q[16];
-                unpack_word(cw.x, q + 0);
-                unpack_word(cw.y, q + 4);
-                unpack_word(cw.z, q + 8);
-                unpack_word(cw.w, q + 12);
-#pragma unroll
-                for (int b = 0; b < BT; ++b) {
-                    if (b0 + b < B) {
-                        const uint4* xb = reinterpret_cast<const uint4*>(x + static_cast<size_t>(b0 + b) * ldx) + 4 * g;
-                        const float a01 = fma8(q + 4, __ldg(xb + 1), fma8(q + 0, __ldg(xb + 0), 0.f));
-                        const float a23 = fma8(q + 12, __ldg(xb + 3), fma8(q + 8, __ldg(xb + 2), 0.f));
-                        acc[b] = fmaf(sc, a01 + a23, acc[b]);
-                    }
-                }
-            }
-#pragma unroll
-            for (int b = 0; b < BT; ++b) {
-                const float v = warp_sum(acc[b]);
-                const int bb = b0 + b;
-                if (lane == b && bb < B) {
-                    const uint16_t yv = float_to_half_bits(r ? r[bb] * v : v);
-                    y[static_cast<size_t>(bb) * ldy + n] = yv;
-                    if (res)
-                        y2[static_cast<size_t>(bb) * ldy2 + n] =
-                            add_h(half_bits_to_float(res[static_cast<size_t>(bb) * ldres + n]), half_bits_to_float(yv));
-                }
-            }
-        }
-    }
-}
-
-// m[b][j] = fp16(silu(g) * u) with g = gu[b][j], u = gu[b][F + j].
-__global__ void __launch_bounds__(256) silu_mul_kernel(const uint16_t* __restrict__ gu, int F, int B,
-                                                       uint16_t* __restrict__ m)
-{
-    const int total = B * F;
-    for (int i = blockIdx.x * blockDim.x + threadIdx.x; i < total; i += gridDim.x * blockDim.x) {
-        const int b = i / F, j = i - b * F;
-        const float gf = half_bits_to_float(gu[static_cast<size_t>(b) * 2 * F + j]);
-        const float uf = half_bits_to_float(gu[static_cast<size_t>(b) * 2 * F + F + j]);
-        m[i] = float_to_half_bits(gf / (1.f + expf(-gf)) * uf);
-    }
-}
 
 // ---------------------------------------------------------------- host --
 
 struct Layout {
     size_t header, mats, llA, llX1, llM, llX, llV, pV, pX2, pQKV, pO, pX1, pGU, pM, pD, x_stage, logits_stage, rfac,
-        total;
+        xpH, xpF, part, total;
     size_t ll_begin, ll_end;
 };
 
@@ -910,7 +816,14 @@ Layout make_layout(const Dims& d)
     y.pD = take(2 * L * B * H);
     y.x_stage = take(2 * B * H);
     y.logits_stage = take(2 * B * static_cast<size_t>(d.V));
-    y.rfac = take(4 * (3 * L + 1) * B);   // RMS factors of the graph path: [L][3][B] + [B]
+    y.rfac = take(4 * (3 * L + 3) * B);   // RMS factors of the graph path: [L + 1][3][B]
+    if (d.B > kMaxChainBatch) {
+        y.xpH = take(2 * 32 * H);
+        y.xpF = take(2 * 32 * F);
+        y.part = take(4 * tc_part_floats(d.L, d.H, d.F, d.Nqkv, d.V, d.B, 256));
+    } else {
+        y.xpH = y.xpF = y.part = 0;
+    }
     y.total = o;
     return y;
 }
@@ -1013,62 +926,46 @@ bool ring_ok(const Dims& d, int nslots, uint32_t slot_bytes, int nw)
 // Records one token of the graph path on `cs`: every stage kernel of every
 // layer, reading the token input from the workspace staging area and writing
 // the logits to the workspace logits area.
-void record_graph_token(const wq4_layer_table* t, const Dims& d, const Layout& y, int sms, cudaStream_t cs)
-{
-    uint8_t* ws = static_cast<uint8_t*>(t->workspace);
-    const int B = d.B, H = d.H, F = d.F, L = d.L;
-    auto U16 = [&](size_t off) { return reinterpret_cast<uint16_t*>(ws + off); };
-    float* rf = reinterpret_cast<float*>(ws + y.rfac);
-    const size_t LH = static_cast<size_t>(B) * H;
-    auto gemv = [&](const wq4_mat& m, int N, int K, const uint16_t* x, int ldx, const float* r, uint16_t* out, int ldy,
-                    const uint16_t* res, uint16_t* out2) {
-        int grid = (N + 7) / 8;
-        if (grid > sms * 8) grid = sms * 8;
-        stage_gemv_kernel<8><<<grid, 256, 0, cs>>>(m.W, m.s, N, K, x, ldx, B, r, out, ldy, res, H, out2, H);
-    };
-    for (int l = 0; l < L; ++l) {
-        const wq4_layer& ly = t->layers[l];
-        const uint16_t* u = (l == 0) ? U16(y.x_stage) : U16(y.pX2) + static_cast<size_t>(l - 1) * LH;
-        float* r = rf + static_cast<size_t>(3 * l) * B;
-        uint16_t* v = U16(y.pV) + static_cast<size_t>(l) * LH;
-        uint16_t* qkv = U16(y.pQKV) + static_cast<size_t>(l) * B * d.Nqkv;
-        uint16_t* o = U16(y.pO) + static_cast<size_t>(l) * LH;
-        uint16_t* x1 = U16(y.pX1) + static_cast<size_t>(l) * LH;
-        uint16_t* gu = U16(y.pGU) + static_cast<size_t>(l) * B * 2 * F;
-        uint16_t* m = U16(y.pM) + static_cast<size_t>(l) * B * F;
-        uint16_t* dn = U16(y.pD) + static_cast<size_t>(l) * LH;
-        uint16_t* x2 = U16(y.pX2) + static_cast<size_t>(l) * LH;
-        rms_rows_kernel<<<B, 256, 0, cs>>>(u, H, H, t->rms_eps, r, v, H);
-        gemv(ly.qkv, d.Nqkv, H, u, H, r, qkv, d.Nqkv, nullptr, nullptr);
-        rms_rows_kernel<<<B, 256, 0, cs>>>(qkv, d.Nqkv, H, t->rms_eps, r + B, nullptr, 0);
-        gemv(ly.o, H, H, qkv, d.Nqkv, r + B, o, H, v, x1);
-        rms_rows_kernel<<<B, 256, 0, cs>>>(x1, H, H, t->rms_eps, r + 2 * B, nullptr, 0);
-        gemv(ly.gate_up, 2 * F, H, x1, H, r + 2 * B, gu, 2 * F, nullptr, nullptr);
-        silu_mul_kernel<<<sms * 4, 256, 0, cs>>>(gu, F, B, m);
-        gemv(ly.down, H, F, m, F, nullptr, dn, H, x1, x2);
-    }
-    const uint16_t* xl = U16(y.pX2) + static_cast<size_t>(L - 1) * LH;
-    float* r = rf + static_cast<size_t>(3 * L) * B;
-    rms_rows_kernel<<<B, 256, 0, cs>>>(xl, H, H, t->rms_eps, r, U16(y.pV) + static_cast<size_t>(L) * LH, H);
-    gemv(t->lm_head, d.V, H, xl, H, r, U16(y.logits_stage), d.V, nullptr, nullptr);
-}
-
 int build_graph_plan(const wq4_layer_table* t, const Dims& d, const Layout& lay, int dev, const DeviceInfo* di,
                      Plan* pl)
 {
+    uint8_t* ws = static_cast<uint8_t*>(t->workspace);
+    auto U16 = [&](size_t off) { return reinterpret_cast<uint16_t*>(ws + off); };
+    TcBuffers buf;
+    buf.x_stage = U16(lay.x_stage);
+    buf.pV = U16(lay.pV);
+    buf.pQKV = U16(lay.pQKV);
+    buf.pO = U16(lay.pO);
+    buf.pX1 = U16(lay.pX1);
+    buf.pGU = U16(lay.pGU);
+    buf.pM = U16(lay.pM);
+    buf.pD = U16(lay.pD);
+    buf.pX2 = U16(lay.pX2);
+    buf.logits = U16(lay.logits_stage);
+    buf.rf = reinterpret_cast<float*>(ws + lay.rfac);
+    buf.xpH = U16(lay.xpH);
+    buf.xpF = U16(lay.xpF);
+    buf.part = reinterpret_cast<float*>(ws + lay.part);
+    TcPlan* tc = nullptr;
+    int rc = tc_plan_create(t, d.H, d.F, d.Nqkv, d.V, d.B, buf, di->sm_count, status_word(), &tc);
+    if (rc != WQ4_OK) return rc;
     cudaStream_t cs = nullptr;
-    if (cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking) != cudaSuccess) return WQ4_ERR_CUDA;
+    if (cudaStreamCreateWithFlags(&cs, cudaStreamNonBlocking) != cudaSuccess) {
+        tc_plan_destroy(tc);
+        return WQ4_ERR_CUDA;
+    }
     cudaGraph_t graph = nullptr;
     cudaGraphExec_t exec = nullptr;
-    int rc = WQ4_ERR_CUDA;
+    rc = WQ4_ERR_CUDA;
     if (cudaStreamBeginCapture(cs, cudaStreamCaptureModeThreadLocal) == cudaSuccess) {
-        record_graph_token(t, d, lay, di->sm_count, cs);
+        tc_record_token(tc, cs);
         if (cudaStreamEndCapture(cs, &graph) == cudaSuccess && graph &&
             cudaGraphInstantiate(&exec, graph, 0) == cudaSuccess)
             rc = WQ4_OK;
     }
     if (graph) cudaGraphDestroy(graph);
     cudaStreamDestroy(cs);
+    tc_plan_destroy(tc);   // the graph holds copies of every launch argument
     if (rc != WQ4_OK) return rc;
     pl->table = *t;
     pl->layers.assign(t->layers, t->layers + d.L);

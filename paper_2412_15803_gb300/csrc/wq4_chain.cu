@@ -756,7 +756,7 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
 
 struct Layout {
     size_t header, mats, llA, llX1, llM, llX, llV, pV, pX2, pQKV, pO, pX1, pGU, pM, pD, x_stage, logits_stage, rfac,
-        xpH, xpF, part, total;
+        xpH0, xpH1, xpF, cnt, part, total;
     size_t ll_begin, ll_end;
 };
 
@@ -816,13 +816,17 @@ Layout make_layout(const Dims& d)
     y.pD = take(2 * L * B * H);
     y.x_stage = take(2 * B * H);
     y.logits_stage = take(2 * B * static_cast<size_t>(d.V));
-    y.rfac = take(4 * (3 * L + 3) * B);   // RMS factors of the graph path: [L + 1][3][B]
     if (d.B > kMaxChainBatch) {
-        y.xpH = take(2 * 32 * H);
+        // batched path: sums of squares of 128-element tiles (u, a, x1),
+        // arrival counters, permuted stage inputs, K-part partial sums
+        y.rfac = take(4 * 3 * (H / 128) * B);
+        y.cnt = take(4 * static_cast<size_t>(kTcCounterWords));
+        y.xpH0 = take(2 * 32 * H);
+        y.xpH1 = take(2 * 32 * H);
         y.xpF = take(2 * 32 * F);
         y.part = take(4 * tc_part_floats(d.L, d.H, d.F, d.Nqkv, d.V, d.B, 256));
     } else {
-        y.xpH = y.xpF = y.part = 0;
+        y.rfac = y.cnt = y.xpH0 = y.xpH1 = y.xpF = y.part = 0;
     }
     y.total = o;
     return y;
@@ -927,9 +931,12 @@ bool ring_ok(const Dims& d, int nslots, uint32_t slot_bytes, int nw)
 // layer, reading the token input from the workspace staging area and writing
 // the logits to the workspace logits area.
 int build_graph_plan(const wq4_layer_table* t, const Dims& d, const Layout& lay, int dev, const DeviceInfo* di,
-                     Plan* pl)
+                     Plan* pl, cudaStream_t stream)
 {
     uint8_t* ws = static_cast<uint8_t*>(t->workspace);
+    // the split stages' arrival counters start at zero (each stage leaves them so)
+    if (cudaMemsetAsync(ws + lay.cnt, 0, 4 * static_cast<size_t>(kTcCounterWords), stream) != cudaSuccess)
+        return WQ4_ERR_CUDA;
     auto U16 = [&](size_t off) { return reinterpret_cast<uint16_t*>(ws + off); };
     TcBuffers buf;
     buf.x_stage = U16(lay.x_stage);
@@ -942,8 +949,10 @@ int build_graph_plan(const wq4_layer_table* t, const Dims& d, const Layout& lay,
     buf.pD = U16(lay.pD);
     buf.pX2 = U16(lay.pX2);
     buf.logits = U16(lay.logits_stage);
-    buf.rf = reinterpret_cast<float*>(ws + lay.rfac);
-    buf.xpH = U16(lay.xpH);
+    buf.sq = reinterpret_cast<float*>(ws + lay.rfac);
+    buf.cnt = reinterpret_cast<uint32_t*>(ws + lay.cnt);
+    buf.xpH[0] = U16(lay.xpH0);
+    buf.xpH[1] = U16(lay.xpH1);
     buf.xpF = U16(lay.xpF);
     buf.part = reinterpret_cast<float*>(ws + lay.part);
     TcPlan* tc = nullptr;
@@ -958,8 +967,8 @@ int build_graph_plan(const wq4_layer_table* t, const Dims& d, const Layout& lay,
     cudaGraphExec_t exec = nullptr;
     rc = WQ4_ERR_CUDA;
     if (cudaStreamBeginCapture(cs, cudaStreamCaptureModeThreadLocal) == cudaSuccess) {
-        tc_record_token(tc, cs);
-        if (cudaStreamEndCapture(cs, &graph) == cudaSuccess && graph &&
+        const int rrec = tc_record_token(tc, cs);
+        if (cudaStreamEndCapture(cs, &graph) == cudaSuccess && graph && rrec == WQ4_OK &&
             cudaGraphInstantiate(&exec, graph, 0) == cudaSuccess)
             rc = WQ4_OK;
     }
@@ -1001,7 +1010,7 @@ int build_plan(const wq4_layer_table* t, Plan* pl, cudaStream_t stream)
     if (!di) return WQ4_ERR_CUDA;
     if (d.B > kMaxChainBatch) {
         if (d.Nqkv % 8) return WQ4_ERR_UNSUPPORTED;   // the O stage reads qkv rows with 16-byte loads
-        return build_graph_plan(t, d, lay, dev, di, pl);
+        return build_graph_plan(t, d, lay, dev, di, pl, stream);
     }
     if (!di->coop_launch) return WQ4_ERR_UNSUPPORTED;
     const uint32_t x_bytes = static_cast<uint32_t>(align_up(static_cast<size_t>(d.B) * 2 * (d.H > d.F ? d.H : d.F), 128));

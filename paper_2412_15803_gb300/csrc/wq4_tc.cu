@@ -41,50 +41,233 @@ namespace wq4 {
 namespace {
 
 constexpr int kTcStages = 4;          // ring slots
-constexpr int kTcThreads = 192;       // warps 0-3 dequant, 4 producer, 5 MMA
+constexpr int kTcThreads = 448;       // warps 0-7 dequant, 8 producer, 9 MMA, 10-13 epilogue
+constexpr int kTcProducer = 8, kTcIssuer = 9;
 constexpr int kTcCodes = 128 * 128;   // one chunk of codes: 128 rows x 256 codes
 constexpr int kTcScales = 128 * 16;   // 128 rows x 8 fp16 scales
 constexpr int kTcTmemCols = 512;      // A: 2 x 128 columns, D: 2 x 32 columns at 256
 
 template <int NB>
 struct TcSmem {
+    static_assert(256 + 4 * (192 + 128 * 33) <= 18432, "epilogue scratch overlaps the ring");
     static constexpr int kX = NB * 512;                       // 4 slabs x NB rows x 128 B
     static constexpr int kSlot = kTcCodes + kX + kTcScales;   // multiple of 1024
-    static constexpr int kBytes = 1024 + kTcStages * kSlot;
+    static constexpr int kRing = 18432;                        // header + epilogue scratch, then the ring
+    static constexpr int kBytes = kRing + kTcStages * kSlot;
 };
 
-__device__ __forceinline__ bool tc_wait(uint64_t* bar, uint32_t parity, uint32_t* err)
+__device__ __forceinline__ bool tc_wait_ok(uint64_t* bar, uint32_t parity, uint32_t* err)
 {
     return mbar_wait(bar, parity, err);
+}
+
+// Kernel arguments besides the tensor maps.  A stage's "tile" is 128 weight
+// rows: rows [128 t, 128 t + 128), or for gate_up gate rows [64 t, 64 t + 64)
+// followed by the matching up rows [F + 64 t, F + 64 t + 64), so that one tile
+// holds both halves of SiLU(gate) * up.
+struct TcArgs {
+    int type, N, K, B, P, units, tiles, H, F;
+    float eps;
+    float* part;            // [P][B][N] partial sums (P > 1)
+    uint32_t* cnt;          // [tiles] arrival counters (P > 1), zero between stages
+    const float* sq_in;     // per-tile sums of squares of this stage's input [H/128][B]; null: factor 1
+    const float* sq_u;      // O: sums of squares of the layer input u
+    const uint16_t* res;    // O: the layer input u; down: x1
+    uint16_t* y;            // QKV: qkv, O: o, gate_up: gate|up, down: d, LM: logits
+    uint16_t* y2;           // O: x1, gate_up: m, down: x2
+    uint16_t* y3;           // O: v = fp16(r(u) u)
+    float* sq_out;          // per-tile sums of squares of the next stage's input [H/128][B]
+    uint16_t* xp;           // next stage's permuted input [32][ldxp]
+    int ldxp;
+    uint32_t* err;
+};
+
+__device__ __forceinline__ void grid_dep_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_dep_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
+// fp16(a + b) for fp16 operands: the fp32 sum rounded once to fp16.
+__device__ __forceinline__ uint16_t add_h(float a, float b) { return float_to_half_bits(a + b); }
+
+// Logical position, within its 8-block, of element p (0..7) of a packed
+// word: the unpack pairs (p, p + 4), so logical order is 0 4 1 5 2 6 3 7.
+__device__ __forceinline__ int perm_pos(int p) { return p < 4 ? 2 * p : 2 * (p - 4) + 1; }
+
+// r = 1/sqrt(mean + eps) from per-tile sums of squares, summed in tile order
+// (loads issued eight at a time).
+__device__ __forceinline__ float rms_of(const float* sq, int ntiles, int B, int b, int n, float eps)
+{
+    float t = 0.f;
+    int i = 0;
+    for (; i + 8 <= ntiles; i += 8) {
+        float v[8];
+#pragma unroll
+        for (int k = 0; k < 8; ++k) v[k] = __ldcg(sq + (i + k) * B + b);
+#pragma unroll
+        for (int k = 0; k < 8; ++k) t += v[k];
+    }
+    for (; i < ntiles; ++i) t += __ldcg(sq + i * B + b);
+    return rsqrtf(t * (1.f / static_cast<float>(n)) + eps);
+}
+
+// Epilogue of one tile by the 128 dequant threads (row = 32 warp + lane): v[b]
+// the row's sums over K for batch row b.  ep: shared scratch.
+template <int NB>
+__device__ void tile_epilogue(const TcArgs& a, int tile, int row, const float v[NB], float* ep)
+{
+    float* r_in = ep;          // [32]
+    float* r_u = ep + 32;      // [32]
+    float* red = ep + 64;      // [4][32]
+    float* sqs = ep + 192;     // [128][33] squares of the next input (padded rows), ends before the ring
+    uint16_t* upart = reinterpret_cast<uint16_t*>(ep + 192);   // [64][32] up values of gate_up (aliases sqs)
+    const int warp = row >> 5, lane = row & 31, B = a.B, H = a.H, F = a.F;
+    if (warp == 0 && lane < B) {
+        r_in[lane] = a.sq_in ? rms_of(a.sq_in, H / 128, B, lane, H, a.eps) : 1.f;
+        if (a.sq_u) r_u[lane] = rms_of(a.sq_u, H / 128, B, lane, H, a.eps);
+    }
+    named_barrier_sync(3, 128);
+    float nxt[NB];              // value of the next stage's input at this row (if any)
+    bool has_next = false;
+    int nidx = 0;               // its index in the next input
+    if (a.type == kTcGU) {
+        const bool up = row >= 64;
+        const int j = 64 * tile + (row & 63);
+        if (up) {
+#pragma unroll
+            for (int b = 0; b < NB; ++b)
+                if (b < B) {
+                    const uint16_t uu = float_to_half_bits(r_in[b] * v[b]);
+                    a.y[static_cast<size_t>(b) * 2 * F + F + j] = uu;
+                    upart[(row - 64) * 32 + b] = uu;
+                }
+        }
+        named_barrier_sync(3, 128);
+        if (!up) {
+#pragma unroll
+            for (int b = 0; b < NB; ++b)
+                if (b < B) {
+                    const uint16_t g = float_to_half_bits(r_in[b] * v[b]);
+                    const float gf = half_bits_to_float(g);
+                    const uint16_t m =
+                        float_to_half_bits(gf / (1.f + expf(-gf)) * half_bits_to_float(upart[row * 32 + b]));
+                    a.y[static_cast<size_t>(b) * 2 * F + j] = g;
+                    a.y2[static_cast<size_t>(b) * F + j] = m;
+                    a.xp[static_cast<size_t>(b) * a.ldxp + (j & ~7) + perm_pos(j & 7)] = m;
+                }
+        }
+        return;
+    }
+    const int n = 128 * tile + row;
+    if (n < a.N) {
+        switch (a.type) {
+            case kTcQKV:
+#pragma unroll
+                for (int b = 0; b < NB; ++b)
+                    if (b < B) {
+                        const uint16_t q = float_to_half_bits(r_in[b] * v[b]);
+                        a.y[static_cast<size_t>(b) * a.N + n] = q;
+                        nxt[b] = half_bits_to_float(q);
+                    }
+                has_next = n < H;
+                nidx = n;
+                break;
+            case kTcO:
+#pragma unroll
+                for (int b = 0; b < NB; ++b)
+                    if (b < B) {
+                        const uint16_t o = float_to_half_bits(r_in[b] * v[b]);
+                        const uint16_t vn = float_to_half_bits(r_u[b] * half_bits_to_float(a.res[static_cast<size_t>(b) * H + n]));
+                        const uint16_t x1 = add_h(half_bits_to_float(vn), half_bits_to_float(o));
+                        a.y[static_cast<size_t>(b) * H + n] = o;
+                        a.y2[static_cast<size_t>(b) * H + n] = x1;
+                        a.y3[static_cast<size_t>(b) * H + n] = vn;
+                        nxt[b] = half_bits_to_float(x1);
+                    }
+                has_next = true;
+                nidx = n;
+                break;
+            case kTcDOWN:
+#pragma unroll
+                for (int b = 0; b < NB; ++b)
+                    if (b < B) {
+                        const uint16_t d = float_to_half_bits(v[b]);
+                        const uint16_t x2 = add_h(half_bits_to_float(a.res[static_cast<size_t>(b) * H + n]), half_bits_to_float(d));
+                        a.y[static_cast<size_t>(b) * H + n] = d;
+                        a.y2[static_cast<size_t>(b) * H + n] = x2;
+                        nxt[b] = half_bits_to_float(x2);
+                    }
+                has_next = true;
+                nidx = n;
+                break;
+            default:   // LM head; its first H / 128 tiles also keep v = fp16(r x_L)
+#pragma unroll
+                for (int b = 0; b < NB; ++b)
+                    if (b < B) {
+                        a.y[static_cast<size_t>(b) * a.N + n] = float_to_half_bits(r_in[b] * v[b]);
+                        if (n < H)
+                            a.y3[static_cast<size_t>(b) * H + n] =
+                                float_to_half_bits(r_in[b] * half_bits_to_float(a.res[static_cast<size_t>(b) * H + n]));
+                    }
+                break;
+        }
+    }
+    if (a.type == kTcLM) return;
+    // the next stage's permuted input and, per tile of its rows, its sum of squares
+    if (has_next) {
+#pragma unroll
+        for (int b = 0; b < NB; ++b)
+            if (b < B) a.xp[static_cast<size_t>(b) * a.ldxp + (nidx & ~7) + perm_pos(nidx & 7)] = float_to_half_bits(nxt[b]);
+    }
+    if (tile < H / 128) {
+        // sum over the tile's 128 rows per batch row, in a fixed order:
+        // 32-row runs, then the four runs
+#pragma unroll
+        for (int b = 0; b < NB; ++b)
+            if (b < B) sqs[row * 33 + b] = has_next ? nxt[b] * nxt[b] : 0.f;
+        named_barrier_sync(3, 128);
+        {
+            const int b = row & 31, run = row >> 5;
+            float t = 0.f;
+            if (b < B)
+                for (int k = 0; k < 32; ++k) t += sqs[(32 * run + k) * 33 + b];
+            red[run * 32 + b] = t;
+        }
+        named_barrier_sync(3, 128);
+        if (row < B) a.sq_out[tile * B + row] = ((red[row] + red[32 + row]) + red[64 + row]) + red[96 + row];
+    }
 }
 
 template <int NB>
 __global__ void __launch_bounds__(kTcThreads, 1)
     tc_stage_kernel(const __grid_constant__ CUtensorMap tm_codes, const __grid_constant__ CUtensorMap tm_scales,
-                    const __grid_constant__ CUtensorMap tm_x, int N, int K, int B, int P, int units,
-                    float* __restrict__ part, uint32_t* err)
+                    const __grid_constant__ CUtensorMap tm_x, const TcArgs a)
 {
     using L = TcSmem<NB>;
     extern __shared__ __align__(1024) uint8_t smem[];
-    uint64_t* full = reinterpret_cast<uint64_t*>(smem);
-    uint64_t* empty = full + kTcStages;
+    uint64_t* fullw = reinterpret_cast<uint64_t*>(smem);   // codes + scales landed
+    uint64_t* fullx = fullw + kTcStages;                     // input columns landed
+    uint64_t* empty = fullx + kTcStages;
     uint64_t* afull = empty + kTcStages;
     uint64_t* aempty = afull + 2;
     uint64_t* dfull = aempty + 2;
     uint64_t* dempty = dfull + 2;
-    uint64_t* drain = dempty + 2;
-    uint32_t* tbase_sh = reinterpret_cast<uint32_t*>(smem + 256);
-    uint8_t* ring = smem + 1024;
+    uint64_t* drain = dempty + 2;                            // ends at byte 168
+    uint32_t* tbase_sh = reinterpret_cast<uint32_t*>(smem + 192);
+    uint32_t* last_sh = tbase_sh + 1;
+    float* ep = reinterpret_cast<float*>(smem + 256);        // epilogue scratch: 768 B + 128 x 33 floats
+    uint8_t* ring = smem + L::kRing;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int nch = K >> 8;   // chunks of 256 along K
+    const int nch = a.K >> 8;   // chunks of 256 along K
+    const int P = a.P, units = a.units;
+    uint32_t* err = a.err;
 
     if (threadIdx.x == 0) {
         for (int i = 0; i < kTcStages; ++i) {
-            mbar_init(&full[i], 1);
-            mbar_init(&empty[i], 5);   // 4 dequant warps + the MMA commit
+            mbar_init(&fullw[i], 1);
+            mbar_init(&fullx[i], 1);
+            mbar_init(&empty[i], 9);   // 8 dequant warps + the MMA commit
         }
         for (int i = 0; i < 2; ++i) {
-            mbar_init(&afull[i], 4);
+            mbar_init(&afull[i], 8);
             mbar_init(&aempty[i], 1);
             mbar_init(&dfull[i], 1);
             mbar_init(&dempty[i], 4);
@@ -92,43 +275,85 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         mbar_init(drain, 1);
         mbar_fence_init();
     }
-    if (warp == 5) tc::tmem_alloc(tbase_sh, kTcTmemCols);
+    if (warp == kTcIssuer) tc::tmem_alloc(tbase_sh, kTcTmemCols);
     tc::fence_before_sync();
     __syncthreads();
     tc::fence_after_sync();
     const uint32_t tbase = *tbase_sh;
+    // the next stage may start its set-up and weight stream now; it reads our
+    // outputs only after this grid has completed
+    grid_dep_launch();
 
-    if (warp == 4) {
+    auto tile_rows = [&](int tile, int half) {   // first weight row of a 64-row half tile
+        return a.type == kTcGU ? (half ? a.F : 0) + 64 * tile : 128 * tile + 64 * half;
+    };
+
+    if (warp == kTcProducer) {
         // ---------------------------------------------------- producer
         if (lane == 0) {
             tc::prefetch_map(&tm_codes);
             tc::prefetch_map(&tm_scales);
             tc::prefetch_map(&tm_x);
             int it = 0;
-            bool ok = true;
+            bool ok = true, waited = false;
+            int pend_c[kTcStages];   // chunks whose input columns wait for the previous stage
+            int npend = 0;
             for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
                 const int tile = u / P, pt = u - tile * P;
                 const int c0 = pt * nch / P, c1 = (pt + 1) * nch / P;
                 for (int c = c0; c < c1; ++c, ++it) {
                     const int slot = it % kTcStages;
-                    if (it >= kTcStages && !tc_wait(&empty[slot], ((it / kTcStages) - 1) & 1, err)) {
-                        ok = false;
-                        break;
+                    if (it >= kTcStages) {
+                        if (!waited) {
+                            grid_dep_wait();
+                            waited = true;
+                            for (int i = 0; i < npend; ++i) {
+                                uint8_t* pb = ring + static_cast<size_t>(i) * L::kSlot;
+                                mbar_arrive_expect_tx(&fullx[i], L::kX);
+#pragma unroll
+                                for (int j = 0; j < 4; ++j)
+                                    tc::tma_load_2d(pb + kTcCodes + j * NB * 128, &tm_x, pend_c[i] * 256 + 64 * j, 0, &fullx[i]);
+                            }
+                        }
+                        if (!tc_wait_ok(&empty[slot], ((it / kTcStages) - 1) & 1, err)) {
+                            ok = false;
+                            break;
+                        }
                     }
                     uint8_t* base = ring + static_cast<size_t>(slot) * L::kSlot;
-                    mbar_arrive_expect_tx(&full[slot], kTcCodes + L::kX + kTcScales);
-                    tc::tma_load_2d(base, &tm_codes, c * 128, tile * 128, &full[slot]);
-                    tc::tma_load_2d(base + kTcCodes + L::kX, &tm_scales, c * 8, tile * 128, &full[slot]);
+                    mbar_arrive_expect_tx(&fullw[slot], kTcCodes + kTcScales);
+                    tc::tma_load_2d(base, &tm_codes, c * 128, tile_rows(tile, 0), &fullw[slot]);
+                    tc::tma_load_2d(base + 64 * 128, &tm_codes, c * 128, tile_rows(tile, 1), &fullw[slot]);
+                    tc::tma_load_2d(base + kTcCodes + L::kX, &tm_scales, c * 8, tile_rows(tile, 0), &fullw[slot]);
+                    tc::tma_load_2d(base + kTcCodes + L::kX + 64 * 16, &tm_scales, c * 8, tile_rows(tile, 1), &fullw[slot]);
+                    if (waited) {
+                        mbar_arrive_expect_tx(&fullx[slot], L::kX);
+#pragma unroll
+                        for (int j = 0; j < 4; ++j)
+                            tc::tma_load_2d(base + kTcCodes + j * NB * 128, &tm_x, c * 256 + 64 * j, 0, &fullx[slot]);
+                    } else {
+                        pend_c[npend++] = c;
+                    }
+                }
+            }
+            if (!waited) {
+                grid_dep_wait();
+                for (int i = 0; i < npend; ++i) {
+                    uint8_t* pb = ring + static_cast<size_t>(i) * L::kSlot;
+                    mbar_arrive_expect_tx(&fullx[i], L::kX);
 #pragma unroll
                     for (int j = 0; j < 4; ++j)
-                        tc::tma_load_2d(base + kTcCodes + j * NB * 128, &tm_x, c * 256 + 64 * j, 0, &full[slot]);
+                        tc::tma_load_2d(pb + kTcCodes + j * NB * 128, &tm_x, pend_c[i] * 256 + 64 * j, 0, &fullx[i]);
                 }
             }
             // every copy issued has landed before the CTA's memory goes away
             const int first = it > kTcStages ? it - kTcStages : 0;
-            for (int i = first; i < it; ++i) tc_wait(&full[i % kTcStages], (i / kTcStages) & 1, err);
+            for (int i = first; i < it; ++i) {
+                tc_wait_ok(&fullw[i % kTcStages], (i / kTcStages) & 1, err);
+                tc_wait_ok(&fullx[i % kTcStages], (i / kTcStages) & 1, err);
+            }
         }
-    } else if (warp == 5) {
+    } else if (warp == kTcIssuer) {
         // ---------------------------------------------------- MMA issuer
         if (lane == 0) {
             constexpr uint32_t idesc = tc::idesc_f16_f32(128, NB);
@@ -137,12 +362,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
                 const int tile = u / P, pt = u - tile * P;
                 const int c0 = pt * nch / P, c1 = (pt + 1) * nch / P;
+                (void)tile;
                 const int dbuf = dit & 1;
-                if (dit >= 2 && !tc_wait(&dempty[dbuf], ((dit >> 1) - 1) & 1, err)) break;
+                if (dit >= 2 && !tc_wait_ok(&dempty[dbuf], ((dit >> 1) - 1) & 1, err)) break;
                 const uint32_t dt = tbase + 256 + 32 * dbuf;
                 for (int c = c0; c < c1; ++c, ++it, ++ait) {
                     const int slot = it % kTcStages, abuf = ait & 1;
-                    if (!tc_wait(&full[slot], (it / kTcStages) & 1, err) || !tc_wait(&afull[abuf], (ait >> 1) & 1, err)) {
+                    if (!tc_wait_ok(&fullx[slot], (it / kTcStages) & 1, err) ||
+                        !tc_wait_ok(&afull[abuf], (ait >> 1) & 1, err)) {
                         ok = false;
                         break;
                     }
@@ -162,32 +389,36 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             }
             // all MMAs issued have completed before tensor memory is released
             tc::commit(drain);
-            tc_wait(drain, 0, err);
+            tc_wait_ok(drain, 0, err);
         }
-    } else {
-        // ---------------------------------------------------- dequant + readout
-        const int row = 32 * warp + lane;            // tile row = tensor-memory lane
-        const uint32_t lane_base = tbase + (static_cast<uint32_t>(32 * warp) << 16);
-        int it = 0, ait = 0, dit = 0;
+    } else if (warp < 8) {
+        // ---------------------------------------------------- dequant
+        // warp w: rows 32 (w % 4) + lane (its tensor-memory lanes), groups
+        // 4 (w / 4) .. + 3 of each chunk
+        const int row = 32 * (warp & 3) + lane;
+        const int jg = 4 * (warp >> 2);
+        const uint32_t lane_base = tbase + (static_cast<uint32_t>(32 * (warp & 3)) << 16);
+        int it = 0, ait = 0;
         bool ok = true;
         for (int u = blockIdx.x; u < units && ok; u += gridDim.x) {
             const int tile = u / P, pt = u - tile * P;
             const int c0 = pt * nch / P, c1 = (pt + 1) * nch / P;
             for (int c = c0; c < c1; ++c, ++it, ++ait) {
                 const int slot = it % kTcStages, abuf = ait & 1;
-                if (!tc_wait(&full[slot], (it / kTcStages) & 1, err) ||
-                    (ait >= 2 && !tc_wait(&aempty[abuf], ((ait >> 1) - 1) & 1, err))) {
+                if (!tc_wait_ok(&fullw[slot], (it / kTcStages) & 1, err) ||
+                    (ait >= 2 && !tc_wait_ok(&aempty[abuf], ((ait >> 1) - 1) & 1, err))) {
                     ok = false;
                     break;
                 }
                 const uint8_t* base = ring + static_cast<size_t>(slot) * L::kSlot;
                 const uint8_t* crow = base + row * 128;
-                const uint4 sv = *reinterpret_cast<const uint4*>(base + kTcCodes + L::kX + row * 16);
-                const uint32_t sw[4] = {sv.x, sv.y, sv.z, sv.w};
+                const uint2 sv = *reinterpret_cast<const uint2*>(base + kTcCodes + L::kX + row * 16 + 2 * jg);
+                const uint32_t sw[2] = {sv.x, sv.y};
 #pragma unroll
-                for (int j = 0; j < 8; ++j) {
+                for (int jj = 0; jj < 4; ++jj) {
+                    const int j = jg + jj;
                     const uint4 cw = *reinterpret_cast<const uint4*>(crow + ((j ^ (row & 7)) << 4));
-                    const uint32_t sh = (j & 1) ? (sw[j >> 1] >> 16) : (sw[j >> 1] & 0xFFFFu);
+                    const uint32_t sh = (jj & 1) ? (sw[jj >> 1] >> 16) : (sw[jj >> 1] & 0xFFFFu);
                     const uint32_t s2 = sh | (sh << 16);
                     uint32_t q[16];
                     unpack_word(cw.x, q + 0);
@@ -207,163 +438,102 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 }
             }
             if (!ok) break;
+        }
+    } else {
+        // ---------------------------------------------------- epilogue warps
+        // warp w reads tensor-memory lanes 32 (w % 4) .. + 31
+        const int quad = warp & 3;
+        const int row = 32 * quad + lane;
+        const uint32_t lane_base = tbase + (static_cast<uint32_t>(32 * quad) << 16);
+        int dit = 0;
+        bool waited = false;
+        for (int u = blockIdx.x; u < units; u += gridDim.x) {
+            const int tile = u / P, pt = u - tile * P;
             const int dbuf = dit & 1;
-            if (!tc_wait(&dfull[dbuf], (dit >> 1) & 1, err)) break;
+            if (!tc_wait_ok(&dfull[dbuf], (dit >> 1) & 1, err)) break;
             tc::fence_after_sync();
             uint32_t d[32];
             tc::ld16(lane_base + 256 + 32 * dbuf, d);
             if (NB > 16) tc::ld16(lane_base + 256 + 32 * dbuf + 16, d + 16);
             tc::ld_wait();
-            const int n = tile * 128 + row;
-            if (n < N) {
-                float* pb = part + static_cast<size_t>(pt) * B * N + n;
-#pragma unroll
-                for (int b = 0; b < NB; ++b)
-                    if (b < B) pb[static_cast<size_t>(b) * N] = __uint_as_float(d[b]);
-            }
             tc::fence_before_sync();
             __syncwarp();
             if (lane == 0) mbar_arrive(&dempty[dbuf]);
             ++dit;
+            if (!waited) {
+                grid_dep_wait();   // the previous stage's outputs are complete and visible
+                waited = true;
+            }
+            float v[NB];
+#pragma unroll
+            for (int b = 0; b < NB; ++b) v[b] = __uint_as_float(d[b]);
+            if (P > 1) {
+                // K is split over units: publish this part; the last part of
+                // the tile sums all parts in order and runs the epilogue
+                const int nrow = a.type == kTcGU ? tile_rows(tile, row >> 6) + (row & 63) : 128 * tile + row;
+                const bool valid = nrow < a.N;
+                if (valid) {
+                    float* pb = a.part + static_cast<size_t>(pt) * a.B * a.N + nrow;
+#pragma unroll
+                    for (int b = 0; b < NB; ++b)
+                        if (b < a.B) pb[static_cast<size_t>(b) * a.N] = v[b];
+                }
+                __threadfence();
+                named_barrier_sync(3, 128);
+                if (row == 0) {
+                    const uint32_t prev = atomicAdd(&a.cnt[tile], 1u);
+                    *last_sh = (prev == static_cast<uint32_t>(P - 1)) ? 1u : 0u;
+                    if (prev == static_cast<uint32_t>(P - 1)) a.cnt[tile] = 0u;   // ready for the next stage
+                }
+                named_barrier_sync(3, 128);
+                if (*last_sh == 0u) continue;
+                __threadfence();
+                if (valid) {
+                    // every part, this unit's included, from L2 in part order
+#pragma unroll
+                    for (int b = 0; b < NB; ++b) v[b] = 0.f;
+                    for (int q = 0; q < P; ++q) {
+                        const float* src = a.part + static_cast<size_t>(q) * a.B * a.N + nrow;
+                        float t[NB];
+#pragma unroll
+                        for (int b = 0; b < NB; ++b) t[b] = (b < a.B) ? __ldcg(src + static_cast<size_t>(b) * a.N) : 0.f;
+#pragma unroll
+                        for (int b = 0; b < NB; ++b) v[b] += t[b];
+                    }
+                }
+            }
+            tile_epilogue<NB>(a, tile, row, v, ep);
+            named_barrier_sync(3, 128);   // scratch reuse across units
         }
     }
 
     tc::fence_before_sync();
     __syncthreads();
     tc::fence_after_sync();
-    if (warp == 5) tc::tmem_dealloc(tbase, kTcTmemCols);
+    if (warp == kTcIssuer) tc::tmem_dealloc(tbase, kTcTmemCols);
 }
 
-// ------------------------------------------------------------ epilogues --
-
-__device__ __forceinline__ int perm8(int l) { return (l & 1) ? (l >> 1) + 4 : (l >> 1); }
-
-// fp16(a + b) for fp16 operands: the fp32 sum rounded once to fp16.
-__device__ __forceinline__ uint16_t add_h(float a, float b) { return float_to_half_bits(a + b); }
-
-// Sum of squares of vec[0, n) in a fixed order (same bits on every run).
-__device__ float block_sumsq(const uint16_t* vec, int n, float* red)
+// Token start (one CTA per batch row b): the permuted token input and the sums
+// of squares of its 128-element tiles.
+__global__ void __launch_bounds__(128) tc_prologue_kernel(const uint16_t* __restrict__ x, int H, int B,
+                                                          float* __restrict__ sq_out, uint16_t* __restrict__ xp)
 {
-    float s = 0.f;
-    for (int k = threadIdx.x; k < n; k += blockDim.x) {
-        const float t = half_bits_to_float(vec[k]);
-        s = fmaf(t, t, s);
-    }
-    s = warp_sum(s);
-    __syncthreads();
-    if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
-    __syncthreads();
-    float t = 0.f;
-    for (int w = 0; w < static_cast<int>(blockDim.x >> 5); ++w) t += red[w];
-    return t;
-}
-
-// xp[8w + l] = vec[8w + perm8(l)]
-__device__ void write_perm(const uint16_t* vec, int n, uint16_t* xp)
-{
-    for (int w = threadIdx.x; w < (n >> 3); w += blockDim.x) {
-        uint16_t o[8];
-#pragma unroll
-        for (int l = 0; l < 8; ++l) o[l] = vec[8 * w + perm8(l)];
-        uint4 v;
-        v.x = o[0] | (static_cast<uint32_t>(o[1]) << 16);
-        v.y = o[2] | (static_cast<uint32_t>(o[3]) << 16);
-        v.z = o[4] | (static_cast<uint32_t>(o[5]) << 16);
-        v.w = o[6] | (static_cast<uint32_t>(o[7]) << 16);
-        reinterpret_cast<uint4*>(xp)[w] = v;
-    }
-}
-
-__device__ __forceinline__ float rms_factor(float sumsq, int n, float eps)
-{
-    return rsqrtf(sumsq * (1.f / static_cast<float>(n)) + eps);
-}
-
-// Token start (one CTA per batch row): r = r(u), v = fp16(r u), xp = perm(u).
-__global__ void __launch_bounds__(1024) tc_prologue_kernel(const uint16_t* __restrict__ u, int H, float eps,
-                                                           float* __restrict__ r_out, uint16_t* __restrict__ v_out,
-                                                           uint16_t* __restrict__ xp)
-{
-    __shared__ float red[32];
+    __shared__ float red[4];
+    grid_dep_wait();
+    grid_dep_launch();
     const int b = blockIdx.x;
-    const uint16_t* ub = u + static_cast<size_t>(b) * H;
-    const float r = rms_factor(block_sumsq(ub, H, red), H, eps);
-    if (threadIdx.x == 0) r_out[b] = r;
-    for (int k = threadIdx.x; k < H; k += blockDim.x)
-        v_out[static_cast<size_t>(b) * H + k] = float_to_half_bits(r * half_bits_to_float(ub[k]));
-    write_perm(ub, H, xp + static_cast<size_t>(b) * H);
-}
-
-// One stage's epilogue for batch row b = blockIdx.x; vec (shared memory) holds
-// the next stage's input.
-__global__ void __launch_bounds__(1024) tc_epilogue_kernel(TcEpi e)
-{
-    extern __shared__ __align__(16) uint16_t vec[];
-    __shared__ float red[32];
-    const int b = blockIdx.x, B = e.B, N = e.N, H = e.H, F = e.F;
-    auto ysum = [&](int n) {
-        float t = 0.f;
-        for (int p = 0; p < e.P; ++p) t += e.part[(static_cast<size_t>(p) * B + b) * N + n];
-        return t;
-    };
-    const float r = e.r_in ? e.r_in[b] : 1.f;
-    int nvec = 0;
-    switch (e.type) {
-        case kTcQKV:
-            for (int n = threadIdx.x; n < N; n += blockDim.x) {
-                const uint16_t q = float_to_half_bits(r * ysum(n));
-                e.y[static_cast<size_t>(b) * N + n] = q;
-                if (n < H) vec[n] = q;
-            }
-            nvec = H;
-            break;
-        case kTcO:
-            for (int n = threadIdx.x; n < H; n += blockDim.x) {
-                const uint16_t o = float_to_half_bits(r * ysum(n));
-                const uint16_t x1 = add_h(half_bits_to_float(e.v_in[static_cast<size_t>(b) * H + n]), half_bits_to_float(o));
-                e.y[static_cast<size_t>(b) * H + n] = o;
-                e.y2[static_cast<size_t>(b) * H + n] = x1;
-                vec[n] = x1;
-            }
-            nvec = H;
-            break;
-        case kTcGU:
-            for (int j = threadIdx.x; j < F; j += blockDim.x) {
-                const uint16_t g = float_to_half_bits(r * ysum(j));
-                const uint16_t uu = float_to_half_bits(r * ysum(F + j));
-                const float gf = half_bits_to_float(g);
-                const uint16_t m = float_to_half_bits(gf / (1.f + expf(-gf)) * half_bits_to_float(uu));
-                e.y[static_cast<size_t>(b) * 2 * F + j] = g;
-                e.y[static_cast<size_t>(b) * 2 * F + F + j] = uu;
-                e.y2[static_cast<size_t>(b) * F + j] = m;
-                vec[j] = m;
-            }
-            nvec = F;
-            break;
-        case kTcDOWN:
-            for (int n = threadIdx.x; n < H; n += blockDim.x) {
-                const uint16_t d = float_to_half_bits(ysum(n));
-                const uint16_t x2 = add_h(half_bits_to_float(e.v_in[static_cast<size_t>(b) * H + n]), half_bits_to_float(d));
-                e.y[static_cast<size_t>(b) * H + n] = d;
-                e.y2[static_cast<size_t>(b) * H + n] = x2;
-                vec[n] = x2;
-            }
-            nvec = H;
-            break;
-        default:   // LM head
-            for (int n = threadIdx.x; n < N; n += blockDim.x)
-                e.y[static_cast<size_t>(b) * N + n] = float_to_half_bits(r * ysum(n));
-            return;
+    const uint16_t* xb = x + static_cast<size_t>(b) * H;
+    for (int t = 0; t < H / 128; ++t) {
+        const int n = 128 * t + threadIdx.x;
+        const uint16_t val = xb[n];
+        xp[static_cast<size_t>(b) * H + (n & ~7) + perm_pos(n & 7)] = val;
+        const float f = half_bits_to_float(val);
+        const float s = warp_sum(f * f);
+        if ((threadIdx.x & 31) == 0) red[threadIdx.x >> 5] = s;
+        __syncthreads();
+        if (threadIdx.x == 0) sq_out[t * B + b] = ((red[0] + red[1]) + red[2]) + red[3];
+        __syncthreads();
     }
-    __syncthreads();
-    if (e.r_out) {
-        const float rn = rms_factor(block_sumsq(vec, nvec, red), nvec, e.eps);
-        if (threadIdx.x == 0) e.r_out[b] = rn;
-        if (e.v_out)
-            for (int k = threadIdx.x; k < nvec; k += blockDim.x)
-                e.v_out[static_cast<size_t>(b) * nvec + k] = float_to_half_bits(rn * half_bits_to_float(vec[k]));
-    }
-    write_perm(vec, nvec, e.xp + static_cast<size_t>(b) * nvec);
 }
 
 // ----------------------------------------------------------------- host --
@@ -396,7 +566,7 @@ bool encode_2d(CUtensorMap* m, CUtensorMapDataType dt, const void* base, uint64_
 }
 
 struct TcMatMaps {
-    CUtensorMap codes, scales;
+    CUtensorMap codes, scales;   // boxes of 64 rows
     int N, K;
 };
 
@@ -414,11 +584,20 @@ int set_stage_attr()
     return rc;
 }
 
+// K parts of a stage: enough units to fill the GPU, each at least one chunk.
+int stage_parts(int tiles, int nch, int sms)
+{
+    int P = sms / tiles;
+    if (P < 1) P = 1;
+    if (P > nch) P = nch;
+    return P;
+}
+
 }  // namespace
 
 struct TcPlan {
     std::vector<TcMatMaps> mats;   // [4L + 1]
-    CUtensorMap xH, xF;
+    CUtensorMap xH[2], xF;
     TcBuffers buf;
     int L, H, F, Nqkv, V, B, NB, sms;
     float eps;
@@ -428,18 +607,15 @@ struct TcPlan {
 size_t tc_part_floats(int L, int H, int F, int Nqkv, int V, int B, int sms)
 {
     (void)L;
-    auto pn = [&](int N, int K) {
-        const int tiles = (N + 127) / 128, nch = K / 256;
-        int P = sms / tiles;
-        if (P < 1) P = 1;
-        if (P > nch) P = nch;
-        return static_cast<size_t>(P) * N;
+    auto pn = [&](int N, int K, int tiles) {
+        const int P = stage_parts(tiles, K / 256, sms);
+        return P > 1 ? static_cast<size_t>(P) * N : 0;
     };
-    size_t m = pn(Nqkv, H);
-    m = std::max(m, pn(H, H));
-    m = std::max(m, pn(2 * F, H));
-    m = std::max(m, pn(H, F));
-    m = std::max(m, pn(V, H));
+    size_t m = pn(Nqkv, H, (Nqkv + 127) / 128);
+    m = std::max(m, pn(H, H, H / 128));
+    m = std::max(m, pn(2 * F, H, F / 64));
+    m = std::max(m, pn(H, F, H / 128));
+    m = std::max(m, pn(V, H, (V + 127) / 128));
     return m * B;
 }
 
@@ -448,6 +624,8 @@ int tc_plan_create(const wq4_layer_table* t, int H, int F, int Nqkv, int V, int 
 {
     *out = nullptr;
     if (B > 32 || H % 256 || F % 256 || !encode_fn()) return WQ4_ERR_UNSUPPORTED;
+    if ((Nqkv + 127) / 128 > kTcCounterWords || H / 128 > kTcCounterWords || F / 64 > kTcCounterWords)
+        return WQ4_ERR_UNSUPPORTED;
     TcPlan* p = new TcPlan();
     p->L = t->num_layers;
     p->H = H;
@@ -464,9 +642,9 @@ int tc_plan_create(const wq4_layer_table* t, int H, int F, int Nqkv, int V, int 
         TcMatMaps mm;
         mm.N = N;
         mm.K = K;
-        const bool ok = encode_2d(&mm.codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, m.W, K / 2, N, K / 2, 128, 128,
+        const bool ok = encode_2d(&mm.codes, CU_TENSOR_MAP_DATA_TYPE_UINT8, m.W, K / 2, N, K / 2, 128, 64,
                                   CU_TENSOR_MAP_SWIZZLE_128B) &&
-                        encode_2d(&mm.scales, CU_TENSOR_MAP_DATA_TYPE_UINT16, m.s, K / 32, N, K / 16, 8, 128,
+                        encode_2d(&mm.scales, CU_TENSOR_MAP_DATA_TYPE_UINT16, m.s, K / 32, N, K / 16, 8, 64,
                                   CU_TENSOR_MAP_SWIZZLE_NONE);
         p->mats.push_back(mm);
         return ok;
@@ -477,9 +655,10 @@ int tc_plan_create(const wq4_layer_table* t, int H, int F, int Nqkv, int V, int 
         ok = add(ly.qkv, Nqkv, H) && add(ly.o, H, H) && add(ly.gate_up, 2 * F, H) && add(ly.down, H, F);
     }
     ok = ok && add(t->lm_head, V, H);
-    ok = ok && encode_2d(&p->xH, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, buf.xpH, H, p->NB, static_cast<uint64_t>(H) * 2, 64,
-                         p->NB, CU_TENSOR_MAP_SWIZZLE_128B);
-    ok = ok && encode_2d(&p->xF, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, buf.xpF, F, p->NB, static_cast<uint64_t>(F) * 2, 64,
+    for (int i = 0; i < 2 && ok; ++i)
+        ok = encode_2d(&p->xH[i], CU_TENSOR_MAP_DATA_TYPE_FLOAT16, buf.xpH[i], H, 32, static_cast<uint64_t>(H) * 2, 64,
+                       p->NB, CU_TENSOR_MAP_SWIZZLE_128B);
+    ok = ok && encode_2d(&p->xF, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, buf.xpF, F, 32, static_cast<uint64_t>(F) * 2, 64,
                          p->NB, CU_TENSOR_MAP_SWIZZLE_128B);
     ok = ok && set_stage_attr<16>() == 0 && set_stage_attr<32>() == 0;
     if (!ok) {
@@ -492,91 +671,115 @@ int tc_plan_create(const wq4_layer_table* t, int H, int F, int Nqkv, int V, int 
 
 void tc_plan_destroy(TcPlan* p) { delete p; }
 
-// Records one token on `cs` (inside a stream capture).
-void tc_record_token(const TcPlan* p, cudaStream_t cs)
+// Records one token on `cs` (inside a stream capture): the prologue, then per
+// layer the QKV, O, gate_up and down stages, then the LM head.  Every launch
+// may overlap its set-up and weight stream with the tail of the previous one
+// (programmatic dependent launch); it reads the previous stage's outputs only
+// after that grid has completed.
+int tc_record_token(const TcPlan* p, cudaStream_t cs)
 {
     const int B = p->B, H = p->H, F = p->F, L = p->L;
     const TcBuffers& u = p->buf;
     const size_t LH = static_cast<size_t>(B) * H;
-    auto stage = [&](const TcMatMaps& m, const CUtensorMap& xmap) {
-        const int tiles = (m.N + 127) / 128, nch = m.K / 256;
-        int P = p->sms / tiles;
-        if (P < 1) P = 1;
-        if (P > nch) P = nch;
-        const int units = tiles * P;
-        const int grid = units < p->sms ? units : p->sms;
-        if (p->NB == 16)
-            tc_stage_kernel<16><<<grid, kTcThreads, TcSmem<16>::kBytes, cs>>>(m.codes, m.scales, xmap, m.N, m.K, B, P,
-                                                                             units, u.part, p->err);
-        else
-            tc_stage_kernel<32><<<grid, kTcThreads, TcSmem<32>::kBytes, cs>>>(m.codes, m.scales, xmap, m.N, m.K, B, P,
-                                                                             units, u.part, p->err);
-        return P;
+    float* sq_u = u.sq;                                           // [H/128][B] each
+    float* sq_a = u.sq + static_cast<size_t>(H / 128) * B;
+    float* sq_x1 = u.sq + 2 * static_cast<size_t>(H / 128) * B;
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    bool ok = true;
+    auto stage = [&](int type, const TcMatMaps& m, const CUtensorMap& xmap, TcArgs a) {
+        const int tiles = type == kTcGU ? F / 64 : (m.N + 127) / 128;
+        const int P = stage_parts(tiles, m.K / 256, p->sms);
+        a.type = type;
+        a.N = m.N;
+        a.K = m.K;
+        a.B = B;
+        a.P = P;
+        a.tiles = tiles;
+        a.units = tiles * P;
+        a.H = H;
+        a.F = F;
+        a.eps = p->eps;
+        a.part = u.part;
+        a.cnt = u.cnt;
+        a.err = p->err;
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(a.units < p->sms ? a.units : p->sms);
+        cfg.blockDim = dim3(kTcThreads);
+        cfg.stream = cs;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        cudaError_t e;
+        if (p->NB == 16) {
+            cfg.dynamicSmemBytes = TcSmem<16>::kBytes;
+            e = cudaLaunchKernelEx(&cfg, tc_stage_kernel<16>, m.codes, m.scales, xmap, a);
+        } else {
+            cfg.dynamicSmemBytes = TcSmem<32>::kBytes;
+            e = cudaLaunchKernelEx(&cfg, tc_stage_kernel<32>, m.codes, m.scales, xmap, a);
+        }
+        ok = ok && e == cudaSuccess;
     };
-    auto epi = [&](TcEpi e, int nvec_max) {
-        e.B = B;
-        e.H = H;
-        e.F = F;
-        e.eps = p->eps;
-        e.part = u.part;
-        tc_epilogue_kernel<<<B, 1024, 2 * nvec_max, cs>>>(e);
-    };
-    float* rf = u.rf;   // [L + 1][3][B]
-    tc_prologue_kernel<<<B, 1024, 0, cs>>>(u.x_stage, H, p->eps, rf, u.pV, u.xpH);
-    for (int l = 0; l < L; ++l) {
-        float* r = rf + static_cast<size_t>(3 * l) * B;
-        const TcMatMaps* m = &p->mats[4 * static_cast<size_t>(l)];
-        TcEpi e{};
-        e.type = kTcQKV;
-        e.N = p->Nqkv;
-        e.P = stage(m[0], p->xH);
-        e.r_in = r;
-        e.y = u.pQKV + static_cast<size_t>(l) * B * p->Nqkv;
-        e.r_out = r + B;
-        e.xp = u.xpH;
-        epi(e, H);
-
-        e = TcEpi{};
-        e.type = kTcO;
-        e.N = H;
-        e.P = stage(m[1], p->xH);
-        e.r_in = r + B;
-        e.v_in = u.pV + static_cast<size_t>(l) * LH;
-        e.y = u.pO + static_cast<size_t>(l) * LH;
-        e.y2 = u.pX1 + static_cast<size_t>(l) * LH;
-        e.r_out = r + 2 * B;
-        e.xp = u.xpH;
-        epi(e, H);
-
-        e = TcEpi{};
-        e.type = kTcGU;
-        e.N = 2 * F;
-        e.P = stage(m[2], p->xH);
-        e.r_in = r + 2 * B;
-        e.y = u.pGU + static_cast<size_t>(l) * B * 2 * F;
-        e.y2 = u.pM + static_cast<size_t>(l) * B * F;
-        e.xp = u.xpF;
-        epi(e, F);
-
-        e = TcEpi{};
-        e.type = kTcDOWN;
-        e.N = H;
-        e.P = stage(m[3], p->xF);
-        e.v_in = u.pX1 + static_cast<size_t>(l) * LH;
-        e.y = u.pD + static_cast<size_t>(l) * LH;
-        e.y2 = u.pX2 + static_cast<size_t>(l) * LH;
-        e.r_out = r + 3 * B;                                   // next layer's (or the LM head's) factor
-        e.v_out = u.pV + static_cast<size_t>(l + 1) * LH;
-        e.xp = u.xpH;
-        epi(e, H);
+    {
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(B);
+        cfg.blockDim = dim3(128);
+        cfg.stream = cs;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        ok = ok && cudaLaunchKernelEx(&cfg, tc_prologue_kernel, u.x_stage, H, B, sq_u, u.xpH[0]) == cudaSuccess;
     }
-    TcEpi e{};
-    e.type = kTcLM;
-    e.N = p->V;
-    e.P = stage(p->mats[4 * static_cast<size_t>(L)], p->xH);
-    e.r_in = rf + static_cast<size_t>(3 * L) * B;
-    e.y = u.logits;
-    epi(e, 0);
+    int hb = 0;   // which permuted H buffer holds the current stage's input
+    for (int l = 0; l < L; ++l) {
+        const TcMatMaps* m = &p->mats[4 * static_cast<size_t>(l)];
+        const uint16_t* ul = (l == 0) ? u.x_stage : u.pX2 + static_cast<size_t>(l - 1) * LH;
+        TcArgs a{};
+        a.sq_in = sq_u;
+        a.y = u.pQKV + static_cast<size_t>(l) * B * p->Nqkv;
+        a.sq_out = sq_a;
+        a.xp = u.xpH[hb ^ 1];
+        a.ldxp = H;
+        stage(kTcQKV, m[0], p->xH[hb], a);
+        hb ^= 1;
+
+        a = TcArgs{};
+        a.sq_in = sq_a;
+        a.sq_u = sq_u;
+        a.res = ul;
+        a.y = u.pO + static_cast<size_t>(l) * LH;
+        a.y2 = u.pX1 + static_cast<size_t>(l) * LH;
+        a.y3 = u.pV + static_cast<size_t>(l) * LH;
+        a.sq_out = sq_x1;
+        a.xp = u.xpH[hb ^ 1];
+        a.ldxp = H;
+        stage(kTcO, m[1], p->xH[hb], a);
+        hb ^= 1;
+
+        a = TcArgs{};
+        a.sq_in = sq_x1;
+        a.y = u.pGU + static_cast<size_t>(l) * B * 2 * F;
+        a.y2 = u.pM + static_cast<size_t>(l) * B * F;
+        a.xp = u.xpF;
+        a.ldxp = F;
+        stage(kTcGU, m[2], p->xH[hb], a);
+
+        a = TcArgs{};
+        a.res = u.pX1 + static_cast<size_t>(l) * LH;
+        a.y = u.pD + static_cast<size_t>(l) * LH;
+        a.y2 = u.pX2 + static_cast<size_t>(l) * LH;
+        a.sq_out = sq_u;                      // the next layer's (or the LM head's) input
+        a.xp = u.xpH[hb ^ 1];
+        a.ldxp = H;
+        stage(kTcDOWN, m[3], p->xF, a);
+        hb ^= 1;
+    }
+    TcArgs a{};
+    a.sq_in = sq_u;
+    a.res = u.pX2 + static_cast<size_t>(L - 1) * LH;
+    a.y = u.logits;
+    a.y3 = u.pV + static_cast<size_t>(L) * LH;
+    stage(kTcLM, p->mats[4 * static_cast<size_t>(L)], p->xH[hb], a);
+    return ok ? WQ4_OK : WQ4_ERR_CUDA;
 }
 
 }  // namespace wq4

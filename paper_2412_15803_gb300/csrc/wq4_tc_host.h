@@ -24,25 +24,14 @@ struct TcBuffers {
     uint16_t* pD;              // [L][B][H]
     uint16_t* pX2;             // [L][B][H]
     uint16_t* logits;          // [B][V]
-    float* rf;                 // [L+1][3][B] RMS factors
-    uint16_t* xpH;             // [32][H] permuted stage input (K = H)
+    float* sq;                 // 3 x [H/128][B] sums of squares of 128-element tiles (u, a, x1)
+    uint32_t* cnt;             // [kTcCounterWords] arrival counters, zero-initialised
+    uint16_t* xpH[2];          // [32][H] permuted stage inputs (K = H), alternating
     uint16_t* xpF;             // [32][F] permuted stage input (K = F)
     float* part;               // fp32 partial sums [P][B][N]
 };
 
-// Arguments of one stage epilogue (one CTA per batch row).
-struct TcEpi {
-    int type, N, B, P, H, F;
-    float eps;
-    const float* part;
-    const float* r_in;       // row factor of the stage (null: 1)
-    const uint16_t* v_in;    // residual input (O: v, down: x1)
-    uint16_t* y;             // stage output trace
-    uint16_t* y2;            // second output (O: x1, gate_up: m, down: x2)
-    uint16_t* v_out;         // down: next layer's normalised input
-    float* r_out;            // RMS factor of the next stage's input (null: none)
-    uint16_t* xp;            // next stage's permuted input row
-};
+constexpr int kTcCounterWords = 4096;
 
 struct TcPlan;
 
@@ -53,7 +42,7 @@ int tc_plan_create(const wq4_layer_table* t, int H, int F, int Nqkv, int V, int 
                    uint32_t* err, TcPlan** out);
 void tc_plan_destroy(TcPlan* p);
 
-// Records one token (every stage kernel and epilogue) on `cs`.
-void tc_record_token(const TcPlan* p, cudaStream_t cs);
+// Records one token (prologue and every stage kernel) on `cs`.
+int tc_record_token(const TcPlan* p, cudaStream_t cs);
 
 }  // namespace wq4

@@ -168,14 +168,15 @@ size_t wq4_chain_workspace_bytes(const wq4_layer_table* table);
  * residual stream.
  *   x      : fp16 [batch][hidden] device, 16-byte aligned
  *   logits : fp16 [batch][vocab]  device, 2-byte aligned
- * Batch 1-4 runs as the persistent kernel above.  Batch 5-32 runs as a CUDA
- * graph of stage kernels (RMS factors, a CUDA-core stage GEMV with the row
- * factor and the residual add fused, SiLU * up), captured once per table;
- * each call copies x into the workspace, replays the graph and copies the
- * logits out (all on `stream`).
+ * Batch 1-2 runs as the persistent kernel above.  Batch 3-32 runs as a CUDA
+ * graph, captured once per table, of one tensor-core kernel per projection
+ * (dequantized fp16 weights w = fp16((q - 7) s) times the batch's inputs,
+ * tcgen05 MMAs with fp32 accumulation, the chain's row factors, residual adds
+ * and SiLU fused into each stage's epilogue); each call copies x into the
+ * workspace, replays the graph and copies the logits out (all on `stream`).
  * The first call for a table (or after its contents changed) validates it and
  * uploads its pointer table into the workspace (cudaMemcpyAsync on `stream`);
- * later calls only launch.  Rebuilding the plan of a batch 5-32 table
+ * later calls only launch.  Rebuilding the plan of a batch 3-32 table
  * synchronizes `stream` before freeing the old graph.  Calls on one table must
  * not overlap on the GPU.
  * Returns WQ4_OK, WQ4_ERR_INVALID, WQ4_ERR_ALIGN, WQ4_ERR_UNSUPPORTED or

@@ -52,7 +52,7 @@ constexpr int kChainMaxSlots = 16;
 // for every stage, which bounds how far ahead of the oldest unconsumed chunk
 // a warp can be (nslots - 1 + ceil(NW / items per slot) chunks).
 constexpr int kFullBars = 48;
-constexpr int kMaxChainBatch = 4;
+constexpr int kMaxChainBatch = 2;   // larger batches take the tensor-core graph path
 // A ring slot is released after kSlotRelease arrivals: one per item consumed
 // from it, plus (kSlotRelease - items) from the warp that consumed its first
 // item.  Only warps that own items of a chunk touch its barriers.
@@ -74,10 +74,10 @@ __host__ __device__ constexpr int chain_header_bytes(int, int)
 }
 
 // Consumer warps per CTA: with the producer warp, 16 warps (128 registers a
-// thread) for batch 1-2, 8 warps (255 registers) for batch 3-4.
+// thread).
 template <int B>
 struct ChainWarps {
-    static constexpr int NW = (B <= 2) ? 15 : 7;
+    static constexpr int NW = 15;
 };
 
 enum StageType { kQKV = 0, kO = 1, kGU = 2, kDOWN = 3, kLM = 4 };
@@ -745,7 +745,7 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
     }
 }
 
-// ------------------------------------------------- graph path (batch 5-32) --
+// ------------------------------------------------- graph path (batch 3-32) --
 //
 // For batches beyond what the persistent kernel stages in shared memory, the
 // token runs as a CUDA graph (captured once per plan) of tensor-core stage
@@ -871,8 +871,7 @@ int chain_warps(int B)
     switch (B) {
         case 1: return ChainWarps<1>::NW;
         case 2: return ChainWarps<2>::NW;
-        case 3: return ChainWarps<3>::NW;
-        default: return ChainWarps<4>::NW;
+        default: return ChainWarps<2>::NW;
     }
 }
 
@@ -1030,9 +1029,7 @@ int build_plan(const wq4_layer_table* t, Plan* pl, cudaStream_t stream)
     cudaError_t e = cudaSuccess;
     switch (d.B) {
         case 1: e = set_chain_attr<1>(di->smem_optin); break;
-        case 2: e = set_chain_attr<2>(di->smem_optin); break;
-        case 3: e = set_chain_attr<3>(di->smem_optin); break;
-        default: e = set_chain_attr<4>(di->smem_optin); break;
+        default: e = set_chain_attr<2>(di->smem_optin); break;
     }
     if (e != cudaSuccess) return WQ4_ERR_CUDA;
 
@@ -1134,8 +1131,7 @@ int launch_chain(const Plan& pl, const uint16_t* x, uint16_t* logits, cudaStream
     switch (pl.dims.B) {
         case 1: e = cudaLaunchKernelEx(&cfg, chain_kernel<1, ChainWarps<1>::NW>, p); break;
         case 2: e = cudaLaunchKernelEx(&cfg, chain_kernel<2, ChainWarps<2>::NW>, p); break;
-        case 3: e = cudaLaunchKernelEx(&cfg, chain_kernel<3, ChainWarps<3>::NW>, p); break;
-        default: e = cudaLaunchKernelEx(&cfg, chain_kernel<4, ChainWarps<4>::NW>, p); break;
+        default: e = cudaLaunchKernelEx(&cfg, chain_kernel<2, ChainWarps<2>::NW>, p); break;
     }
     return e == cudaSuccess ? WQ4_OK : WQ4_ERR_CUDA;
 }

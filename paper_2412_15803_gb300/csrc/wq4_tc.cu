@@ -1,6 +1,6 @@
-// wq4_tc.cu -- batched decode chain on the tensor cores (batch 5-32).
+// wq4_tc.cu -- batched decode chain on the tensor cores (batch 3-32).
 //
-// Above batch 4 the per-weight FMA work of the CUDA-core path grows with the
+// Above batch 2 the per-weight FMA work of the CUDA-core path grows with the
 // batch while the weight stream does not; here every projection becomes a
 // dequantize + tcgen05 GEMM: y[b][n] = sum_k w[n][k] x[b][k] with
 // w = fp16((q - 7) s) (one rounding per weight, at most 2^-11 relative, then

@@ -36,6 +36,7 @@ sys.path.insert(0, ROOT)
 
 METRIC = "GEMV-bound decode tokens/s (batch 1) and achieved HBM GB/s vs ~8 TB/s peak"
 NOMINAL_HBM_GBS = 8000.0
+PERSISTENT_MAX_BATCH = 2      # larger batches run the tensor-core graph path
 FALLBACK_HBM_GBS = 6800.0
 
 
@@ -70,7 +71,7 @@ def measured_peak():
 
 def chain_source_sha() -> str:
     h = hashlib.sha256()
-    for f in ("wq4_chain.cu", "wq4_device.cuh"):
+    for f in ("wq4_chain.cu", "wq4_device.cuh", "wq4_tc.cu", "wq4_tc.cuh"):
         h.update(open(os.path.join(ROOT, "paper_2412_15803_gb300", "csrc", f), "rb").read())
     return h.hexdigest()[:16]
 
@@ -78,7 +79,8 @@ def chain_source_sha() -> str:
 def profiled_traffic(workload: str, batch: int):
     """DRAM bytes per launch from the committed ncu summary, if it was taken
     on the current kernel source (else None)."""
-    path = os.path.join(ROOT, "profiles", f"chain_kernel_{workload}_b{batch}.md")
+    name = "chain_kernel" if batch <= PERSISTENT_MAX_BATCH else "tc_stage_kernel"
+    path = os.path.join(ROOT, "profiles", f"{name}_{workload}_b{batch}.md")
     if not os.path.exists(path):
         return None
     text = open(path).read()
@@ -299,6 +301,12 @@ def run_ours(args, rank, world, local):
     e2e_s = time.perf_counter() - t0
     tokens_per_s, e2e_val, total_ms_max = aggregate_replicas(total_ms, e2e_s / e2e_steps, B, args.steps, "cuda")
 
+    if B <= PERSISTENT_MAX_BATCH:
+        # one cooperative launch of the persistent chain kernel per token
+        kernel_name, launches_per_step = "chain_kernel", 1
+    else:
+        # one CUDA-graph replay: a prologue and one tensor-core stage kernel per projection
+        kernel_name, launches_per_step = "tc_stage_kernel", 4 * shape.num_layers + 2
     if rank == 0:
         ms = total_ms_max / args.steps
         avg_launch_ms = statistics.mean(launch_ms)
@@ -319,7 +327,7 @@ def run_ours(args, rank, world, local):
                        "parallelism": "replicas" if world > 1 else "single GPU"},
             "hbm_gbs": step_bytes * args.steps / (total_ms_max / 1e3) / 1e9,
             "hbm_frac_of_nominal_8tbs": step_bytes * args.steps / (total_ms_max / 1e3) / 1e9 / NOMINAL_HBM_GBS,
-            "roofline": {"bound": "hbm", "kernel": "chain_kernel", "achieved": achieved, "peak": peak,
+            "roofline": {"bound": "hbm", "kernel": kernel_name, "achieved": achieved, "peak": peak,
                          "peak_source": peak_src, "unit": "GB/s", "frac": achieved / peak,
                          "frac_of_nominal_8tbs": achieved / NOMINAL_HBM_GBS,
                          "traffic": profiled_traffic(args.workload, B),
@@ -327,7 +335,7 @@ def run_ours(args, rank, world, local):
                          "avg_launch_ms": avg_launch_ms},
             "e2e": {"value": e2e_val, "unit": "tokens/s", "h2d_bytes_per_step": 2 * B * shape.hidden,
                     "d2h_bytes_per_step": 2 * B * shape.vocab},
-            "gpu_launches": args.steps,
+            "gpu_launches": args.steps * launches_per_step,
             "clocks": clocks,
         }
         if world == 1 and not args.no_cpu_baseline:

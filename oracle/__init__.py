@@ -4,8 +4,10 @@ TEST INFRASTRUCTURE ONLY: only the tests, ``__graft_entry__.smoke()`` and the
 benchmark's CPU-baseline leg may import this package.  The product library
 (``paper_2412_15803_gb300``) never imports it, and the two share no code.
 
-The arithmetic lives in ``wq4_oracle.c`` (plain C, fp64, single-threaded);
-this module compiles it with gcc and wraps it with ctypes and numpy.  Every
+The arithmetic lives in ``wq4_oracle.c`` (the GEMV and the chain glue) and
+``attention_oracle.c`` (decode attention over a paged key/value cache), plain
+C, fp64, single-threaded; this module compiles them with gcc and wraps them
+with ctypes and numpy.  Every
 array is passed as raw bit patterns: fp16 values travel as uint16.
 """
 from __future__ import annotations
@@ -17,7 +19,7 @@ import subprocess
 import numpy as np
 
 _HERE = os.path.dirname(os.path.abspath(__file__))
-_SRC = os.path.join(_HERE, "wq4_oracle.c")
+_SRCS = [os.path.join(_HERE, "wq4_oracle.c"), os.path.join(_HERE, "attention_oracle.c")]
 _BUILD = os.path.join(_HERE, "_build")
 _LIB_PATH = os.path.join(_BUILD, "liboracle.so")
 
@@ -30,10 +32,10 @@ def build(force: bool = False) -> str:
     """Compile the oracle into oracle/_build/liboracle.so (gcc)."""
     os.makedirs(_BUILD, exist_ok=True)
     if (not force and os.path.exists(_LIB_PATH)
-            and os.path.getmtime(_LIB_PATH) >= os.path.getmtime(_SRC)):
+            and all(os.path.getmtime(_LIB_PATH) >= os.path.getmtime(f) for f in _SRCS)):
         return _LIB_PATH
     tmp = _LIB_PATH + f".tmp{os.getpid()}"
-    subprocess.check_call(["gcc", *CFLAGS, _SRC, "-o", tmp, "-lm"])
+    subprocess.check_call(["gcc", *CFLAGS, *_SRCS, "-o", tmp, "-lm"])
     os.replace(tmp, _LIB_PATH)
     return _LIB_PATH
 
@@ -67,6 +69,10 @@ def lib() -> ctypes.CDLL:
         _lib.wq4o_rms_normalize.argtypes = [P, I, D, P]
         _lib.wq4o_silu_mul.argtypes = [P, P, I, P, P]
         _lib.wq4o_add_fp16.argtypes = [P, P, I, P]
+        _lib.wq4o_paged_attention.argtypes = [P, I, P, P, I, I, P, I, P, I, I, I, I, D, P, P, P]
+        _lib.wq4o_paged_attention.restype = I
+        _lib.wq4o_kv_append.argtypes = [P, P, I, P, P, I, I, P, I, P, I, I, I]
+        _lib.wq4o_kv_append.restype = I
     return _lib
 
 
@@ -185,3 +191,72 @@ def add_fp16(a, b) -> np.ndarray:
     z = np.empty(a.shape, np.uint16)
     lib().wq4o_add_fp16(_p(a), _p(b), a.size, _p(z))
     return z
+
+
+# -------------------------------------------------------------- attention --
+
+def paged_attention(q, k_cache, v_cache, page_table, seq_lens, scale: float, n_q_heads: int):
+    """Decode attention over a paged cache (definition in attention_oracle.c).
+
+    q          fp16 bits [batch][>= n_q_heads * head_dim] (row stride = q.shape[1])
+    k_cache,
+    v_cache    fp16 bits [num_pages][n_kv_heads][page_size][head_dim]
+    page_table int32 [batch][pt_stride]
+    seq_lens   int32 [batch]
+
+    Returns (o fp64, A fp64, o16 fp16 bits), each [batch][n_q_heads][head_dim]."""
+    q = _c(q, np.uint16)
+    k_cache = _c(k_cache, np.uint16)
+    v_cache = _c(v_cache, np.uint16)
+    page_table = _c(np.atleast_2d(page_table), np.int32)
+    seq_lens = _c(seq_lens, np.int32)
+    num_pages, n_kv, page_size, head_dim = k_cache.shape
+    assert v_cache.shape == k_cache.shape
+    batch = seq_lens.shape[0]
+    q2 = q.reshape(batch, -1)
+    o = np.empty((batch, n_q_heads, head_dim), np.float64)
+    A = np.empty_like(o)
+    o16 = np.empty(o.shape, np.uint16)
+    rc = lib().wq4o_paged_attention(_p(q2), q2.shape[1], _p(k_cache), _p(v_cache), num_pages, page_size,
+                                    _p(page_table), page_table.shape[1], _p(seq_lens), batch, n_q_heads, n_kv,
+                                    head_dim, float(scale), _p(o), _p(A), _p(o16))
+    if rc != 0:
+        raise ValueError("paged_attention: bad page id or head grouping")
+    return o, A, o16
+
+
+def kv_append(new_k, new_v, k_cache, v_cache, page_table, positions):
+    """Writes each sequence's new key/value rows into the cache (in place).
+
+    new_k, new_v fp16 bits [batch][>= n_kv_heads * head_dim]; the caches are
+    modified in place.  Raises on a bad position or page id (after writing the
+    other sequences)."""
+    new_k = _c(new_k, np.uint16)
+    new_v = _c(new_v, np.uint16)
+    assert k_cache.flags.c_contiguous and v_cache.flags.c_contiguous
+    assert k_cache.dtype == np.uint16 and v_cache.dtype == np.uint16
+    page_table = _c(np.atleast_2d(page_table), np.int32)
+    positions = _c(positions, np.int32)
+    num_pages, n_kv, page_size, head_dim = k_cache.shape
+    batch = positions.shape[0]
+    nk = new_k.reshape(batch, -1)
+    nv = new_v.reshape(batch, -1)
+    assert nk.shape == nv.shape
+    rc = lib().wq4o_kv_append(_p(nk), _p(nv), nk.shape[1], _p(k_cache), _p(v_cache), num_pages, page_size,
+                              _p(page_table), page_table.shape[1], _p(positions), batch, n_kv, head_dim)
+    if rc != 0:
+        raise ValueError("kv_append: bad position or page id")
+
+
+# Tolerance of the attention output.  The GPU path rounds each softmax weight
+# to fp16 (relative error <= 2^-11) before the value product and sums the same
+# rounded weights into the normaliser, so each normalised weight is off by at
+# most about 2 * 2^-11 of itself; fp32 score and accumulation errors add
+# < 1e-4 for scale * sum|q k| <= 64 and sequences of <= 64K tokens.  The bound
+# 2e-3 * A covers both with margin; ulp16(|o|) covers the final rounding.
+ATTN_REL = 2e-3
+
+
+def attention_tolerance(o_ref, A):
+    """Per-element bound |o_gpu - o_ref| <= 2e-3 * A + ulp16(|o_ref|)."""
+    return ATTN_REL * np.asarray(A) + ulp16_array(np.abs(o_ref))

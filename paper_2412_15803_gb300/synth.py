@@ -27,7 +27,15 @@ Drawn tensors (the distributions of the 1-8B 4-bit decode workloads):
   * scales: fp16_RNE(lo + (hi - lo) * u), u = (u64(i) >> 11) * 2^-53,
     evaluated in fp64 as one multiply then one add, lo = 0.005, hi = 0.02;
   * activations: fp16_RNE(sqrt(-2 ln u1) * cos(2 pi u2)) (Box-Muller) with
-    u1 = ((u64(2i) >> 11) + 1) * 2^-53 and u2 = (u64(2i+1) >> 11) * 2^-53.
+    u1 = ((u64(2i) >> 11) + 1) * 2^-53 and u2 = (u64(2i+1) >> 11) * 2^-53;
+  * attention queries, keys and values ("sum4"): the four 16-bit fields of
+    u64(i) summed, centred and scaled, fp16_RNE((a + b + c + d - 131070) *
+    2^-15): an Irwin-Hall(4) approximation of a normal draw with standard
+    deviation 2/sqrt(3) and range [-4, 4].  Integer arithmetic and one
+    rounding, so the device generator reproduces it bit for bit;
+  * page tables: the pages of a pool in the order of an argsort of u64 draws
+    (a random permutation), handed out to the sequences in turn; sequence
+    lengths lo + u64(i) mod (hi - lo + 1).
 
 The CUDA library carries a device implementation of the first two draws (for
 weight matrices too large to generate on the host in reasonable time); the
@@ -51,6 +59,11 @@ SCALE_HI = 0.02
 KIND_CODES = 0
 KIND_SCALES = 1
 KIND_X = 2
+KIND_Q = 3
+KIND_K = 4
+KIND_V = 5
+KIND_PAGES = 6
+KIND_LENS = 7
 
 # projection index within a layer
 MAT_QKV, MAT_O, MAT_GATE_UP, MAT_DOWN, MAT_LM_HEAD = 0, 1, 2, 3, 4
@@ -145,3 +158,50 @@ def matrix(seed: int, N: int, K: int, layer: int = 0, mat: int = 0,
 def activations(seed: int, batch: int, K: int, layer: int = 0) -> np.ndarray:
     """x fp16 bits [batch][K] ~ N(0,1)."""
     return normal_fp16(seed, stream_id(KIND_X, layer, 0), batch * K).reshape(batch, K)
+
+
+def sum4_fp16(seed: int, sid: int, start: int, count: int) -> np.ndarray:
+    """Elements [start, start + count) of a sum4 stream, fp16 bit patterns."""
+    v = u64(key(seed, sid), start, count)
+    m = np.uint64(0xFFFF)
+    c = ((v & m) + ((v >> np.uint64(16)) & m) + ((v >> np.uint64(32)) & m) + (v >> np.uint64(48))).astype(np.int64)
+    return ((c - 131070).astype(np.float64) * 2.0 ** -15).astype(np.float16).view(np.uint16)
+
+
+def seq_lens(seed: int, batch: int, lo: int, hi: int, layer: int = 0) -> np.ndarray:
+    """Sequence lengths uniform on [lo, hi] (int32 [batch])."""
+    v = u64(key(seed, stream_id(KIND_LENS, layer, 0)), 0, batch)
+    return (lo + (v % np.uint64(hi - lo + 1)).astype(np.int64)).astype(np.int32)
+
+
+def page_table(seed: int, lens, page_size: int, num_pages: int, pt_stride: int | None = None,
+               layer: int = 0) -> np.ndarray:
+    """Page table int32 [batch][pt_stride]: sequence b gets ceil(len_b / page_size)
+    pages, taken in turn from a random permutation of the pool; unused entries
+    are -1.  num_pages must cover every sequence's pages."""
+    lens = np.asarray(lens, np.int64)
+    need = (lens + page_size - 1) // page_size
+    if int(need.sum()) > num_pages:
+        raise ValueError("page pool too small")
+    width = int(need.max()) if pt_stride is None else pt_stride
+    order = np.argsort(u64(key(seed, stream_id(KIND_PAGES, layer, 0)), 0, num_pages), kind="stable")
+    table = np.full((len(lens), max(width, 1)), -1, np.int32)
+    off = 0
+    for b, n in enumerate(need):
+        table[b, :n] = order[off:off + n]
+        off += int(n)
+    return table
+
+
+def kv_cache(seed: int, num_pages: int, n_kv_heads: int, page_size: int, head_dim: int, layer: int = 0):
+    """Key and value caches, fp16 bits [num_pages][n_kv_heads][page_size][head_dim] (sum4)."""
+    n = num_pages * n_kv_heads * page_size * head_dim
+    shape = (num_pages, n_kv_heads, page_size, head_dim)
+    k = sum4_fp16(seed, stream_id(KIND_K, layer, 0), 0, n).reshape(shape)
+    v = sum4_fp16(seed, stream_id(KIND_V, layer, 0), 0, n).reshape(shape)
+    return k, v
+
+
+def queries(seed: int, batch: int, n_q_heads: int, head_dim: int, layer: int = 0) -> np.ndarray:
+    """Queries fp16 bits [batch][n_q_heads * head_dim] (sum4)."""
+    return sum4_fp16(seed, stream_id(KIND_Q, layer, 0), 0, batch * n_q_heads * head_dim).reshape(batch, -1)

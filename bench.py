@@ -11,6 +11,12 @@ than L2 (129 MB), so no L2 flush is needed between steps.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
                     [--workload 3b|8b] [--batch B]
+    python bench.py --workload attn-8b|attn-3b|attn-8b-b1     (decode attention)
+
+The attn-* workloads time decode attention of one layer over a paged
+key/value cache instead (wq4_paged_attention, one launch per step): 32
+sequences with context lengths uniform on [1, 8192] (attn-8b-b1: one
+sequence of 4096), Llama-3.1-8B- or 3B-shaped heads, pages of 16 tokens.
 
 --impl reference times the fp64 CPU oracle on a bounded sample of the same
 workload (the only reference this repository has: the paper's WebGPU/Metal
@@ -46,7 +52,7 @@ def parse():
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=["3b", "8b"], default="3b")
+    ap.add_argument("--workload", choices=["3b", "8b", "attn-8b", "attn-3b", "attn-8b-b1"], default="3b")
     ap.add_argument("--batch", type=int, default=1)
     ap.add_argument("--layers", type=int, default=0, help="override the layer count (profiling runs)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -345,13 +351,205 @@ def run_ours(args, rank, world, local):
         dist.destroy_process_group()
 
 
+# -------------------------------------------------------------- attention --
+
+ATTN_METRIC = "paged decode attention sequences/s (one decode step per sequence) and achieved HBM GB/s"
+L2_BYTES = 129 * 1024 * 1024
+
+
+def attn_source_sha() -> str:
+    h = hashlib.sha256()
+    for f in ("wq4_attn.cu", "wq4_device.cuh"):
+        h.update(open(os.path.join(ROOT, "paper_2412_15803_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def attn_profiled_traffic(workload: str):
+    path = os.path.join(ROOT, "profiles", f"paged_attn_kernel_{workload}.md")
+    if not os.path.exists(path):
+        return None
+    text = open(path).read()
+    m = re.search(r"traffic_bytes_per_launch:\s*(\d+)", text)
+    s = re.search(r"source_sha:\s*([0-9a-f]+)", text)
+    if not m or not s or s.group(1) != attn_source_sha():
+        return None
+    return int(m.group(1))
+
+
+def attn_oracle_sample(w, seed: int, target_s: float):
+    """Times the fp64 oracle on whole sequences of the workload (shortest
+    first, sequences regenerated on the host) until about target_s seconds
+    have been spent; returns (seconds, tokens of context processed, sequences)."""
+    import oracle
+    from paper_2412_15803_gb300 import synth
+    sh = w.shape
+    lens = w.lens(seed)
+    P, D = w.page_size, sh.head_dim
+    num_pages = int(((lens.astype(np.int64) + P - 1) // P).sum())
+    table = synth.page_table(seed, lens, P, num_pages)
+    per = sh.n_kv_heads * P * D
+    spent, toks, nseq = 0.0, 0, 0
+    for b in np.argsort(lens, kind="stable"):
+        T = int(lens[b])
+        n = (T + P - 1) // P
+        pages = table[b, :n]
+        k = np.stack([synth.sum4_fp16(seed, synth.stream_id(synth.KIND_K, 0, 0), int(p) * per, per) for p in pages])
+        v = np.stack([synth.sum4_fp16(seed, synth.stream_id(synth.KIND_V, 0, 0), int(p) * per, per) for p in pages])
+        k = k.reshape(n, sh.n_kv_heads, P, D)
+        v = v.reshape(n, sh.n_kv_heads, P, D)
+        q = synth.sum4_fp16(seed, synth.stream_id(synth.KIND_Q, 0, 0), int(b) * sh.n_q_heads * D, sh.n_q_heads * D)
+        t0 = time.perf_counter()
+        oracle.paged_attention(q[None, :], k, v, np.arange(n, dtype=np.int32)[None, :], np.array([T], np.int32),
+                               1.0 / np.sqrt(D), sh.n_q_heads)
+        spent += time.perf_counter() - t0
+        toks += T
+        nseq += 1
+        if spent >= target_s:
+            break
+    return spent, toks, nseq
+
+
+def attn_cpu_line(w, seed: int, target_s: float):
+    t, toks, nseq = attn_oracle_sample(w, seed, target_s)
+    total_toks = int(w.lens(seed).astype(np.int64).sum())
+    est = t * total_toks / max(toks, 1)
+    return {"value": w.batch / est, "unit": "sequences/s", "cores": 1, "kind": "oracle",
+            "sample": f"{nseq} of the {w.batch} sequences (shortest first, {toks} of {total_toks} context "
+                      f"tokens), single-threaded fp64 C oracle, {t:.1f} s, scaled to the whole batch"}
+
+
+def attn_config(w, layers: int):
+    sh = w.shape
+    return {"workload": f"{w.name}: decode attention of one {sh.name}-shaped layer ({sh.n_q_heads} q / "
+                        f"{sh.n_kv_heads} kv heads of {sh.head_dim}), batch {w.batch}, context lengths "
+                        f"uniform on [{w.len_lo}, {w.len_hi}], pages of {w.page_size} tokens, fp16 cache",
+            "batch": w.batch, "page_size": w.page_size,
+            "l2": ("inputs larger than L2, no flush" if layers == 1 else
+                   f"{layers} distinct layers' caches in rotation (together larger than L2)"),
+            "parallelism": "single GPU"}
+
+
+def run_attn_reference(args, rank, world):
+    from paper_2412_15803_gb300.attention import ATTN_WORKLOADS
+    if rank != 0:
+        return
+    w = ATTN_WORKLOADS[args.workload]
+    nsteps = args.steps + args.warmup
+    step_s = min(10.0, 120.0 / max(nsteps, 1))
+    times = []
+    total_toks = int(w.lens(0).astype(np.int64).sum())
+    for i in range(nsteps):
+        t, toks, _ = attn_oracle_sample(w, 0, step_s)
+        if i >= args.warmup:
+            times.append(t * total_toks / max(toks, 1))
+    value = w.batch / statistics.mean(times)
+    line = {"metric": ATTN_METRIC, "value": value, "unit": "sequences/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": 1e3 * statistics.mean(times), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+            "config": attn_config(w, 1),
+            "cpu_baseline": {"value": value, "unit": "sequences/s", "cores": 1, "kind": "oracle",
+                             "sample": f"each step: shortest sequences first for about {step_s:.1f} s of oracle "
+                                       "time, scaled to the whole batch"},
+            "e2e": {"value": value, "unit": "sequences/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def run_attn(args, rank, world, local):
+    import torch
+    import torch.distributed as dist
+    from paper_2412_15803_gb300 import wq4
+    from paper_2412_15803_gb300.attention import ATTN_WORKLOADS, PagedAttentionLayer
+
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    w = ATTN_WORKLOADS[args.workload]
+    lens = w.lens(0)
+    first = PagedAttentionLayer(w.shape, lens, page_size=w.page_size, seed=0, layer=0)
+    nlayers = 1
+    if first.kv_bytes() < 4 * L2_BYTES:
+        nlayers = int(np.ceil(4 * L2_BYTES / first.kv_bytes()))
+    layers = [first] + [PagedAttentionLayer(w.shape, lens, page_size=w.page_size, seed=0, layer=l)
+                        for l in range(1, nlayers)]
+    stream = torch.cuda.current_stream()
+    for i in range(max(args.warmup, 3)):
+        layers[i % nlayers].run(stream)
+    torch.cuda.synchronize()
+    if wq4.wq4_device_status(stream) != 0:
+        raise RuntimeError("attention flagged an error during warm-up")
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.3)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    for i in range(args.steps):
+        starts[i].record(stream)
+        layers[i % nlayers].run(stream)
+        ends[i].record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clocks = sampler.stop()
+    total_ms = starts[0].elapsed_time(ends[-1])
+    launch_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+    if wq4.wq4_device_status(stream) != 0:
+        raise RuntimeError("attention flagged an error during the timed region")
+
+    # end to end: queries copied in from pinned host memory, the call, outputs copied back
+    L0 = layers[0]
+    q_host = L0.q.cpu().pin_memory()
+    o_host = torch.empty_like(L0.out, device="cpu").pin_memory()
+    e2e_steps = max(10, min(args.steps, 500))
+    t0 = time.perf_counter()
+    for i in range(e2e_steps):
+        Li = layers[i % nlayers]
+        Li.q.copy_(q_host, non_blocking=True)
+        Li.run(stream)
+        o_host.copy_(Li.out, non_blocking=True)
+        torch.cuda.current_stream().synchronize()
+    e2e_s = time.perf_counter() - t0
+    seq_per_s, e2e_val, total_ms_max = aggregate_replicas(total_ms, e2e_s / e2e_steps, w.batch, args.steps, "cuda")
+    if rank == 0:
+        avg_launch_ms = statistics.mean(launch_ms)
+        peak, peak_src = measured_peak()
+        step_bytes = L0.algorithmic_bytes()
+        achieved = step_bytes / (avg_launch_ms * 1e-3) / 1e9
+        line = {
+            "metric": ATTN_METRIC, "value": seq_per_s, "unit": "sequences/s", "n_gpus": world,
+            "steps": args.steps, "warmup": args.warmup, "ms_per_step": total_ms_max / args.steps,
+            "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "precision": "fp16 cache and queries, fp32 scores and sums, weights rounded to fp16 for the value product",
+            "data": "synthetic (seeded sum4 keys, values and queries; random page tables)",
+            "config": attn_config(w, nlayers),
+            "hbm_gbs": step_bytes * args.steps / (total_ms_max / 1e3) / 1e9,
+            "roofline": {"bound": "hbm", "kernel": "paged_attn_kernel", "achieved": achieved, "peak": peak,
+                         "peak_source": peak_src, "unit": "GB/s", "frac": achieved / peak,
+                         "frac_of_nominal_8tbs": achieved / NOMINAL_HBM_GBS,
+                         "traffic": attn_profiled_traffic(args.workload),
+                         "algorithmic_bytes_per_launch": step_bytes, "avg_launch_ms": avg_launch_ms},
+            "e2e": {"value": e2e_val, "unit": "sequences/s", "h2d_bytes_per_step": L0.q.numel() * 2,
+                    "d2h_bytes_per_step": L0.out.numel() * 2},
+            "gpu_launches": args.steps,
+            "clocks": clocks,
+        }
+        if world == 1 and not args.no_cpu_baseline:
+            line["cpu_baseline"] = attn_cpu_line(w, 0, 12.0)
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
 def main():
     args = parse()
     rank, world, local = dist_env()
+    attn = args.workload.startswith("attn")
     if args.impl == "reference":
-        run_reference(args, rank, world)
+        (run_attn_reference if attn else run_reference)(args, rank, world)
     else:
-        run_ours(args, rank, world, local)
+        (run_attn if attn else run_ours)(args, rank, world, local)
 
 
 if __name__ == "__main__":

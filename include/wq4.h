@@ -100,8 +100,11 @@ const char* wq4_status_string(int status);
  * Reads and clears the library's device status word on `stream` (this call
  * synchronizes the stream).  *flags_out receives the bits that were set:
  * bit 0 = an mbarrier wait of a weight pipeline gave up, bit 1 = a wait on
- * another CTA's activations gave up.  Returns WQ4_ERR_TIMEOUT if any bit
- * was set, WQ4_OK otherwise, WQ4_ERR_CUDA on a CUDA failure.
+ * another CTA's activations gave up; wq4_attn.h calls add bit 3 = a sequence
+ * length beyond its page table (clamped), bit 4 = a page id outside the pool
+ * (zeros read in its place), bit 5 = an append with a bad position or page
+ * id (nothing written).  Returns WQ4_ERR_TIMEOUT if any bit was set, WQ4_OK
+ * otherwise, WQ4_ERR_CUDA on a CUDA failure.
  */
 int wq4_device_status(void* stream, int* flags_out);
 

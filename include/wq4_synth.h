@@ -1,5 +1,6 @@
 /*
- * wq4_synth.h -- device-side seeded generator for synthetic packed weights.
+ * wq4_synth.h -- device-side seeded generator for synthetic packed weights
+ * and attention inputs.
  *
  * Not part of the method: it only fills buffers with random bits so that
  * large synthetic models (1-8B parameters) can be created directly in HBM.
@@ -36,6 +37,12 @@ int wq4_synth_codes(uint32_t* W, int64_t word_start, int64_t nwords,
  * a single rounding to fp16.  s: device uint16 buffer of n entries. */
 int wq4_synth_scales(uint16_t* s, int64_t start, int64_t n, uint64_t seed,
                      uint64_t sid, double lo, double hi, void* stream);
+
+/* Attention inputs [start, start + n) ("sum4"): fp16_RNE((a + b + c + d -
+ * 131070) * 2^-15), a..d the four 16-bit fields of u64(key, i) (an
+ * Irwin-Hall approximation of a normal draw, standard deviation 2/sqrt(3)).
+ * out: device uint16 buffer of n entries. */
+int wq4_synth_sum4(uint16_t* out, int64_t start, int64_t n, uint64_t seed, uint64_t sid, void* stream);
 
 #ifdef __cplusplus
 }

@@ -21,7 +21,7 @@ INCLUDE = os.path.join(ROOT, "include")
 BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libwq4.so")
 
-SOURCES = ["wq4_gemv.cu", "wq4_chain.cu", "wq4_synth.cu", "wq4_tc.cu"]
+SOURCES = ["wq4_gemv.cu", "wq4_chain.cu", "wq4_synth.cu", "wq4_tc.cu", "wq4_attn.cu"]
 HEADERS = ["wq4_device.cuh", "wq4_host.h", "wq4_tc.cuh", "wq4_tc_host.h"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
@@ -42,7 +42,8 @@ def cuda_lib_dir() -> str:
 
 def _inputs():
     files = [os.path.join(CSRC, s) for s in SOURCES + HEADERS]
-    files += [os.path.join(INCLUDE, "wq4.h"), os.path.join(INCLUDE, "wq4_synth.h"), os.path.abspath(__file__)]
+    files += [os.path.join(INCLUDE, h) for h in ("wq4.h", "wq4_synth.h", "wq4_attn.h")]
+    files.append(os.path.abspath(__file__))
     return files
 
 

@@ -17,6 +17,9 @@ namespace wq4 {
 // Bits of the library's device status word.
 constexpr uint32_t kErrPipeTimeout = 1u;   // an mbarrier wait gave up
 constexpr uint32_t kErrFlagTimeout = 2u;   // a wait on another CTA's data gave up
+constexpr uint32_t kErrSeqLen = 8u;        // attention: a length beyond the page table (clamped)
+constexpr uint32_t kErrPageId = 16u;       // attention: a page id outside the pool (zeros read)
+constexpr uint32_t kErrAppend = 32u;       // append: bad position or page id (row not written)
 
 // Every spin-wait gives up after this long (a legitimate wait lasts
 // microseconds); the kernel then records the error and runs to its end.

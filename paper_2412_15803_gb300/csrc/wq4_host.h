@@ -1,6 +1,7 @@
 // wq4_host.h -- host-side helpers shared by the library's translation units.
 #pragma once
 
+#include <cuda.h>
 #include <cuda_runtime.h>
 
 #include <cstddef>
@@ -19,6 +20,12 @@ const DeviceInfo* current_device_info(int* device_out);
 
 // Device address of the library's status word on the current device.
 uint32_t* status_word();
+
+// 2-D tiled tensor map (driver entry point, no libcuda link): dims
+// {inner, outer} elements, row pitch row_bytes, box {box_inner, box_outer}.
+bool encode_tensor_map_2d(CUtensorMap* m, CUtensorMapDataType dt, const void* base, uint64_t inner,
+                          uint64_t outer, uint64_t row_bytes, uint32_t box_inner, uint32_t box_outer,
+                          CUtensorMapSwizzle swz);
 
 inline bool aligned(const void* p, size_t a)
 {

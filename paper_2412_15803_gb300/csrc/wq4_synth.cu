@@ -64,6 +64,22 @@ __global__ void scales_kernel(uint16_t* __restrict__ s, int64_t start, int64_t n
     }
 }
 
+// sum4: fp16_RNE((a + b + c + d - 131070) * 2^-15), a..d the four 16-bit
+// fields of u64(key, i); integer arithmetic then a single rounding.
+__global__ void sum4_kernel(uint16_t* __restrict__ out, int64_t start, int64_t n, uint64_t key)
+{
+    for (int64_t t = static_cast<int64_t>(blockIdx.x) * blockDim.x + threadIdx.x; t < n;
+         t += static_cast<int64_t>(gridDim.x) * blockDim.x) {
+        const uint64_t v = mix64(key + static_cast<uint64_t>(start + t + 1) * kGamma);
+        const int64_t c = static_cast<int64_t>((v & 0xFFFF) + ((v >> 16) & 0xFFFF) + ((v >> 32) & 0xFFFF) + (v >> 48)) -
+                          131070;
+        const double x = static_cast<double>(c) * 0x1.0p-15;   // exact
+        unsigned short h;
+        asm("cvt.rn.f16.f64 %0, %1;" : "=h"(h) : "d"(x));
+        out[t] = h;
+    }
+}
+
 int grid_for(int64_t n)
 {
     int64_t b = (n + 255) / 256;
@@ -92,5 +108,13 @@ extern "C" int wq4_synth_scales(uint16_t* s, int64_t start, int64_t n, uint64_t 
     if (n == 0) return 0;
     scales_kernel<<<grid_for(n), 256, 0, static_cast<cudaStream_t>(stream)>>>(s, start, n, stream_key(seed, sid),
                                                                                lo, hi - lo);
+    return cudaGetLastError() == cudaSuccess ? 0 : -4;
+}
+
+extern "C" int wq4_synth_sum4(uint16_t* out, int64_t start, int64_t n, uint64_t seed, uint64_t sid, void* stream)
+{
+    if (!out || start < 0 || n < 0) return -1;
+    if (n == 0) return 0;
+    sum4_kernel<<<grid_for(n), 256, 0, static_cast<cudaStream_t>(stream)>>>(out, start, n, stream_key(seed, sid));
     return cudaGetLastError() == cudaSuccess ? 0 : -4;
 }

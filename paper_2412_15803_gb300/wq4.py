@@ -50,6 +50,11 @@ class wq4_layer_table(ctypes.Structure):
                 ("lm_head", wq4_mat), ("workspace", _P), ("workspace_bytes", _SZ)]
 
 
+class wq4_kv_cache(ctypes.Structure):
+    _fields_ = [("k", _P), ("v", _P), ("num_pages", _I), ("n_kv_heads", _I), ("page_size", _I),
+                ("head_dim", _I), ("page_table", _P), ("page_table_stride", _I)]
+
+
 class wq4_chain_trace(ctypes.Structure):
     _fields_ = [(n, _SZ) for n in ("x_in", "qkv", "o", "x_mid", "gate_up", "act", "down", "x_out")]
 
@@ -88,6 +93,12 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
                                           ctypes.POINTER(wq4_chain_trace)]
     L.wq4_synth_codes.argtypes = [_P, _I64, _I64, _U64, _U64, _I, _P]
     L.wq4_synth_scales.argtypes = [_P, _I64, _I64, _U64, _U64, ctypes.c_double, ctypes.c_double, _P]
+    L.wq4_synth_sum4.argtypes = [_P, _I64, _I64, _U64, _U64, _P]
+    L.wq4_paged_attention_workspace_bytes.argtypes = [_I, _I, _I, _I]
+    L.wq4_paged_attention_workspace_bytes.restype = _SZ
+    L.wq4_paged_attention.argtypes = [ctypes.POINTER(wq4_kv_cache), _P, _I, _P, _P, _I, _I, _I, ctypes.c_float,
+                                      _P, _SZ, _P]
+    L.wq4_kv_append.argtypes = [ctypes.POINTER(wq4_kv_cache), _P, _P, _I, _P, _I, _P]
     _lib = L
     return L
 
@@ -96,7 +107,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
 EXPORTED = ["wq4_gemv", "wq4_unpack_debug", "wq4_pack_host", "wq4_status_string",
             "wq4_device_status", "wq4_chain_workspace_bytes", "wq4_decode_chain",
             "wq4_decode_chain_host", "wq4_decode_chain_noalloc", "wq4_chain_plan_destroy", "wq4_chain_trace_offsets",
-            "wq4_synth_codes", "wq4_synth_scales"]
+            "wq4_synth_codes", "wq4_synth_scales", "wq4_synth_sum4",
+            "wq4_paged_attention_workspace_bytes", "wq4_paged_attention", "wq4_kv_append"]
 
 
 def _ptr(t) -> int | None:
@@ -197,3 +209,38 @@ def wq4_synth_scales(s, start: int, n: int, seed: int, sid: int, lo: float, hi: 
     rc = load().wq4_synth_scales(_ptr(s), start, n, seed, sid, lo, hi, _stream(stream))
     if rc != 0:
         raise Wq4Error("wq4_synth_scales", rc)
+
+
+def wq4_synth_sum4(out, start: int, n: int, seed: int, sid: int, stream=None) -> None:
+    rc = load().wq4_synth_sum4(_ptr(out), start, n, seed, sid, _stream(stream))
+    if rc != 0:
+        raise Wq4Error("wq4_synth_sum4", rc)
+
+
+def kv_cache_desc(k, v, page_table, page_size: int) -> wq4_kv_cache:
+    """wq4_kv_cache of device tensors k, v [num_pages][n_kv_heads][page_size][head_dim]
+    and page_table int32 [batch][stride]."""
+    num_pages, n_kv, ps, head_dim = k.shape
+    if ps != page_size:
+        raise ValueError("cache shape does not match page_size")
+    return wq4_kv_cache(_ptr(k), _ptr(v), num_pages, n_kv, page_size, head_dim, _ptr(page_table),
+                        page_table.shape[1])
+
+
+def wq4_paged_attention_workspace_bytes(batch: int, n_q_heads: int, n_kv_heads: int, head_dim: int) -> int:
+    return load().wq4_paged_attention_workspace_bytes(batch, n_q_heads, n_kv_heads, head_dim)
+
+
+def wq4_paged_attention(cache: wq4_kv_cache, q, q_stride: int, seq_lens, out, out_stride: int, batch: int,
+                        n_q_heads: int, scale: float, workspace, workspace_bytes: int, stream=None,
+                        check: bool = True) -> int:
+    rc = load().wq4_paged_attention(ctypes.byref(cache), _ptr(q), q_stride, _ptr(seq_lens), _ptr(out), out_stride,
+                                    batch, n_q_heads, scale, _ptr(workspace), workspace_bytes, _stream(stream))
+    return _check("wq4_paged_attention", rc) if check else rc
+
+
+def wq4_kv_append(cache: wq4_kv_cache, new_k, new_v, new_stride: int, positions, batch: int, stream=None,
+                  check: bool = True) -> int:
+    rc = load().wq4_kv_append(ctypes.byref(cache), _ptr(new_k), _ptr(new_v), new_stride, _ptr(positions), batch,
+                              _stream(stream))
+    return _check("wq4_kv_append", rc) if check else rc

@@ -16,7 +16,7 @@ ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
 
 def declared_functions():
     names = set()
-    for h in ("wq4.h", "wq4_synth.h"):
+    for h in ("wq4.h", "wq4_synth.h", "wq4_attn.h"):
         text = open(os.path.join(ROOT, "include", h)).read()
         text = re.sub(r"/\*.*?\*/", "", text, flags=re.S)
         names |= set(re.findall(r"^[A-Za-z_][\w \*]*?\b(wq4_\w+)\s*\(", text, flags=re.M))
@@ -134,3 +134,59 @@ def test_synth_rejects_bad_arguments():
     assert L.wq4_synth_codes(A16, 1, 4, 0, 0, 0, None) == -1
     assert L.wq4_synth_codes(A16, 0, 3, 0, 0, 1, None) == -1
     assert L.wq4_synth_scales(None, 0, 4, 0, 0, 0.005, 0.02, None) == -1
+
+    assert L.wq4_synth_sum4(None, 0, 4, 0, 0, None) == -1
+    assert L.wq4_synth_sum4(A16, -1, 4, 0, 0, None) == -1
+
+
+def _cache(**kw):
+    c = wq4.wq4_kv_cache(A16, 64 * A16, 64, 2, 16, 128, 128 * A16, 8)
+    for k, v in kw.items():
+        setattr(c, k, v)
+    return c
+
+
+@pytest.mark.parametrize("cache_kw,call_kw,expect", [
+    (dict(), dict(q=0), wq4.WQ4_ERR_INVALID),
+    (dict(k=0), dict(), wq4.WQ4_ERR_INVALID),
+    (dict(page_table=0), dict(), wq4.WQ4_ERR_INVALID),
+    (dict(page_size=8), dict(), wq4.WQ4_ERR_INVALID),
+    (dict(page_size=24), dict(), wq4.WQ4_ERR_INVALID),
+    (dict(num_pages=0), dict(), wq4.WQ4_ERR_INVALID),
+    (dict(), dict(batch=0), wq4.WQ4_ERR_INVALID),
+    (dict(), dict(batch=1025), wq4.WQ4_ERR_INVALID),
+    (dict(), dict(n_q_heads=5), wq4.WQ4_ERR_INVALID),
+    (dict(), dict(n_q_heads=1), wq4.WQ4_ERR_INVALID),
+    (dict(head_dim=64), dict(), wq4.WQ4_ERR_UNSUPPORTED),
+    (dict(), dict(n_q_heads=18), wq4.WQ4_ERR_UNSUPPORTED),
+    (dict(), dict(q_stride=1000), wq4.WQ4_ERR_INVALID),
+    (dict(), dict(q=256 * A16 + 8), wq4.WQ4_ERR_ALIGN),
+    (dict(), dict(q_stride=1028), wq4.WQ4_ERR_ALIGN),
+    (dict(k=A16 + 2), dict(), wq4.WQ4_ERR_ALIGN),
+    (dict(), dict(scale=float("nan")), wq4.WQ4_ERR_INVALID),
+])
+def test_paged_attention_rejects_bad_arguments(cache_kw, call_kw, expect):
+    a = dict(q=256 * A16, q_stride=1024, lens=300 * A16, out=400 * A16, out_stride=1024, batch=2, n_q_heads=8,
+             scale=0.088, ws=500 * A16, ws_bytes=1 << 30)
+    a.update(call_kw)
+    c = _cache(**cache_kw)
+    rc = wq4.load().wq4_paged_attention(ctypes.byref(c), a["q"], a["q_stride"], a["lens"], a["out"],
+                                        a["out_stride"], a["batch"], a["n_q_heads"], a["scale"], a["ws"],
+                                        a["ws_bytes"], None)
+    assert rc == expect
+
+
+def test_paged_attention_workspace_bytes_rejects_bad_geometry():
+    L = wq4.load()
+    for args in ((0, 8, 2, 128), (2, 8, 2, 64), (2, 6, 4, 128), (2, 36, 4, 128), (2000, 8, 2, 128)):
+        assert L.wq4_paged_attention_workspace_bytes(*args) == 0
+
+
+def test_kv_append_rejects_bad_arguments():
+    L = wq4.load()
+    c = _cache()
+    assert L.wq4_kv_append(ctypes.byref(c), None, A16 * 2, 256, A16 * 3, 1, None) == wq4.WQ4_ERR_INVALID
+    assert L.wq4_kv_append(ctypes.byref(c), 200 * A16, 210 * A16, 100, 220 * A16, 1, None) == wq4.WQ4_ERR_INVALID
+    assert L.wq4_kv_append(ctypes.byref(c), 200 * A16 + 8, 210 * A16, 256, 220 * A16, 1, None) == wq4.WQ4_ERR_ALIGN
+    c64 = _cache(head_dim=64)
+    assert L.wq4_kv_append(ctypes.byref(c64), 200 * A16, 210 * A16, 256, 220 * A16, 1, None) == wq4.WQ4_ERR_UNSUPPORTED

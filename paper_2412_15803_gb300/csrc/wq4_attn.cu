@@ -44,6 +44,7 @@ constexpr int kSlotBytes = 2 * kTile * kD * 2;   // keys + values of one tile: 8
 constexpr int kBoxBytes = kTile * 64 * 2;        // 16 rows x 64 dims: 2 KiB
 constexpr int kPartHdr = 16;                     // floats: M[8], L[8]
 constexpr int kCtasPerSm = 2;
+constexpr int kMaxParts = kConsumers * kD;      // parts of one segment the merge stages: grid <= 512
 
 // Shared memory map (dynamic, base 1024-aligned).
 constexpr int kOffRing = 0;
@@ -217,7 +218,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) paged_attn_kernel(const 
     __syncthreads();
 
     const int total = P.Hkv * pre[P.batch];
-    const int R = (total + gridDim.x - 1) / gridDim.x;
+    const int R = (total + static_cast<int>(gridDim.x) - 1) / static_cast<int>(gridDim.x);
     const int cta = blockIdx.x;
     const int g_begin = min(total, cta * R);
     const int g_end = min(total, g_begin + R);
@@ -320,9 +321,11 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) paged_attn_kernel(const 
             }
         }
         float m = -INFINITY, l = 0.f;
-        float o[16][4];
+        // o[j]: output dims 16j + lane/4 (0, 1) and 16j + 8 + lane/4 (2, 3) of
+        // heads 2(lane&3) (0, 2) and 2(lane&3) + 1 (1, 3)
+        float o[8][4];
 #pragma unroll
-        for (int n = 0; n < 16; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
+        for (int n = 0; n < 8; ++n) o[n][0] = o[n][1] = o[n][2] = o[n][3] = 0.f;
 
         // tiles k of the piece with (ibase + k) % W == warp
         int k0 = (warp - ibase % kConsumers + kConsumers) % kConsumers;
@@ -369,24 +372,33 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) paged_attn_kernel(const 
             const uint32_t p23 = pack_half2(exp2f(x2 - msafe), exp2f(x3 - msafe));
             const float2 f01 = unpack_half2(p01), f23 = unpack_half2(p23);
             l = l * alpha + ((f01.x + f01.y) + (f23.x + f23.y));
-            const uint32_t pa[4] = {p01, 0u, p23, 0u};
 
+            // weights x values, transposed: o^T (128 dims x 8 heads) += V^T (dims x 16
+            // tokens) * P^T (tokens x heads).  The score layout above leaves this
+            // lane's weights of head gq, tokens qc, qc+1 and qc+8, qc+9, exactly the
+            // B fragment of P^T; A = V^T comes from the value tile by a transposing
+            // ldmatrix.  Output columns = heads 2(lane&3), +1: fetch their factors.
+            const float al0 = __shfl_sync(0xffffffffu, alpha, 8 * (lane & 3));
+            const float al1 = __shfl_sync(0xffffffffu, alpha, 8 * (lane & 3) + 4);
             // masks of the value rows past the sequence end (their contents may be anything)
             const uint32_t mlo = (qc < valid ? 0x0000FFFFu : 0u) | (qc + 1 < valid ? 0xFFFF0000u : 0u);
             const uint32_t mhi = (qc + 8 < valid ? 0x0000FFFFu : 0u) | (qc + 9 < valid ? 0xFFFF0000u : 0u);
             {
-                const int r = (((lane >> 3) & 1) << 3) + (lane & 7);
-                const int cadd = lane >> 4;
+                const int mi = lane >> 3;
+                const int r = ((mi >> 1) << 3) + (lane & 7);
 #pragma unroll
                 for (int j = 0; j < 8; ++j) {
-                    uint32_t vf[4];
-                    ldsm_x4_trans(vb + (j >> 2) * kBoxBytes + sw128(r, ((2 * j) & 7) + cadd), vf);
-                    o[2 * j][0] *= alpha;
-                    o[2 * j][1] *= alpha;
-                    o[2 * j + 1][0] *= alpha;
-                    o[2 * j + 1][1] *= alpha;
-                    mma16816(o[2 * j], pa, vf[0] & mlo, vf[1] & mhi);
-                    mma16816(o[2 * j + 1], pa, vf[2] & mlo, vf[3] & mhi);
+                    uint32_t va[4];
+                    ldsm_x4_trans(vb + (j >> 2) * kBoxBytes + sw128(r, ((2 * j) & 7) + (mi & 1)), va);
+                    va[0] &= mlo;
+                    va[1] &= mlo;
+                    va[2] &= mhi;
+                    va[3] &= mhi;
+                    o[j][0] *= al0;
+                    o[j][1] *= al1;
+                    o[j][2] *= al0;
+                    o[j][3] *= al1;
+                    mma16816(o[j], va, p01, p23);
                 }
             }
             __syncwarp();
@@ -396,12 +408,21 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) paged_attn_kernel(const 
         // ---- merge the warps' states of this piece (fixed warp order)
         l += __shfl_xor_sync(0xffffffffu, l, 1);
         l += __shfl_xor_sync(0xffffffffu, l, 2);
-        if (gq < G) {
-            float* sw = scr + (warp * kMaxGroup + gq) * kD;
+        {
+            const int h0 = 2 * (lane & 3), dl = lane >> 2;
+            float* s0 = scr + (warp * kMaxGroup + h0) * kD;
 #pragma unroll
-            for (int n = 0; n < 16; ++n)
-                *reinterpret_cast<float2*>(sw + 8 * n + qc) = make_float2(o[n][0], o[n][1]);
-            if ((lane & 3) == 0) {
+            for (int j = 0; j < 8; ++j) {
+                if (h0 < G) {
+                    s0[16 * j + dl] = o[j][0];
+                    s0[16 * j + 8 + dl] = o[j][2];
+                }
+                if (h0 + 1 < G) {
+                    s0[kD + 16 * j + dl] = o[j][1];
+                    s0[kD + 16 * j + 8 + dl] = o[j][3];
+                }
+            }
+            if (gq < G && (lane & 3) == 0) {
                 mrow[warp * kMaxGroup + gq] = m;
                 lrow[warp * kMaxGroup + gq] = l;
             }
@@ -445,28 +466,70 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) paged_attn_kernel(const 
             named_barrier_sync(1, kConsumers * 32);
             if (misc[1]) {
                 __threadfence();
-                // parts p = 0..npieces-1 of this segment, in order
-                for (int e = tid; e < G * (kD / 2); e += kConsumers * 32) {
-                    const int gg = e / (kD / 2), d = 2 * (e % (kD / 2));
-                    float M = -INFINITY;
-                    for (int p = 0; p < pc.npieces; ++p) {
-                        const float* pp = P.part + static_cast<size_t>(pc.first + p + pc.seg) * (kPartHdr + G * kD);
-                        M = fmaxf(M, __ldcg(pp + gg));
+                // Merge parts p = 0..np-1 of this segment.  (1) per head row: 16
+                // threads run the online max/normaliser merge over the parts'
+                // (M_p, L_p), then a fixed shuffle tree joins them; the factors
+                // 2^(M_p - M*) land in shared memory.  (2) every output element
+                // sums f_p * O_p in part order, loads independent of each other.
+                const int np = pc.npieces;
+                const size_t pstride = kPartHdr + static_cast<size_t>(G) * kD;
+                const float* pbase = P.part + static_cast<size_t>(pc.first + pc.seg) * pstride;
+                float* fsm = scr;     // [np][8] (np <= kMaxParts)
+                float* mls = mrow;    // M*[8], L*[8]
+                {
+                    const int gg = tid >> 4, sub = tid & 15;
+                    float m = -INFINITY, l = 0.f;
+                    if (gg < G) {
+#pragma unroll 4
+                        for (int p = sub; p < np; p += 16) {
+                            const float Mp = __ldcg(pbase + p * pstride + gg);
+                            const float Lp = __ldcg(pbase + p * pstride + kMaxGroup + gg);
+                            fsm[p * kMaxGroup + gg] = Mp;
+                            const float mn = fmaxf(m, Mp);
+                            const float ms = mn == -INFINITY ? 0.f : mn;
+                            l = l * exp2f(m - ms) + Lp * exp2f(Mp - ms);
+                            m = mn;
+                        }
                     }
-                    const float Ms = M == -INFINITY ? 0.f : M;
-                    float L = 0.f, O0 = 0.f, O1 = 0.f;
-                    for (int p = 0; p < pc.npieces; ++p) {
-                        const float* pp = P.part + static_cast<size_t>(pc.first + p + pc.seg) * (kPartHdr + G * kD);
-                        const float f = exp2f(__ldcg(pp + gg) - Ms);
-                        L += __ldcg(pp + kMaxGroup + gg) * f;
-                        const float2 ov = __ldcg(reinterpret_cast<const float2*>(pp + kPartHdr + gg * kD + d));
-                        O0 += ov.x * f;
-                        O1 += ov.y * f;
+#pragma unroll
+                    for (int o = 1; o < 16; o <<= 1) {
+                        const float m2 = __shfl_xor_sync(0xffffffffu, m, o);
+                        const float l2 = __shfl_xor_sync(0xffffffffu, l, o);
+                        const float mn = fmaxf(m, m2);
+                        const float ms = mn == -INFINITY ? 0.f : mn;
+                        l = l * exp2f(m - ms) + l2 * exp2f(m2 - ms);
+                        m = mn;
                     }
+                    if (gg < G && sub == 0) {
+                        mls[gg] = m;
+                        mls[kMaxGroup + gg] = l;
+                    }
+                    named_barrier_sync(1, kConsumers * 32);
+                    if (gg < G) {
+                        const float ms = mls[gg] == -INFINITY ? 0.f : mls[gg];
+                        for (int p = sub; p < np; p += 16) fsm[p * kMaxGroup + gg] = exp2f(fsm[p * kMaxGroup + gg] - ms);
+                    }
+                    named_barrier_sync(1, kConsumers * 32);
+                }
+                for (int e = tid; e < G * (kD / 4); e += kConsumers * 32) {
+                    const int gg = e / (kD / 4), d = 4 * (e % (kD / 4));
+                    const float* po = pbase + kPartHdr + gg * kD + d;
+                    float a0 = 0.f, a1 = 0.f, a2 = 0.f, a3 = 0.f;
+#pragma unroll 8
+                    for (int p = 0; p < np; ++p) {
+                        const float f = fsm[p * kMaxGroup + gg];
+                        const float4 ov = __ldcg(reinterpret_cast<const float4*>(po + p * pstride));
+                        a0 = fmaf(ov.x, f, a0);
+                        a1 = fmaf(ov.y, f, a1);
+                        a2 = fmaf(ov.z, f, a2);
+                        a3 = fmaf(ov.w, f, a3);
+                    }
+                    const float L = mls[kMaxGroup + gg];
                     const float inv = L > 0.f ? 1.f / L : 0.f;
                     uint16_t* ob =
-                        P.out + static_cast<size_t>(pc.b) * P.out_stride + static_cast<size_t>(pc.h * G + gg) * kD;
-                    *reinterpret_cast<uint32_t*>(ob + d) = pack_half2(O0 * inv, O1 * inv);
+                        P.out + static_cast<size_t>(pc.b) * P.out_stride + static_cast<size_t>(pc.h * G + gg) * kD + d;
+                    reinterpret_cast<uint32_t*>(ob)[0] = pack_half2(a0 * inv, a1 * inv);
+                    reinterpret_cast<uint32_t*>(ob)[1] = pack_half2(a2 * inv, a3 * inv);
                 }
                 if (tid == 0) P.cnt[pc.seg] = 0u;
             }
@@ -519,7 +582,8 @@ int attn_grid(int dev, int sms)
         return 0;
     if (per_sm < 1) return 0;
     if (per_sm > kCtasPerSm) per_sm = kCtasPerSm;
-    const int g = sms * per_sm;
+    int g = sms * per_sm;
+    if (g > kMaxParts) g = kMaxParts;
     if (dev >= 0 && dev < 64) cached[dev] = g;
     return g;
 }

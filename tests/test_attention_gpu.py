@@ -136,7 +136,7 @@ def test_deterministic_and_counters_left_zero():
     q, k, v, table, lens = make_case(8, [900, 17, 3000], 32, 8, 16)
     scale = 1.0 / math.sqrt(128)
     o1, _, ws = run_attention(q, k, v, table, lens, 32, scale)
-    assert int(ws[: 4 * 3 * 8].count_nonzero()) == 0
+    assert int(ws[: 4 * 3 * 8].count_nonzero()) == 0   # arrival counters
     o2, _, _ = run_attention(q, k, v, table, lens, 32, scale, ws=ws)
     assert np.array_equal(o1, o2)
 

@@ -41,11 +41,11 @@ namespace wq4 {
 namespace {
 
 constexpr int kTcStages = 4;          // ring slots
-constexpr int kTcThreads = 448;       // warps 0-7 dequant, 8 producer, 9 MMA, 10-13 epilogue
-constexpr int kTcProducer = 8, kTcIssuer = 9;
+constexpr int kTcThreads = 480;       // warps 0-7 dequant, 8 producer, 9 and 14 MMA, 10-13 epilogue
+constexpr int kTcProducer = 8, kTcIssuer = 9, kTcIssuer2 = 14;
 constexpr int kTcCodes = 128 * 128;   // one chunk of codes: 128 rows x 256 codes
 constexpr int kTcScales = 128 * 16;   // 128 rows x 8 fp16 scales
-constexpr int kTcTmemCols = 512;      // A: 2 x 128 columns, D: 2 x 32 columns at 256
+constexpr int kTcTmemCols = 512;      // A: 2 x 128 columns; D at 256: 2 buffers x 2 issuers x 32 columns
 
 template <int NB>
 struct TcSmem {
@@ -269,10 +269,10 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         for (int i = 0; i < 2; ++i) {
             mbar_init(&afull[i], 8);
             mbar_init(&aempty[i], 1);
-            mbar_init(&dfull[i], 1);
+            mbar_init(&dfull[i], 2);   // one commit per issuer
             mbar_init(&dempty[i], 4);
         }
-        mbar_init(drain, 1);
+        mbar_init(drain, 2);
         mbar_fence_init();
     }
     if (warp == kTcIssuer) tc::tmem_alloc(tbase_sh, kTcTmemCols);
@@ -353,8 +353,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 tc_wait_ok(&fullx[i % kTcStages], (i / kTcStages) & 1, err);
             }
         }
-    } else if (warp == kTcIssuer) {
-        // ---------------------------------------------------- MMA issuer
+    } else if (warp == kTcIssuer || warp == kTcIssuer2) {
+        // ---------------------------------------------------- MMA issuers
+        // Two issuing warps: chunk ait goes to issuer ait & 1, which owns A
+        // buffer ait & 1 and its own accumulator.  One thread issues a
+        // tcgen05.mma only every ~45 cycles at these shapes, so a second
+        // issuer doubles the rate; the epilogue adds the two accumulators.
+        const int iss = warp == kTcIssuer ? 0 : 1;
         if (lane == 0) {
             constexpr uint32_t idesc = tc::idesc_f16_f32(128, NB);
             int it = 0, ait = 0, dit = 0;
@@ -365,9 +370,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 (void)tile;
                 const int dbuf = dit & 1;
                 if (dit >= 2 && !tc_wait_ok(&dempty[dbuf], ((dit >> 1) - 1) & 1, err)) break;
-                const uint32_t dt = tbase + 256 + 32 * dbuf;
+                const uint32_t dt = tbase + 256 + 64 * dbuf + 32 * iss;
+                bool first = true;
                 for (int c = c0; c < c1; ++c, ++it, ++ait) {
-                    const int slot = it % kTcStages, abuf = ait & 1;
+                    if ((ait & 1) != iss) continue;          // the other issuer's chunk
+                    const int slot = it % kTcStages, abuf = iss;
                     if (!tc_wait_ok(&fullx[slot], (it / kTcStages) & 1, err) ||
                         !tc_wait_ok(&afull[abuf], (ait >> 1) & 1, err)) {
                         ok = false;
@@ -378,13 +385,14 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 #pragma unroll
                     for (int s = 0; s < 16; ++s) {
                         const uint64_t bd = tc::sw128_kmajor_desc(xs + (s >> 2) * NB * 128 + 32 * (s & 3));
-                        tc::mma_f16_ts(dt, tbase + 128 * abuf + 8 * s, bd, idesc, (c > c0 || s > 0) ? 1u : 0u);
+                        tc::mma_f16_ts(dt, tbase + 128 * abuf + 8 * s, bd, idesc, (!first || s > 0) ? 1u : 0u);
                     }
+                    first = false;
                     tc::commit(&aempty[abuf]);
                     tc::commit(&empty[slot]);
                 }
                 if (!ok) break;
-                tc::commit(&dfull[dbuf]);
+                tc::commit(&dfull[dbuf]);   // arrives at once if this issuer had no chunk here
                 ++dit;
             }
             // all MMAs issued have completed before tensor memory is released
@@ -445,19 +453,28 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const int quad = warp & 3;
         const int row = 32 * quad + lane;
         const uint32_t lane_base = tbase + (static_cast<uint32_t>(32 * quad) << 16);
-        int dit = 0;
+        int dit = 0, ait = 0;
         bool waited = false;
         for (int u = blockIdx.x; u < units; u += gridDim.x) {
             const int tile = u / P, pt = u - tile * P;
             const int dbuf = dit & 1;
+            // which issuers accumulated this unit: both unless it has one chunk
+            const int nchk = (pt + 1) * nch / P - pt * nch / P;
+            const bool has0 = nchk >= 2 || (ait & 1) == 0, has1 = nchk >= 2 || (ait & 1) == 1;
+            ait += nchk;
             if (!tc_wait_ok(&dfull[dbuf], (dit >> 1) & 1, err)) break;
             tc::fence_after_sync();
-            uint32_t d[32];
-            tc::ld16(lane_base + 256 + 32 * dbuf, d);
-            if (NB > 16) tc::ld16(lane_base + 256 + 32 * dbuf + 16, d + 16);
+            uint32_t d[32], d1[32];
+            tc::ld16(lane_base + 256 + 64 * dbuf, d);
+            if (NB > 16) tc::ld16(lane_base + 256 + 64 * dbuf + 16, d + 16);
+            tc::ld16(lane_base + 256 + 64 * dbuf + 32, d1);
+            if (NB > 16) tc::ld16(lane_base + 256 + 64 * dbuf + 48, d1 + 16);
             tc::ld_wait();
             tc::fence_before_sync();
             __syncwarp();
+#pragma unroll
+            for (int b = 0; b < NB; ++b)
+                d[b] = __float_as_uint((has0 ? __uint_as_float(d[b]) : 0.f) + (has1 ? __uint_as_float(d1[b]) : 0.f));
             if (lane == 0) mbar_arrive(&dempty[dbuf]);
             ++dit;
             if (!waited) {

@@ -45,6 +45,7 @@ constexpr int kTcThreads = 480;       // warps 0-7 dequant, 8 producer, 9 and 14
 constexpr int kTcProducer = 8, kTcIssuer = 9, kTcIssuer2 = 14;
 constexpr int kTcCodes = 128 * 128;   // one chunk of codes: 128 rows x 256 codes
 constexpr int kTcScales = 128 * 16;   // 128 rows x 8 fp16 scales
+constexpr int kTcMaxParts = 8;        // K parts of a split stage (bounds the epilogue's loads in flight)
 constexpr int kTcTmemCols = 512;      // A: 2 x 128 columns; D at 256: 2 buffers x 2 issuers x 32 columns
 
 template <int NB>
@@ -93,38 +94,39 @@ __device__ __forceinline__ uint16_t add_h(float a, float b) { return float_to_ha
 __device__ __forceinline__ int perm_pos(int p) { return p < 4 ? 2 * p : 2 * (p - 4) + 1; }
 
 // r = 1/sqrt(mean + eps) from per-tile sums of squares, summed in tile order
-// (loads issued eight at a time).
+// (up to 32 loads issued at once, then the rest).
 __device__ __forceinline__ float rms_of(const float* sq, int ntiles, int B, int b, int n, float eps)
 {
+    float v[32];
+#pragma unroll
+    for (int k = 0; k < 32; ++k) v[k] = k < ntiles ? __ldcg(sq + k * B + b) : 0.f;
     float t = 0.f;
-    int i = 0;
-    for (; i + 8 <= ntiles; i += 8) {
-        float v[8];
 #pragma unroll
-        for (int k = 0; k < 8; ++k) v[k] = __ldcg(sq + (i + k) * B + b);
-#pragma unroll
-        for (int k = 0; k < 8; ++k) t += v[k];
-    }
-    for (; i < ntiles; ++i) t += __ldcg(sq + i * B + b);
+    for (int k = 0; k < 32; ++k)
+        if (k < ntiles) t += v[k];
+    for (int i = 32; i < ntiles; ++i) t += __ldcg(sq + i * B + b);
     return rsqrtf(t * (1.f / static_cast<float>(n)) + eps);
 }
 
-// Epilogue of one tile by the 128 dequant threads (row = 32 warp + lane): v[b]
-// the row's sums over K for batch row b.  ep: shared scratch.
+// Epilogue of one tile by the 128 epilogue threads (row = 32 quad + lane):
+// v[b] the row's sums over K for batch row b, resv the row's residual
+// inputs (O, down, LM head) as fp16 pairs, already loaded when NB is 16.  ep: shared scratch whose first
+// 64 floats hold the RMS factors r_in[b] and r_u[b] of the stage.
 template <int NB>
-__device__ void tile_epilogue(const TcArgs& a, int tile, int row, const float v[NB], float* ep)
+__device__ void tile_epilogue(const TcArgs& a, int tile, int row, const float v[NB], const uint32_t resv[NB / 2],
+                              float* ep)
 {
-    float* r_in = ep;          // [32]
-    float* r_u = ep + 32;      // [32]
+    const int n_row = 128 * tile + row;
+    auto res_b = [&](int b) {
+        return NB == 16 ? half_bits_to_float(static_cast<uint16_t>(resv[b >> 1] >> (16 * (b & 1))))
+                        : half_bits_to_float(a.res[static_cast<size_t>(b) * a.H + n_row]);
+    };
+    const float* r_in = ep;    // [32]
+    const float* r_u = ep + 32;
     float* red = ep + 64;      // [4][32]
     float* sqs = ep + 192;     // [128][33] squares of the next input (padded rows), ends before the ring
     uint16_t* upart = reinterpret_cast<uint16_t*>(ep + 192);   // [64][32] up values of gate_up (aliases sqs)
-    const int warp = row >> 5, lane = row & 31, B = a.B, H = a.H, F = a.F;
-    if (warp == 0 && lane < B) {
-        r_in[lane] = a.sq_in ? rms_of(a.sq_in, H / 128, B, lane, H, a.eps) : 1.f;
-        if (a.sq_u) r_u[lane] = rms_of(a.sq_u, H / 128, B, lane, H, a.eps);
-    }
-    named_barrier_sync(3, 128);
+    const int B = a.B, H = a.H, F = a.F;
     float nxt[NB];              // value of the next stage's input at this row (if any)
     bool has_next = false;
     int nidx = 0;               // its index in the next input
@@ -175,7 +177,7 @@ __device__ void tile_epilogue(const TcArgs& a, int tile, int row, const float v[
                 for (int b = 0; b < NB; ++b)
                     if (b < B) {
                         const uint16_t o = float_to_half_bits(r_in[b] * v[b]);
-                        const uint16_t vn = float_to_half_bits(r_u[b] * half_bits_to_float(a.res[static_cast<size_t>(b) * H + n]));
+                        const uint16_t vn = float_to_half_bits(r_u[b] * res_b(b));
                         const uint16_t x1 = add_h(half_bits_to_float(vn), half_bits_to_float(o));
                         a.y[static_cast<size_t>(b) * H + n] = o;
                         a.y2[static_cast<size_t>(b) * H + n] = x1;
@@ -190,7 +192,7 @@ __device__ void tile_epilogue(const TcArgs& a, int tile, int row, const float v[
                 for (int b = 0; b < NB; ++b)
                     if (b < B) {
                         const uint16_t d = float_to_half_bits(v[b]);
-                        const uint16_t x2 = add_h(half_bits_to_float(a.res[static_cast<size_t>(b) * H + n]), half_bits_to_float(d));
+                        const uint16_t x2 = add_h(res_b(b), half_bits_to_float(d));
                         a.y[static_cast<size_t>(b) * H + n] = d;
                         a.y2[static_cast<size_t>(b) * H + n] = x2;
                         nxt[b] = half_bits_to_float(x2);
@@ -205,7 +207,7 @@ __device__ void tile_epilogue(const TcArgs& a, int tile, int row, const float v[
                         a.y[static_cast<size_t>(b) * a.N + n] = float_to_half_bits(r_in[b] * v[b]);
                         if (n < H)
                             a.y3[static_cast<size_t>(b) * H + n] =
-                                float_to_half_bits(r_in[b] * half_bits_to_float(a.res[static_cast<size_t>(b) * H + n]));
+                                float_to_half_bits(r_in[b] * res_b(b));
                     }
                 break;
         }
@@ -454,46 +456,62 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         const int row = 32 * quad + lane;
         const uint32_t lane_base = tbase + (static_cast<uint32_t>(32 * quad) << 16);
         int dit = 0, ait = 0;
-        bool waited = false;
+        // the previous stage's outputs are complete and visible from here on;
+        // the stage's RMS factors are computed while the MMAs run
+        grid_dep_wait();
+        if (quad == 0 && lane < a.B)
+            ep[lane] = a.sq_in ? rms_of(a.sq_in, a.H / 128, a.B, lane, a.H, a.eps) : 1.f;
+        if (quad == 1 && lane < a.B && a.sq_u) ep[32 + lane] = rms_of(a.sq_u, a.H / 128, a.B, lane, a.H, a.eps);
+        named_barrier_sync(3, 128);
         for (int u = blockIdx.x; u < units; u += gridDim.x) {
             const int tile = u / P, pt = u - tile * P;
             const int dbuf = dit & 1;
+            // this row's residual input, loaded before the accumulator is ready
+            uint32_t resv[NB / 2];   // fp16 pairs: batch rows 2i (low half), 2i + 1
+            {
+                const int n = 128 * tile + row;
+                // (batch > 16: loaded in the epilogue instead, registers are short)
+                const bool need = NB == 16 && a.res && a.type != kTcGU && n < a.N && (a.type != kTcLM || n < a.H);
+#pragma unroll
+                for (int i = 0; i < NB / 2; ++i) {
+                    const uint32_t lo = (need && 2 * i < a.B) ? __ldcg(a.res + static_cast<size_t>(2 * i) * a.H + n) : 0u;
+                    const uint32_t hi = (need && 2 * i + 1 < a.B) ? __ldcg(a.res + static_cast<size_t>(2 * i + 1) * a.H + n) : 0u;
+                    resv[i] = lo | (hi << 16);
+                }
+            }
             // which issuers accumulated this unit: both unless it has one chunk
             const int nchk = (pt + 1) * nch / P - pt * nch / P;
             const bool has0 = nchk >= 2 || (ait & 1) == 0, has1 = nchk >= 2 || (ait & 1) == 1;
             ait += nchk;
             if (!tc_wait_ok(&dfull[dbuf], (dit >> 1) & 1, err)) break;
             tc::fence_after_sync();
-            uint32_t d[32], d1[32];
-            tc::ld16(lane_base + 256 + 64 * dbuf, d);
-            if (NB > 16) tc::ld16(lane_base + 256 + 64 * dbuf + 16, d + 16);
-            tc::ld16(lane_base + 256 + 64 * dbuf + 32, d1);
-            if (NB > 16) tc::ld16(lane_base + 256 + 64 * dbuf + 48, d1 + 16);
-            tc::ld_wait();
-            tc::fence_before_sync();
-            __syncwarp();
-#pragma unroll
-            for (int b = 0; b < NB; ++b)
-                d[b] = __float_as_uint((has0 ? __uint_as_float(d[b]) : 0.f) + (has1 ? __uint_as_float(d1[b]) : 0.f));
-            if (lane == 0) mbar_arrive(&dempty[dbuf]);
-            ++dit;
-            if (!waited) {
-                grid_dep_wait();   // the previous stage's outputs are complete and visible
-                waited = true;
-            }
+            // the two issuers' accumulators, 16 columns at a time, added in issuer order
             float v[NB];
 #pragma unroll
-            for (int b = 0; b < NB; ++b) v[b] = __uint_as_float(d[b]);
+            for (int h = 0; h < NB / 16; ++h) {
+                uint32_t d[16], d1[16];
+                tc::ld16(lane_base + 256 + 64 * dbuf + 16 * h, d);
+                tc::ld16(lane_base + 256 + 64 * dbuf + 32 + 16 * h, d1);
+                tc::ld_wait();
+#pragma unroll
+                for (int b = 0; b < 16; ++b)
+                    v[16 * h + b] = (has0 ? __uint_as_float(d[b]) : 0.f) + (has1 ? __uint_as_float(d1[b]) : 0.f);
+            }
+            tc::fence_before_sync();
+            __syncwarp();
+            if (lane == 0) mbar_arrive(&dempty[dbuf]);
+            ++dit;
             if (P > 1) {
                 // K is split over units: publish this part; the last part of
                 // the tile sums all parts in order and runs the epilogue
                 const int nrow = a.type == kTcGU ? tile_rows(tile, row >> 6) + (row & 63) : 128 * tile + row;
                 const bool valid = nrow < a.N;
+                // parts are rows of NB floats: [part][row][NB]
                 if (valid) {
-                    float* pb = a.part + static_cast<size_t>(pt) * a.B * a.N + nrow;
+                    float4* pb = reinterpret_cast<float4*>(a.part + (static_cast<size_t>(pt) * a.N + nrow) * NB);
 #pragma unroll
-                    for (int b = 0; b < NB; ++b)
-                        if (b < a.B) pb[static_cast<size_t>(b) * a.N] = v[b];
+                    for (int c = 0; c < NB / 4; ++c)
+                        if (4 * c < a.B) pb[c] = make_float4(v[4 * c], v[4 * c + 1], v[4 * c + 2], v[4 * c + 3]);
                 }
                 __threadfence();
                 named_barrier_sync(3, 128);
@@ -506,20 +524,34 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 if (*last_sh == 0u) continue;
                 __threadfence();
                 if (valid) {
-                    // every part, this unit's included, from L2 in part order
+                    // every part, this unit's included, from L2, summed in part
+                    // order; all parts of four batch rows are loaded at once
 #pragma unroll
-                    for (int b = 0; b < NB; ++b) v[b] = 0.f;
-                    for (int q = 0; q < P; ++q) {
-                        const float* src = a.part + static_cast<size_t>(q) * a.B * a.N + nrow;
-                        float t[NB];
+                    for (int c = 0; c < NB / 4; ++c) {
+                        if (4 * c < a.B) {
+                            float4 t[kTcMaxParts];
 #pragma unroll
-                        for (int b = 0; b < NB; ++b) t[b] = (b < a.B) ? __ldcg(src + static_cast<size_t>(b) * a.N) : 0.f;
+                            for (int q = 0; q < kTcMaxParts; ++q)
+                                if (q < P)
+                                    t[q] = __ldcg(reinterpret_cast<const float4*>(a.part + (static_cast<size_t>(q) * a.N + nrow) * NB) + c);
+                            float s0 = 0.f, s1 = 0.f, s2 = 0.f, s3 = 0.f;
 #pragma unroll
-                        for (int b = 0; b < NB; ++b) v[b] += t[b];
+                            for (int q = 0; q < kTcMaxParts; ++q)
+                                if (q < P) {
+                                    s0 += t[q].x;
+                                    s1 += t[q].y;
+                                    s2 += t[q].z;
+                                    s3 += t[q].w;
+                                }
+                            v[4 * c] = s0;
+                            v[4 * c + 1] = s1;
+                            v[4 * c + 2] = s2;
+                            v[4 * c + 3] = s3;
+                        }
                     }
                 }
             }
-            tile_epilogue<NB>(a, tile, row, v, ep);
+            tile_epilogue<NB>(a, tile, row, v, resv, ep);
             named_barrier_sync(3, 128);   // scratch reuse across units
         }
     }
@@ -586,6 +618,7 @@ int stage_parts(int tiles, int nch, int sms)
     int P = sms / tiles;
     if (P < 1) P = 1;
     if (P > nch) P = nch;
+    if (P > kTcMaxParts) P = kTcMaxParts;
     return P;
 }
 
@@ -639,7 +672,7 @@ size_t tc_part_floats(int L, int H, int F, int Nqkv, int V, int B, int sms)
     m = std::max(m, pn(2 * F, H, F / 64));
     m = std::max(m, pn(H, F, H / 128));
     m = std::max(m, pn(V, H, (V + 127) / 128));
-    return m * B;
+    return m * (B <= 16 ? 16 : 32);   // rows of NB floats (batch padded)
 }
 
 int tc_plan_create(const wq4_layer_table* t, int H, int F, int Nqkv, int V, int B, const TcBuffers& buf, int sms,

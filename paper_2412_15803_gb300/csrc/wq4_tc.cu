@@ -46,7 +46,9 @@ constexpr int kTcProducer = 8, kTcIssuer = 9, kTcIssuer2 = 14;
 constexpr int kTcCodes = 128 * 128;   // one chunk of codes: 128 rows x 256 codes
 constexpr int kTcScales = 128 * 16;   // 128 rows x 8 fp16 scales
 constexpr int kTcMaxParts = 8;        // K parts of a split stage (bounds the epilogue's loads in flight)
-constexpr int kTcTmemCols = 512;      // A: 2 x 128 columns; D at 256: 2 buffers x 2 issuers x 32 columns
+constexpr int kTcABufs = 3;           // dequantized A buffers (128 columns each)
+constexpr int kTcDCol = 128 * kTcABufs;  // accumulators: 2 buffers x 2 issuers x 32 columns
+constexpr int kTcTmemCols = 512;
 
 template <int NB>
 struct TcSmem {
@@ -249,11 +251,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
     uint64_t* fullx = fullw + kTcStages;                     // input columns landed
     uint64_t* empty = fullx + kTcStages;
     uint64_t* afull = empty + kTcStages;
-    uint64_t* aempty = afull + 2;
-    uint64_t* dfull = aempty + 2;
+    uint64_t* aempty = afull + kTcABufs;
+    uint64_t* dfull = aempty + kTcABufs;
     uint64_t* dempty = dfull + 2;
-    uint64_t* drain = dempty + 2;                            // ends at byte 168
-    uint32_t* tbase_sh = reinterpret_cast<uint32_t*>(smem + 192);
+    uint64_t* drain = dempty + 2;
+    static_assert((3 * kTcStages + 2 * kTcABufs + 5) * 8 <= 240, "barriers overlap the tensor-memory base word");
+    static_assert(kTcDCol + 128 <= kTcTmemCols, "tensor memory overflow");
+    uint32_t* tbase_sh = reinterpret_cast<uint32_t*>(smem + 240);
     uint32_t* last_sh = tbase_sh + 1;
     float* ep = reinterpret_cast<float*>(smem + 256);        // epilogue scratch: 768 B + 128 x 33 floats
     uint8_t* ring = smem + L::kRing;
@@ -268,9 +272,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             mbar_init(&fullx[i], 1);
             mbar_init(&empty[i], 9);   // 8 dequant warps + the MMA commit
         }
-        for (int i = 0; i < 2; ++i) {
+        for (int i = 0; i < kTcABufs; ++i) {
             mbar_init(&afull[i], 8);
             mbar_init(&aempty[i], 1);
+        }
+        for (int i = 0; i < 2; ++i) {
             mbar_init(&dfull[i], 2);   // one commit per issuer
             mbar_init(&dempty[i], 4);
         }
@@ -357,10 +363,11 @@ __global__ void __launch_bounds__(kTcThreads, 1)
         }
     } else if (warp == kTcIssuer || warp == kTcIssuer2) {
         // ---------------------------------------------------- MMA issuers
-        // Two issuing warps: chunk ait goes to issuer ait & 1, which owns A
-        // buffer ait & 1 and its own accumulator.  One thread issues a
+        // Two issuing warps: chunk ait goes to issuer ait & 1 (own
+        // accumulator) from A buffer ait % 3.  One thread issues a
         // tcgen05.mma only every ~45 cycles at these shapes, so a second
         // issuer doubles the rate; the epilogue adds the two accumulators.
+        // The third A buffer lets the dequant warps run a chunk ahead.
         const int iss = warp == kTcIssuer ? 0 : 1;
         if (lane == 0) {
             constexpr uint32_t idesc = tc::idesc_f16_f32(128, NB);
@@ -372,13 +379,13 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                 (void)tile;
                 const int dbuf = dit & 1;
                 if (dit >= 2 && !tc_wait_ok(&dempty[dbuf], ((dit >> 1) - 1) & 1, err)) break;
-                const uint32_t dt = tbase + 256 + 64 * dbuf + 32 * iss;
+                const uint32_t dt = tbase + kTcDCol + 64 * dbuf + 32 * iss;
                 bool first = true;
                 for (int c = c0; c < c1; ++c, ++it, ++ait) {
                     if ((ait & 1) != iss) continue;          // the other issuer's chunk
-                    const int slot = it % kTcStages, abuf = iss;
+                    const int slot = it % kTcStages, abuf = ait % kTcABufs;
                     if (!tc_wait_ok(&fullx[slot], (it / kTcStages) & 1, err) ||
-                        !tc_wait_ok(&afull[abuf], (ait >> 1) & 1, err)) {
+                        !tc_wait_ok(&afull[abuf], (ait / kTcABufs) & 1, err)) {
                         ok = false;
                         break;
                     }
@@ -414,9 +421,9 @@ __global__ void __launch_bounds__(kTcThreads, 1)
             const int tile = u / P, pt = u - tile * P;
             const int c0 = pt * nch / P, c1 = (pt + 1) * nch / P;
             for (int c = c0; c < c1; ++c, ++it, ++ait) {
-                const int slot = it % kTcStages, abuf = ait & 1;
+                const int slot = it % kTcStages, abuf = ait % kTcABufs;
                 if (!tc_wait_ok(&fullw[slot], (it / kTcStages) & 1, err) ||
-                    (ait >= 2 && !tc_wait_ok(&aempty[abuf], ((ait >> 1) - 1) & 1, err))) {
+                    (ait >= kTcABufs && !tc_wait_ok(&aempty[abuf], ((ait / kTcABufs) - 1) & 1, err))) {
                     ok = false;
                     break;
                 }
@@ -490,8 +497,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
 #pragma unroll
             for (int h = 0; h < NB / 16; ++h) {
                 uint32_t d[16], d1[16];
-                tc::ld16(lane_base + 256 + 64 * dbuf + 16 * h, d);
-                tc::ld16(lane_base + 256 + 64 * dbuf + 32 + 16 * h, d1);
+                tc::ld16(lane_base + kTcDCol + 64 * dbuf + 16 * h, d);
+                tc::ld16(lane_base + kTcDCol + 64 * dbuf + 32 + 16 * h, d1);
                 tc::ld_wait();
 #pragma unroll
                 for (int b = 0; b < 16; ++b)

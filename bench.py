@@ -75,9 +75,17 @@ def measured_peak():
         return FALLBACK_HBM_GBS, "fallback"
 
 
-def chain_source_sha() -> str:
+KERNEL_SOURCES = {
+    "chain_kernel": ("wq4_chain.cu", "wq4_device.cuh"),
+    "tc_stage_kernel": ("wq4_tc.cu", "wq4_tc.cuh", "wq4_device.cuh"),
+}
+
+
+def chain_source_sha(kernel: str) -> str:
+    """Hash of the sources of one kernel (the committed ncu summary of that
+    kernel carries the same hash)."""
     h = hashlib.sha256()
-    for f in ("wq4_chain.cu", "wq4_device.cuh", "wq4_tc.cu", "wq4_tc.cuh"):
+    for f in KERNEL_SOURCES[kernel]:
         h.update(open(os.path.join(ROOT, "paper_2412_15803_gb300", "csrc", f), "rb").read())
     return h.hexdigest()[:16]
 
@@ -92,7 +100,7 @@ def profiled_traffic(workload: str, batch: int):
     text = open(path).read()
     m = re.search(r"traffic_bytes_per_launch:\s*(\d+)", text)
     s = re.search(r"source_sha:\s*([0-9a-f]+)", text)
-    if not m or not s or s.group(1) != chain_source_sha():
+    if not m or not s or s.group(1) != chain_source_sha(name):
         return None
     return int(m.group(1))
 
@@ -471,8 +479,10 @@ def run_attn(args, rank, world, local):
         nlayers = int(np.ceil(4 * L2_BYTES / first.kv_bytes()))
     layers = [first] + [PagedAttentionLayer(w.shape, lens, page_size=w.page_size, seed=0, layer=l)
                         for l in range(1, nlayers)]
-    # one step = one launch per layer cache, captured once in a CUDA graph (as a
-    # decode step would be), so host-side call overhead stays out of the timing
+    # one step = launches over the layer caches in turn (at least 8), captured
+    # once in a CUDA graph as a decode step would be, so host-side call and
+    # graph-launch overheads stay out of the per-launch time
+    per_graph = max(nlayers, 8)
     stream = torch.cuda.Stream()
     with torch.cuda.stream(stream):
         for L in layers:
@@ -480,8 +490,8 @@ def run_attn(args, rank, world, local):
         stream.synchronize()
         graph = torch.cuda.CUDAGraph()
         with torch.cuda.graph(graph, stream=stream):
-            for L in layers:
-                L.run(stream)
+            for j in range(per_graph):
+                layers[j % nlayers].run(stream)
         for _ in range(max(args.warmup, 3)):
             graph.replay()
     torch.cuda.synchronize()
@@ -505,7 +515,7 @@ def run_attn(args, rank, world, local):
         dist.barrier()
     clocks = sampler.stop()
     total_ms = starts[0].elapsed_time(ends[-1])
-    launch_ms = [s.elapsed_time(e) / nlayers for s, e in zip(starts, ends)]
+    launch_ms = [s.elapsed_time(e) / per_graph for s, e in zip(starts, ends)]
     if wq4.wq4_device_status(stream) != 0:
         raise RuntimeError("attention flagged an error during the timed region")
 
@@ -514,17 +524,18 @@ def run_attn(args, rank, world, local):
     q_host = L0.q.cpu().pin_memory()
     o_host = torch.empty_like(L0.out, device="cpu").pin_memory()
     e2e_steps = max(10, min(args.steps, 500))
-    t0 = time.perf_counter()
-    for i in range(e2e_steps):
-        Li = layers[i % nlayers]
-        Li.q.copy_(q_host, non_blocking=True)
-        Li.run(stream)
-        o_host.copy_(Li.out, non_blocking=True)
-        torch.cuda.current_stream().synchronize()
-    e2e_s = time.perf_counter() - t0
+    with torch.cuda.stream(stream):
+        t0 = time.perf_counter()
+        for i in range(e2e_steps):
+            Li = layers[i % nlayers]
+            Li.q.copy_(q_host, non_blocking=True)
+            Li.run(stream)
+            o_host.copy_(Li.out, non_blocking=True)
+            stream.synchronize()
+        e2e_s = time.perf_counter() - t0
     # a step attends every layer cache once: batch sequences per layer launch
-    seq_per_s, e2e_val, total_ms_max = aggregate_replicas(total_ms / nlayers, e2e_s / e2e_steps, w.batch, args.steps,
-                                                          "cuda")
+    seq_per_s, e2e_val, total_ms_max = aggregate_replicas(total_ms / per_graph, e2e_s / e2e_steps, w.batch,
+                                                          args.steps, "cuda")
     if rank == 0:
         avg_launch_ms = statistics.mean(launch_ms)
         peak, peak_src = measured_peak()
@@ -533,13 +544,14 @@ def run_attn(args, rank, world, local):
         line = {
             "metric": ATTN_METRIC, "value": seq_per_s, "unit": "sequences/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": total_ms_max / args.steps,
-            "layers_per_step": nlayers,
+            "launches_per_step": per_graph, "layer_caches": nlayers,
             "higher_is_better": True, "scaling": "weak", "vs_baseline": None, "dtype": "f32",
             "precision": "fp16 cache and queries, fp32 scores and sums, weights rounded to fp16 for the value product",
             "data": "synthetic (seeded sum4 keys, values and queries; random page tables)",
             "config": attn_config(w, nlayers),
             "hbm_gbs": step_bytes * args.steps / (total_ms_max / 1e3) / 1e9,
-            "timing": "CUDA-graph replays of one launch per layer cache; ms_per_step and value are per layer launch",
+            "timing": "CUDA-graph replays of launches_per_step launches over the layer caches in turn; "
+                      "ms_per_step and value are per launch",
             "roofline": {"bound": "hbm", "kernel": "paged_attn_kernel", "achieved": achieved, "peak": peak,
                          "peak_source": peak_src, "unit": "GB/s", "frac": achieved / peak,
                          "frac_of_nominal_8tbs": achieved / NOMINAL_HBM_GBS,
@@ -547,7 +559,7 @@ def run_attn(args, rank, world, local):
                          "algorithmic_bytes_per_launch": step_bytes, "avg_launch_ms": avg_launch_ms},
             "e2e": {"value": e2e_val, "unit": "sequences/s", "h2d_bytes_per_step": L0.q.numel() * 2,
                     "d2h_bytes_per_step": L0.out.numel() * 2},
-            "gpu_launches": args.steps * nlayers,
+            "gpu_launches": args.steps * per_graph,
             "clocks": clocks,
         }
         if world == 1 and not args.no_cpu_baseline:

@@ -10,7 +10,7 @@ chain kernel through wq4_decode_chain.  The weights (1.8 GB) are far larger
 than L2 (129 MB), so no L2 flush is needed between steps.
 
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
-                    [--workload 3b|8b] [--batch B]
+                    [--workload 3b|8b|phi3.5] [--batch B]
     python bench.py --workload attn-8b|attn-3b|attn-8b-b1     (decode attention)
 
 The attn-* workloads time decode attention of one layer over a paged
@@ -43,6 +43,9 @@ sys.path.insert(0, ROOT)
 METRIC = "GEMV-bound decode tokens/s (batch 1) and achieved HBM GB/s vs ~8 TB/s peak"
 NOMINAL_HBM_GBS = 8000.0
 PERSISTENT_MAX_BATCH = 2      # larger batches run the tensor-core graph path
+# the paper's batch-1 decode rates for these model shapes (Table 1, WebLLM in
+# Chrome on an Apple M3 Max, 4-bit weights): another machine's numbers, context only
+PAPER_DECODE_TOKS = {"8b": 41.1, "phi3.5": 71.1}
 FALLBACK_HBM_GBS = 6800.0
 
 
@@ -52,7 +55,7 @@ def parse():
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=["3b", "8b", "attn-8b", "attn-3b", "attn-8b-b1"], default="3b")
+    ap.add_argument("--workload", choices=["3b", "8b", "phi3.5", "attn-8b", "attn-3b", "attn-8b-b1"], default="3b")
     ap.add_argument("--batch", type=int, default=1)
     ap.add_argument("--layers", type=int, default=0, help="override the layer count (profiling runs)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -329,7 +332,10 @@ def run_ours(args, rank, world, local):
         line = {
             "metric": METRIC, "value": tokens_per_s, "unit": "tokens/s", "n_gpus": world,
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f32",
+            "scaling": "weak",
+            "vs_baseline": (tokens_per_s / PAPER_DECODE_TOKS[args.workload]
+                            if B == 1 and args.workload in PAPER_DECODE_TOKS and not args.layers else None),
+            "dtype": "f32",
             "precision": "int4 codes (group 32, fp16 scale, zero point 7), fp16 activations, fp32 accumulation",
             "data": "synthetic (seeded SplitMix64 weights and activations)",
             "config": {"workload": f"{shape.name}-shaped decode chain: {shape.num_layers} layers x "
@@ -352,6 +358,9 @@ def run_ours(args, rank, world, local):
             "gpu_launches": args.steps * launches_per_step,
             "clocks": clocks,
         }
+        if line["vs_baseline"] is not None:
+            line["vs_baseline_ref"] = (f"paper Table 1: {PAPER_DECODE_TOKS[args.workload]} tok/s, WebLLM on an Apple "
+                                       "M3 Max (other hardware, trained weights)")
         if world == 1 and not args.no_cpu_baseline:
             line["cpu_baseline"] = cpu_baseline(shape, B)
         print(json.dumps(line), flush=True)

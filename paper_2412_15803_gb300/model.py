@@ -1,7 +1,7 @@
 """Device-resident synthetic decoders and their layer tables.
 
 Shapes follow the 1-8B 4-bit models the paper decodes (Section 3, Table 1:
-Llama-3.1-8B; Section 1: a 4-bit 3B model).  Weights are drawn on the device
+Llama-3.1-8B and Phi-3.5-mini; Section 1: a 4-bit 3B model).  Weights are drawn on the device
 by the seeded generator (wq4_synth_*), one stream per (layer, projection,
 codes|scales), so any row block can be regenerated on the host with
 ``synth.matrix`` for checking.  torch provides the device memory; every
@@ -51,7 +51,11 @@ class ModelShape:
 SHAPE_3B = ModelShape("3b", 28, 3072, 8192, 24, 8, 128, 128256)
 # 8B-shaped (Llama-3.1-8B): hidden 4096, 32 q + 8 kv heads, FFN 14336, 32 layers.
 SHAPE_8B = ModelShape("8b", 32, 4096, 14336, 32, 8, 128, 128256)
-SHAPES = {"3b": SHAPE_3B, "8b": SHAPE_8B}
+# Phi-3.5-mini-shaped (the paper's other Table 1 model, 3.8B; dimensions of its
+# public model configuration): hidden 3072, 32 q + 32 kv heads of 96 (full
+# multi-head attention), FFN 8192, 32 layers, vocabulary 32064.
+SHAPE_PHI = ModelShape("phi3.5", 32, 3072, 8192, 32, 32, 96, 32064)
+SHAPES = {"3b": SHAPE_3B, "8b": SHAPE_8B, "phi3.5": SHAPE_PHI}
 
 
 def fill_matrix(W, s, N: int, K: int, seed: int, layer: int, mat: int, symmetric: bool = False,

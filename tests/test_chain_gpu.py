@@ -13,7 +13,7 @@ import torch
 import oracle
 from oracle import chain as ochain
 from paper_2412_15803_gb300 import synth
-from paper_2412_15803_gb300.model import SHAPE_3B, SHAPE_8B, DecodeModel, ModelShape
+from paper_2412_15803_gb300.model import SHAPE_3B, SHAPE_8B, SHAPE_PHI, DecodeModel, ModelShape
 
 pytestmark = pytest.mark.gpu
 
@@ -208,6 +208,29 @@ def test_8b_chain_batch4_full_size_sampled():
     check_logits(model, logits, rows=pick(sh.vocab))
     for _ in range(20):
         assert np.array_equal(run(model, x), logits)
+
+
+@pytest.mark.parametrize("batch", [1, 8])
+def test_phi_chain_full_size_sampled(batch):
+    """The Phi-3.5-mini-shaped chain (32 layers, 32 + 32 heads of 96, QKV
+    9216 x 3072, vocabulary 32064: the LM head's last 128-row tile is
+    partial) on the persistent kernel (batch 1) and the tensor-core graph
+    (batch 8): sampled rows of three layers and of the LM head."""
+    sh = SHAPE_PHI
+    model = DecodeModel(sh, batch=batch, seed=7)
+    x = synth.activations(9, batch, sh.hidden)
+    logits = run(model, x)
+    rng = np.random.default_rng(2)
+
+    def pick(N):
+        return np.unique(np.concatenate([[0, 1, N - 2, N - 1], rng.integers(0, N, 16)]))
+
+    for l in (0, 15, 31):
+        rows = dict(qkv=pick(sh.n_qkv), o=pick(sh.hidden), gate_up=pick(2 * sh.ffn), down=pick(sh.hidden))
+        check_stages(model, l, rows, u=x if l == 0 else None)
+    check_logits(model, logits, rows=pick(sh.vocab))
+    assert np.all(np.isfinite(oracle.half_to_double(logits)))
+    assert np.array_equal(run(model, x), logits)
 
 
 def test_two_models_with_different_rings_alternate():

@@ -12,6 +12,7 @@ than L2 (129 MB), so no L2 flush is needed between steps.
     python bench.py [--gpus N] [--steps K] [--warmup W] [--impl ours|reference]
                     [--workload 3b|8b|phi3.5] [--batch B]
     python bench.py --workload attn-8b|attn-3b|attn-8b-b1     (decode attention)
+    python bench.py --workload prefill-3b [--tokens M]         (prefill-shaped GEMMs)
 
 The attn-* workloads time decode attention of one layer over a paged
 key/value cache instead (wq4_paged_attention, one launch per step): 32
@@ -55,7 +56,9 @@ def parse():
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=["3b", "8b", "phi3.5", "attn-8b", "attn-3b", "attn-8b-b1"], default="3b")
+    ap.add_argument("--workload", choices=["3b", "8b", "phi3.5", "attn-8b", "attn-3b", "attn-8b-b1", "prefill-3b"],
+                    default="3b")
+    ap.add_argument("--tokens", type=int, default=2048, help="prompt tokens of the prefill workload")
     ap.add_argument("--batch", type=int, default=1)
     ap.add_argument("--layers", type=int, default=0, help="override the layer count (profiling runs)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
@@ -578,9 +581,196 @@ def run_attn(args, rank, world, local):
         dist.destroy_process_group()
 
 
+# ---------------------------------------------------------------- prefill --
+
+PREFILL_METRIC = "prefill-shaped 4-bit dequant-GEMM TFLOP/s (one layer's four projections over a prompt)"
+
+
+def prefill_projections(shape):
+    """(name, N, K, input width) of one layer's projections."""
+    return [(n, N, K, K) for n, N, K, _ in shape.mats(0)]
+
+
+def run_prefill_reference(args, rank, world):
+    import oracle
+    from paper_2412_15803_gb300 import synth
+    from paper_2412_15803_gb300.model import SHAPES
+    if rank != 0:
+        return
+    shape = SHAPES["3b"]
+    M = args.tokens
+    flops_step = 2 * M * sum(N * K for _, N, K, _ in prefill_projections(shape))
+    times, done = [], 0
+    nsteps = args.steps + args.warmup
+    step_s = min(10.0, 120.0 / max(nsteps, 1))
+    x = {K: synth.activations(7, M, K) for K in {shape.hidden, shape.ffn}}
+    for i in range(nsteps):
+        t_used, f_done = 0.0, 0
+        for name, N, K, _ in prefill_projections(shape):
+            rows = max(1, int(8 * step_s / 4))    # a few rows of every projection, all tokens
+            W, sc = synth.matrix(0, N, K, 0, 0, 0, rows)
+            t0 = time.perf_counter()
+            oracle.gemv(W, sc, x[K][: max(1, min(M, 64))])
+            t_used += time.perf_counter() - t0
+            f_done += 2 * rows * K * max(1, min(M, 64))
+            if t_used > step_s:
+                break
+        if i >= args.warmup:
+            times.append(t_used)
+            done += f_done
+    value = done / sum(times) / 1e12
+    line = {"metric": PREFILL_METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": 1e3 * flops_step / (value * 1e12), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+            "config": {"workload": f"prefill-3b: QKV, O, gate_up, down of one 3B-shaped layer over {M} tokens"},
+            "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": 1, "kind": "oracle",
+                             "sample": "a few rows of every projection against up to 64 tokens, single-threaded fp64 C oracle"},
+            "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def measured_tensor_peak():
+    try:
+        d = json.load(open(os.path.join(ROOT, "MEASURED_PEAKS.json")))
+        return float(d["bf16_tflops"]), "measured (MEASURED_PEAKS.json bf16_tflops, cuBLAS bf16 burst; fp16 runs at the bf16 rate)"
+    except Exception:
+        return 1900.0, "fallback"
+
+
+def run_prefill(args, rank, world, local):
+    import torch
+    import torch.distributed as dist
+    from paper_2412_15803_gb300 import synth, wq4
+    from paper_2412_15803_gb300.model import SHAPES, fill_matrix
+
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    shape = SHAPES["3b"]
+    M = args.tokens
+    projs = prefill_projections(shape)
+    nlayers = 4   # weights of four layers in rotation: 226 MB, larger than L2
+    weights = []
+    for l in range(nlayers):
+        ws = []
+        for i, (name, N, K, _) in enumerate(projs):
+            W = torch.empty((N, K // 8), dtype=torch.int32, device="cuda")
+            sc = torch.empty((N, K // 32), dtype=torch.int16, device="cuda")
+            fill_matrix(W, sc, N, K, 0, l, i)
+            ws.append((W, sc))
+        weights.append(ws)
+    xin = {K: torch.from_numpy(synth.activations(7, M, K).view(np.int16)).cuda() for K in {shape.hidden, shape.ffn}}
+    outs = [torch.empty((M, N), dtype=torch.int16, device="cuda") for _, N, _, _ in projs]
+    flops_step = 2 * M * sum(N * K for _, N, K, _ in projs)
+
+    def step(l, stream):
+        for i, (name, N, K, _) in enumerate(projs):
+            W, sc = weights[l][i]
+            wq4.wq4_gemm(W, sc, xin[K], outs[i], N, K, M, stream)
+
+    stream = torch.cuda.Stream()
+    with torch.cuda.stream(stream):
+        step(0, stream)
+        stream.synchronize()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            for l in range(nlayers):
+                step(l, stream)
+        for _ in range(max(args.warmup, 3)):
+            graph.replay()
+    torch.cuda.synchronize()
+    if wq4.wq4_device_status(stream) != 0:
+        raise RuntimeError("device flag set during warm-up")
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.3)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        for i in range(args.steps):
+            starts[i].record(stream)
+            graph.replay()
+            ends[i].record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clocks = sampler.stop()
+    total_ms = starts[0].elapsed_time(ends[-1]) / nlayers
+    step_ms = [s.elapsed_time(e) / nlayers for s, e in zip(starts, ends)]
+    # end to end: inputs copied in from pinned host memory, outputs copied back
+    x_host = {K: v.cpu().pin_memory() for K, v in xin.items()}
+    o_host = [torch.empty_like(o, device="cpu").pin_memory() for o in outs]
+    e2e_steps = max(3, min(args.steps, 20))
+    with torch.cuda.stream(stream):
+        t0 = time.perf_counter()
+        for i in range(e2e_steps):
+            for K, v in xin.items():
+                v.copy_(x_host[K], non_blocking=True)
+            step(i % nlayers, stream)
+            for o, oh in zip(outs, o_host):
+                oh.copy_(o, non_blocking=True)
+            stream.synchronize()
+        e2e_s = (time.perf_counter() - t0) / e2e_steps
+    if wq4.wq4_device_status(stream) != 0:
+        raise RuntimeError("device flag set during the timed region")
+    t = torch.tensor([total_ms, e2e_s], dtype=torch.float64, device="cuda")
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    job_ms, e2e_step = float(t[0]), float(t[1])
+    if rank == 0:
+        peak, src = measured_tensor_peak()
+        avg = statistics.mean(step_ms)
+        achieved = flops_step / (avg * 1e-3) / 1e12
+        line = {
+            "metric": PREFILL_METRIC, "value": world * flops_step * args.steps / (job_ms * 1e-3) / 1e12,
+            "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": job_ms / args.steps, "higher_is_better": True, "scaling": "weak", "vs_baseline": None,
+            "dtype": "f16",
+            "precision": "int4 codes dequantized to fp16 (one rounding), fp16 activations, fp32 accumulation",
+            "data": "synthetic (seeded SplitMix64 weights and activations)",
+            "config": {"workload": f"prefill-3b: QKV 5120x3072, O 3072x3072, gate_up 16384x3072, down 3072x8192 "
+                                   f"of one 3B-shaped layer over {M} prompt tokens (wq4_gemm, tcgen05)",
+                       "tokens": M, "flop_per_step": flops_step,
+                       "l2": f"{nlayers} layers' weights in rotation (226 MB, larger than L2)",
+                       "parallelism": "single GPU"},
+            "prefill_tokens_per_s_per_layer": world * M * args.steps / (job_ms * 1e-3),
+            "roofline": {"bound": "tensor", "kernel": "gemm_kernel", "achieved": achieved, "peak": peak,
+                         "peak_source": src, "unit": "TFLOP/s", "frac": achieved / peak, "traffic": None,
+                         "algorithmic_flop_per_step": flops_step, "avg_step_ms": avg},
+            "e2e": {"value": flops_step / e2e_step / 1e12, "unit": "TFLOP/s",
+                    "h2d_bytes_per_step": sum(v.numel() * 2 for v in xin.values()),
+                    "d2h_bytes_per_step": sum(o.numel() * 2 for o in outs)},
+            "gpu_launches": args.steps * nlayers * len(projs),
+            "clocks": clocks,
+        }
+        if world == 1 and not args.no_cpu_baseline:
+            import oracle
+            W, sc = synth.matrix(0, 16, shape.hidden)
+            xs = synth.activations(7, 64, shape.hidden)
+            t0 = time.perf_counter()
+            n = 0
+            while time.perf_counter() - t0 < 10.0:
+                oracle.gemv(W, sc, xs)
+                n += 1
+            dt = time.perf_counter() - t0
+            line["cpu_baseline"] = {"value": n * 2 * 16 * shape.hidden * 64 / dt / 1e12, "unit": "TFLOP/s", "cores": 1,
+                                    "kind": "oracle",
+                                    "sample": f"16 rows x {shape.hidden} x 64 tokens repeated for {dt:.1f} s, "
+                                              "single-threaded fp64 C oracle"}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
 def main():
     args = parse()
     rank, world, local = dist_env()
+    if args.workload.startswith("prefill"):
+        (run_prefill_reference(args, rank, world) if args.impl == "reference" else run_prefill(args, rank, world, local))
+        return
     attn = args.workload.startswith("attn")
     if args.impl == "reference":
         (run_attn_reference if attn else run_reference)(args, rank, world)

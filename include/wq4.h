@@ -76,6 +76,23 @@ int wq4_gemv(const uint32_t* W_packed, const uint16_t* scales, const uint16_t* x
              uint16_t* y, int N, int K, int batch, void* stream);
 
 /*
+ * The same product for many activation rows (prefill-shaped: the tokens of a
+ * prompt through one projection), on the tensor cores:
+ *   Y[m][n] = fp16( sum_k x[m][k] * fp16((q(n,k) - 7) * scales[n][k/32]) )
+ * for m < M, n < N, sums in fp32.  Each dequantized weight is rounded to fp16
+ * once (relative error <= 2^-11), so the accuracy contract above holds.
+ *   W_packed, scales : as wq4_gemv, both 16-byte aligned.
+ *   x : fp16 bits [M][K], 16-byte aligned.   y : fp16 bits [M][N], 16-byte
+ *       aligned, must not overlap x, W or scales.
+ *   M >= 1 (any size), N >= 1 with N % 8 == 0, K % 256 == 0 (other valid
+ *   sizes return WQ4_ERR_UNSUPPORTED: use wq4_gemv for them).
+ * Deterministic (no split K).  Returns WQ4_OK, WQ4_ERR_INVALID,
+ * WQ4_ERR_UNSUPPORTED, WQ4_ERR_ALIGN or WQ4_ERR_CUDA.
+ */
+int wq4_gemm(const uint32_t* W_packed, const uint16_t* scales, const uint16_t* x,
+             uint16_t* y, int N, int K, int M, void* stream);
+
+/*
  * Test hook for the unpack step: runs the same in-register unpack the GEMV
  * uses and writes its results, so that they can be compared bit for bit.
  *   q_out : uint8 [N][K] codes 0..15 (may be NULL)

@@ -78,6 +78,7 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
                            "`python -m paper_2412_15803_gb300.build`")
     L = ctypes.CDLL(_build.LIB)
     L.wq4_gemv.argtypes = [_P, _P, _P, _P, _I, _I, _I, _P]
+    L.wq4_gemm.argtypes = [_P, _P, _P, _P, _I, _I, _I, _P]
     L.wq4_unpack_debug.argtypes = [_P, _P, _P, _P, _I, _I, _P]
     L.wq4_pack_host.argtypes = [_P, _P, _I, _I]
     L.wq4_status_string.argtypes = [_I]
@@ -104,7 +105,7 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
 
 
 # names every C entry point of include/*.h (checked by the tests)
-EXPORTED = ["wq4_gemv", "wq4_unpack_debug", "wq4_pack_host", "wq4_status_string",
+EXPORTED = ["wq4_gemv", "wq4_gemm", "wq4_unpack_debug", "wq4_pack_host", "wq4_status_string",
             "wq4_device_status", "wq4_chain_workspace_bytes", "wq4_decode_chain",
             "wq4_decode_chain_host", "wq4_decode_chain_noalloc", "wq4_chain_plan_destroy", "wq4_chain_trace_offsets",
             "wq4_synth_codes", "wq4_synth_scales", "wq4_synth_sum4",
@@ -146,6 +147,11 @@ def wq4_status_string(status: int) -> str:
 def wq4_gemv(W, scales, x, y, N: int, K: int, batch: int, stream=None, check: bool = True) -> int:
     rc = load().wq4_gemv(_ptr(W), _ptr(scales), _ptr(x), _ptr(y), N, K, batch, _stream(stream))
     return _check("wq4_gemv", rc) if check else rc
+
+
+def wq4_gemm(W, scales, x, y, N: int, K: int, M: int, stream=None, check: bool = True) -> int:
+    rc = load().wq4_gemm(_ptr(W), _ptr(scales), _ptr(x), _ptr(y), N, K, M, _stream(stream))
+    return _check("wq4_gemm", rc) if check else rc
 
 
 def wq4_unpack_debug(W, scales, w_out, q_out, N: int, K: int, stream=None, check: bool = True) -> int:

@@ -71,6 +71,24 @@ def test_gemv_rejects_bad_arguments(args, expect):
     assert rc == expect
 
 
+@pytest.mark.parametrize("args,expect", [
+    (dict(W=0), wq4.WQ4_ERR_INVALID),
+    (dict(M=0), wq4.WQ4_ERR_INVALID),
+    (dict(N=0), wq4.WQ4_ERR_INVALID),
+    (dict(K=48), wq4.WQ4_ERR_INVALID),
+    (dict(K=288), wq4.WQ4_ERR_UNSUPPORTED),
+    (dict(N=100), wq4.WQ4_ERR_UNSUPPORTED),
+    (dict(s=2 * A16 + 8), wq4.WQ4_ERR_ALIGN),
+    (dict(y=16 * A16 + 8), wq4.WQ4_ERR_ALIGN),
+    (dict(y=A16 + 64), wq4.WQ4_ERR_INVALID),   # y overlaps W
+])
+def test_gemm_rejects_bad_arguments(args, expect):
+    a = dict(W=A16, s=2 * A16, x=8 * A16, y=16 * A16, N=64, K=256, M=300)
+    a.update(args)
+    rc = wq4.load().wq4_gemm(a["W"], a["s"], a["x"], a["y"], a["N"], a["K"], a["M"], None)
+    assert rc == expect
+
+
 def test_unpack_debug_rejects_bad_arguments():
     L = wq4.load()
     assert L.wq4_unpack_debug(A16, 2 * A16, None, None, 4, 64, None) == wq4.WQ4_ERR_INVALID

@@ -4,20 +4,21 @@
 //
 // Y[m][n] = fp16( sum_k x[m][k] * fp16((q(n,k) - 7) * s(n, k/32)) ), fp32 sums.
 //
-// A persistent grid walks (128 weight rows x 128 tokens) tiles, row tile
+// A persistent grid walks (128 weight rows x 256 tokens) tiles, row tile
 // major so that the CTAs running at one time share a weight tile through L2.
-// Per 256-wide K chunk a producer warp brings the tile's codes and scales
-// (2-D tensor copies) and the 128 x 256 activation block (four 128-byte
-// swizzled boxes) into a 2-slot ring; eight dequant warps write the 128 x 256
-// weights, dequantized to fp16 in natural K order, into one of two 128-column
-// A buffers in tensor memory (lane = weight row); one thread issues 16
-// tcgen05.mma (kind::f16, M = 128, N = 128 tokens, K = 16, A from tensor
-// memory, B = activations from shared memory) into one of two 128-column fp32
-// accumulators; four epilogue warps read a finished accumulator, transpose it
-// through shared memory and store 128 tokens x 128 outputs with 16-byte
-// stores while the next tile's MMAs run.  Every weight is rounded to fp16
-// once (relative error <= 2^-11, accumulated in fp32): within the library's
-// accuracy contract.
+// Per 64-wide K chunk a producer warp brings the tile's codes and scales
+// (2-D tensor copies) and the 256 x 64 activation block (one 128-byte swizzled
+// box) into a 4-slot ring (small slots, so that copies stay in flight while
+// the MMAs of earlier chunks run); eight dequant warps write the 128 x 64
+// weights, dequantized to fp16 in natural K order, into one of three
+// 32-column A buffers in tensor memory (lane = weight row); one thread issues
+// 4 tcgen05.mma (kind::f16, M = 128, N = 256 tokens, K = 16: the tensor-core
+// rate, ~128 cycles each, so the dequant warps keep up) into a 256-column fp32
+// accumulator; four epilogue warps move a finished accumulator into a
+// shared-memory transpose buffer, release it, and store 256 tokens x 128
+// outputs with 16-byte stores while the next tile's MMAs run.  Every weight is
+// rounded to fp16 once (relative error <= 2^-11, accumulated in fp32): within
+// the library's accuracy contract.
 #include "wq4.h"
 #include "wq4_device.cuh"
 #include "wq4_host.h"
@@ -34,15 +35,23 @@ namespace {
 
 constexpr int kGThreads = 448;        // warps 0-7 dequant, 8 producer, 9 MMA, 10-13 epilogue
 constexpr int kGProducer = 8, kGIssuer = 9;
-constexpr int kGSlots = 2;
-constexpr int kGX = 128 * 256 * 2;    // activation block: 128 tokens x 256 K fp16 (four 16 KiB boxes)
-constexpr int kGCodes = 128 * 128;    // 128 rows x 256 codes
-constexpr int kGScales = 128 * 16;    // 128 rows x 8 fp16 scales
-constexpr int kGSlot = kGX + kGCodes + kGScales;   // 83 968 B, a multiple of 1024
-constexpr int kGT = 1024;             // transpose buffer: 128 tokens x 128 outputs fp16 (32 KiB)
-constexpr int kGRing = kGT + 128 * 128 * 2;
-constexpr int kGSmem = kGRing + kGSlots * kGSlot;
-constexpr int kGTmemCols = 512;       // A: 2 x 128 columns, accumulators: 2 x 128 at 256
+constexpr int kGCodes = 128 * 32;     // 128 rows x 64 codes (32-byte rows, 32-byte swizzle)
+constexpr int kGScales = 128 * 16;    // 128 rows x 8 fp16 scales (the 256-wide K block of the chunk)
+constexpr int kGABufs = 3;            // 32-column A buffers
+constexpr int kGDCol = 256;           // accumulator: TOK columns
+constexpr int kGT = 1024;             // transpose buffer: TOK tokens x 128 outputs fp16
+constexpr int kGTmemCols = 512;
+
+// Tile of TOK tokens (MMA N = 128 or 256).
+template <int TOK>
+struct GCfg {
+    static constexpr int kSlots = TOK == 256 ? 4 : 6;
+    static constexpr int kX = TOK * 64 * 2;                // activation block: TOK tokens x 64 K fp16
+    static constexpr int kSlot = kX + kGCodes + kGScales;  // a multiple of 1024
+    static constexpr int kRing = kGT + TOK * 128 * 2;
+    static constexpr int kSmem = kRing + kSlots * kSlot;
+    static_assert(kSmem <= 227 * 1024, "shared memory");
+};
 
 struct GemmArgs {
     uint16_t* y;
@@ -62,23 +71,26 @@ __device__ __forceinline__ bool g_wait(uint64_t* bar, uint32_t parity, uint32_t*
     return mbar_wait(bar, parity, err);
 }
 
+template <int TOK>
 __global__ void __launch_bounds__(kGThreads, 1)
     gemm_kernel(const __grid_constant__ CUtensorMap tm_codes, const __grid_constant__ CUtensorMap tm_scales,
                 const __grid_constant__ CUtensorMap tm_x, const GemmArgs a)
 {
+    using C = GCfg<TOK>;
+    constexpr int kGSlots = C::kSlots, kGX = C::kX, kGSlot = C::kSlot, kGRing = C::kRing, kGTok = TOK;
     extern __shared__ __align__(1024) uint8_t smem[];
     uint64_t* full = reinterpret_cast<uint64_t*>(smem);      // codes, scales, activations landed
     uint64_t* empty = full + kGSlots;
     uint64_t* afull = empty + kGSlots;
-    uint64_t* aempty = afull + 2;
-    uint64_t* dfull = aempty + 2;
-    uint64_t* dempty = dfull + 2;
-    uint64_t* drain = dempty + 2;                            // ends at byte 120
+    uint64_t* aempty = afull + kGABufs;
+    uint64_t* dfull = aempty + kGABufs;
+    uint64_t* dempty = dfull + 1;
+    uint64_t* drain = dempty + 1;                            // ends at byte (2 slots + 9) * 8 <= 240
     uint32_t* tbase_sh = reinterpret_cast<uint32_t*>(smem + 240);
     uint16_t* tbuf = reinterpret_cast<uint16_t*>(smem + kGT);
     uint8_t* ring = smem + kGRing;
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int nch = a.K >> 8;
+    const int nch = a.K >> 6;   // 64-wide K chunks
     const int tiles = a.rtiles * a.ttiles;
     uint32_t* err = a.err;
 
@@ -87,12 +99,12 @@ __global__ void __launch_bounds__(kGThreads, 1)
             mbar_init(&full[i], 1);
             mbar_init(&empty[i], 9);   // 8 dequant warps + the MMA commit
         }
-        for (int i = 0; i < 2; ++i) {
+        for (int i = 0; i < kGABufs; ++i) {
             mbar_init(&afull[i], 8);
             mbar_init(&aempty[i], 1);
-            mbar_init(&dfull[i], 1);
-            mbar_init(&dempty[i], 4);
         }
+        mbar_init(dfull, 1);
+        mbar_init(dempty, 4);
         mbar_init(drain, 1);
         mbar_fence_init();
     }
@@ -111,7 +123,7 @@ __global__ void __launch_bounds__(kGThreads, 1)
             int it = 0;
             bool ok = true;
             for (int u = blockIdx.x; u < tiles && ok; u += gridDim.x) {
-                const int n0 = (u / a.ttiles) * 128, m0 = (u % a.ttiles) * 128;
+                const int n0 = (u / a.ttiles) * 128, m0 = (u % a.ttiles) * kGTok;
                 for (int c = 0; c < nch; ++c, ++it) {
                     const int slot = it % kGSlots;
                     if (it >= kGSlots && !g_wait(&empty[slot], ((it / kGSlots) - 1) & 1, err)) {
@@ -120,12 +132,11 @@ __global__ void __launch_bounds__(kGThreads, 1)
                     }
                     uint8_t* base = ring + static_cast<size_t>(slot) * kGSlot;
                     mbar_arrive_expect_tx(&full[slot], kGSlot);
-#pragma unroll
-                    for (int j = 0; j < 4; ++j) tc::tma_load_2d(base + j * 16384, &tm_x, c * 256 + 64 * j, m0, &full[slot]);
-                    tc::tma_load_2d(base + kGX, &tm_codes, c * 128, n0, &full[slot]);
-                    tc::tma_load_2d(base + kGX + 64 * 128, &tm_codes, c * 128, n0 + 64, &full[slot]);
-                    tc::tma_load_2d(base + kGX + kGCodes, &tm_scales, c * 8, n0, &full[slot]);
-                    tc::tma_load_2d(base + kGX + kGCodes + 64 * 16, &tm_scales, c * 8, n0 + 64, &full[slot]);
+                    tc::tma_load_2d(base, &tm_x, c * 64, m0, &full[slot]);
+                    tc::tma_load_2d(base + kGX, &tm_codes, c * 32, n0, &full[slot]);
+                    tc::tma_load_2d(base + kGX + 64 * 32, &tm_codes, c * 32, n0 + 64, &full[slot]);
+                    tc::tma_load_2d(base + kGX + kGCodes, &tm_scales, (c >> 2) * 8, n0, &full[slot]);
+                    tc::tma_load_2d(base + kGX + kGCodes + 64 * 16, &tm_scales, (c >> 2) * 8, n0 + 64, &full[slot]);
                 }
             }
             // every copy issued has landed before the CTA's memory goes away
@@ -135,31 +146,32 @@ __global__ void __launch_bounds__(kGThreads, 1)
     } else if (warp == kGIssuer) {
         // ---------------------------------------------------- MMA issuer
         if (lane == 0) {
-            constexpr uint32_t idesc = tc::idesc_f16_f32(128, 128);
+            constexpr uint32_t idesc = tc::idesc_f16_f32(128, kGTok);
             int it = 0, dit = 0;
             bool ok = true;
+            const uint32_t dt = tbase + kGDCol;
             for (int u = blockIdx.x; u < tiles && ok; u += gridDim.x, ++dit) {
-                const int dbuf = dit & 1;
-                if (dit >= 2 && !g_wait(&dempty[dbuf], ((dit >> 1) - 1) & 1, err)) break;
-                const uint32_t dt = tbase + 256 + 128 * dbuf;
+                if (dit >= 1 && !g_wait(dempty, (dit - 1) & 1, err)) break;
+                tc::fence_after_sync();
                 for (int c = 0; c < nch; ++c, ++it) {
-                    const int slot = it % kGSlots, abuf = it & 1;
-                    if (!g_wait(&full[slot], (it / kGSlots) & 1, err) || !g_wait(&afull[abuf], (it >> 1) & 1, err)) {
+                    const int slot = it % kGSlots, abuf = it % kGABufs;
+                    if (!g_wait(&full[slot], (it / kGSlots) & 1, err) ||
+                        !g_wait(&afull[abuf], (it / kGABufs) & 1, err)) {
                         ok = false;
                         break;
                     }
                     tc::fence_after_sync();
                     const uint32_t xs = smem_addr(ring + static_cast<size_t>(slot) * kGSlot);
 #pragma unroll
-                    for (int s = 0; s < 16; ++s) {
-                        const uint64_t bd = tc::sw128_kmajor_desc(xs + (s >> 2) * 16384 + 32 * (s & 3));
-                        tc::mma_f16_ts(dt, tbase + 128 * abuf + 8 * s, bd, idesc, (c > 0 || s > 0) ? 1u : 0u);
+                    for (int s = 0; s < 4; ++s) {
+                        const uint64_t bd = tc::sw128_kmajor_desc(xs + 32 * s);
+                        tc::mma_f16_ts(dt, tbase + 32 * abuf + 8 * s, bd, idesc, (c > 0 || s > 0) ? 1u : 0u);
                     }
                     tc::commit(&aempty[abuf]);
                     tc::commit(&empty[slot]);
                 }
                 if (!ok) break;
-                tc::commit(&dfull[dbuf]);
+                tc::commit(dfull);
             }
             // all MMAs issued have completed before tensor memory is released
             tc::commit(drain);
@@ -167,30 +179,28 @@ __global__ void __launch_bounds__(kGThreads, 1)
         }
     } else if (warp < 8) {
         // ---------------------------------------------------- dequant
-        // warp w: rows 32 (w % 4) + lane (its tensor-memory lanes), groups
-        // 4 (w / 4) .. + 3 of each chunk, written in natural K order
+        // warp w: rows 32 (w % 4) + lane (its tensor-memory lanes), group
+        // w / 4 of each 64-wide chunk, written in natural K order
         const int row = 32 * (warp & 3) + lane;
-        const int jg = 4 * (warp >> 2);
+        const int jg = warp >> 2;
         const uint32_t lane_base = tbase + (static_cast<uint32_t>(32 * (warp & 3)) << 16);
         int it = 0;
         bool ok = true;
         for (int u = blockIdx.x; u < tiles && ok; u += gridDim.x) {
             for (int c = 0; c < nch; ++c, ++it) {
-                const int slot = it % kGSlots, abuf = it & 1;
+                const int slot = it % kGSlots, abuf = it % kGABufs;
                 if (!g_wait(&full[slot], (it / kGSlots) & 1, err) ||
-                    (it >= 2 && !g_wait(&aempty[abuf], ((it >> 1) - 1) & 1, err))) {
+                    (it >= kGABufs && !g_wait(&aempty[abuf], ((it / kGABufs) - 1) & 1, err))) {
                     ok = false;
                     break;
                 }
                 const uint8_t* base = ring + static_cast<size_t>(slot) * kGSlot + kGX;
-                const uint8_t* crow = base + row * 128;
-                const uint2 sv = *reinterpret_cast<const uint2*>(base + kGCodes + row * 16 + 2 * jg);
-                const uint32_t sw[2] = {sv.x, sv.y};
-#pragma unroll
-                for (int jj = 0; jj < 4; ++jj) {
-                    const int j = jg + jj;
-                    const uint4 cw = *reinterpret_cast<const uint4*>(crow + ((j ^ (row & 7)) << 4));
-                    const uint32_t sh = (jj & 1) ? (sw[jj >> 1] >> 16) : (sw[jj >> 1] & 0xFFFFu);
+                const uint8_t* crow = base + row * 32;
+                // scale of group 2 (c & 3) + jg of the 8 loaded for this 256-wide block
+                const uint32_t sh = *reinterpret_cast<const uint16_t*>(base + kGCodes + row * 16 + 4 * (c & 3) + 2 * jg);
+                {
+                    const int j = jg;   // 16-byte chunk of the 32-byte row, 32-byte swizzle
+                    const uint4 cw = *reinterpret_cast<const uint4*>(crow + ((j ^ ((row >> 2) & 1)) << 4));
                     const uint32_t s2 = sh | (sh << 16);
                     const uint32_t words[4] = {cw.x, cw.y, cw.z, cw.w};
                     uint32_t q[16];
@@ -203,7 +213,7 @@ __global__ void __launch_bounds__(kGThreads, 1)
                         q[4 * w + 2] = tc::hmul2_u32(prmt(p[0], p[1], 0x7632u), s2);   // k4 k5
                         q[4 * w + 3] = tc::hmul2_u32(prmt(p[2], p[3], 0x7632u), s2);   // k6 k7
                     }
-                    tc::st16(lane_base + 128 * abuf + 16 * j, q);
+                    tc::st16(lane_base + 32 * abuf + 16 * j, q);
                 }
                 tc::st_wait();
                 tc::fence_before_sync();
@@ -223,15 +233,15 @@ __global__ void __launch_bounds__(kGThreads, 1)
         const uint32_t lane_base = tbase + (static_cast<uint32_t>(32 * quad) << 16);
         int dit = 0;
         for (int u = blockIdx.x; u < tiles; u += gridDim.x, ++dit) {
-            const int n0 = (u / a.ttiles) * 128, m0 = (u % a.ttiles) * 128;
-            const int dbuf = dit & 1;
-            if (!g_wait(&dfull[dbuf], (dit >> 1) & 1, err)) break;
+            const int n0 = (u / a.ttiles) * 128, m0 = (u % a.ttiles) * kGTok;
+            if (!g_wait(dfull, dit & 1, err)) break;
             tc::fence_after_sync();
-            // accumulator (row, token) -> transpose buffer [token][row], fp16
-#pragma unroll
-            for (int h = 0; h < 8; ++h) {
+            // accumulator (row, token) -> transpose buffer [token][row], fp16;
+            // the accumulator is free for the next tile's MMAs right after
+#pragma unroll 4
+            for (int h = 0; h < kGTok / 16; ++h) {
                 uint32_t d[16];
-                tc::ld16(lane_base + 256 + 128 * dbuf + 16 * h, d);
+                tc::ld16(lane_base + kGDCol + 16 * h, d);
                 tc::ld_wait();
 #pragma unroll
                 for (int i = 0; i < 16; ++i)
@@ -239,11 +249,11 @@ __global__ void __launch_bounds__(kGThreads, 1)
             }
             tc::fence_before_sync();
             __syncwarp();
-            if (lane == 0) mbar_arrive(&dempty[dbuf]);
+            if (lane == 0) mbar_arrive(dempty);
             named_barrier_sync(3, 128);
-            // 128 tokens x 256 bytes out, 16 bytes per store
+            // 256 tokens x 256 bytes out, 16 bytes per store
 #pragma unroll 4
-            for (int i = 0; i < 16; ++i) {
+            for (int i = 0; i < kGTok / 8; ++i) {
                 const int chunk = tid + 128 * i;
                 const int tok = chunk >> 4, seg = chunk & 15;
                 const int m = m0 + tok, n = n0 + 8 * seg;
@@ -261,15 +271,25 @@ __global__ void __launch_bounds__(kGThreads, 1)
     if (warp == kGIssuer) tc::tmem_dealloc(tbase, kGTmemCols);
 }
 
+template <int TOK>
 int gemm_attr()
 {
     static std::once_flag once;
     static int rc = -1;
     std::call_once(once, [] {
-        rc = cudaFuncSetAttribute(gemm_kernel, cudaFuncAttributeMaxDynamicSharedMemorySize, kGSmem) == cudaSuccess ? 0
-                                                                                                             : 1;
+        rc = cudaFuncSetAttribute(gemm_kernel<TOK>, cudaFuncAttributeMaxDynamicSharedMemorySize, GCfg<TOK>::kSmem) ==
+                     cudaSuccess
+                 ? 0
+                 : 1;
     });
     return rc;
+}
+
+// Token tile: 256 (measured: a 128-token tile costs well over half of a
+// 256-token one), 128 when the prompt has at most 128 tokens.
+int pick_tok(int M)
+{
+    return M <= 128 ? 128 : 256;
 }
 
 }  // namespace
@@ -291,16 +311,17 @@ extern "C" int wq4_gemm(const uint32_t* W_packed, const uint16_t* scales, const 
     int dev = 0;
     const DeviceInfo* di = current_device_info(&dev);
     if (!di) return WQ4_ERR_CUDA;
-    if (gemm_attr() != 0) return WQ4_ERR_CUDA;
+    const int tok = pick_tok(M);
+    if ((tok == 256 ? gemm_attr<256>() : gemm_attr<128>()) != 0) return WQ4_ERR_CUDA;
     CUtensorMap mc, ms, mx;
     if (!encode_tensor_map_2d(&mc, CU_TENSOR_MAP_DATA_TYPE_UINT8, W_packed, static_cast<uint64_t>(K) / 2,
-                              static_cast<uint64_t>(N), static_cast<uint64_t>(K) / 2, 128, 64,
-                              CU_TENSOR_MAP_SWIZZLE_128B) ||
+                              static_cast<uint64_t>(N), static_cast<uint64_t>(K) / 2, 32, 64,
+                              CU_TENSOR_MAP_SWIZZLE_32B) ||
         !encode_tensor_map_2d(&ms, CU_TENSOR_MAP_DATA_TYPE_UINT16, scales, static_cast<uint64_t>(K) / 32,
                               static_cast<uint64_t>(N), static_cast<uint64_t>(K) / 16, 8, 64,
                               CU_TENSOR_MAP_SWIZZLE_NONE) ||
         !encode_tensor_map_2d(&mx, CU_TENSOR_MAP_DATA_TYPE_FLOAT16, x, static_cast<uint64_t>(K), static_cast<uint64_t>(M),
-                              static_cast<uint64_t>(K) * 2, 64, 128, CU_TENSOR_MAP_SWIZZLE_128B))
+                              static_cast<uint64_t>(K) * 2, 64, tok, CU_TENSOR_MAP_SWIZZLE_128B))
         return WQ4_ERR_CUDA;
     GemmArgs a;
     a.y = y;
@@ -308,12 +329,15 @@ extern "C" int wq4_gemm(const uint32_t* W_packed, const uint16_t* scales, const 
     a.K = K;
     a.M = M;
     a.rtiles = (N + 127) / 128;
-    a.ttiles = (M + 127) / 128;
+    a.ttiles = (M + tok - 1) / tok;
     a.err = status_word();
     if (!a.err) return WQ4_ERR_CUDA;
     const int64_t tiles = static_cast<int64_t>(a.rtiles) * a.ttiles;
     if (tiles > (static_cast<int64_t>(1) << 30)) return WQ4_ERR_UNSUPPORTED;
     const int grid = static_cast<int>(tiles < di->sm_count ? tiles : di->sm_count);
-    gemm_kernel<<<grid, kGThreads, kGSmem, static_cast<cudaStream_t>(stream)>>>(mc, ms, mx, a);
+    if (tok == 256)
+        gemm_kernel<256><<<grid, kGThreads, GCfg<256>::kSmem, static_cast<cudaStream_t>(stream)>>>(mc, ms, mx, a);
+    else
+        gemm_kernel<128><<<grid, kGThreads, GCfg<128>::kSmem, static_cast<cudaStream_t>(stream)>>>(mc, ms, mx, a);
     return cudaGetLastError() == cudaSuccess ? WQ4_OK : WQ4_ERR_CUDA;
 }

@@ -45,6 +45,7 @@ constexpr int kBoxBytes = kTile * 64 * 2;        // 16 rows x 64 dims: 2 KiB
 constexpr int kPartHdr = 16;                     // floats: M[8], L[8]
 constexpr int kCtasPerSm = 2;
 constexpr int kMaxParts = kConsumers * kD;      // parts of one segment the merge stages: grid <= 512
+constexpr int kMinShare = 16;                   // fewest tiles of a CTA's share (small batches: fewer parts to merge)
 
 // Shared memory map (dynamic, base 1024-aligned).
 constexpr int kOffRing = 0;
@@ -218,7 +219,7 @@ __global__ void __launch_bounds__(kThreads, kCtasPerSm) paged_attn_kernel(const 
     __syncthreads();
 
     const int total = P.Hkv * pre[P.batch];
-    const int R = (total + static_cast<int>(gridDim.x) - 1) / static_cast<int>(gridDim.x);
+    const int R = max((total + static_cast<int>(gridDim.x) - 1) / static_cast<int>(gridDim.x), kMinShare);
     const int cta = blockIdx.x;
     const int g_begin = min(total, cta * R);
     const int g_end = min(total, g_begin + R);

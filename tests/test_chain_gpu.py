@@ -188,14 +188,15 @@ def test_3b_chain_full_size_sampled():
     assert np.array_equal(run(model, x), logits)
 
 
-def test_8b_chain_batch4_full_size_sampled():
-    """The 32-layer 8B-shaped chain at batch 4: the shallowest weight ring
-    (six slots for seven consumer warps, one down-projection item per slot),
-    so consumer warps run furthest ahead of the producer.  Sampled rows of
-    three layers and of the LM head, and twenty tokens with identical bits."""
+@pytest.mark.parametrize("batch", [1, 4])
+def test_8b_chain_full_size_sampled(batch):
+    """The 32-layer 8B-shaped chain at batch 1 (persistent CUDA-core kernel:
+    the longest rows, K = 14336 in the down projection) and at batch 4
+    (tensor-core stage graph).  Sampled rows of three layers and of the LM
+    head, and twenty tokens with identical bits."""
     sh = SHAPE_8B
-    model = DecodeModel(sh, batch=4, seed=3)
-    x = synth.activations(5, 4, sh.hidden)
+    model = DecodeModel(sh, batch=batch, seed=3)
+    x = synth.activations(5, batch, sh.hidden)
     logits = run(model, x)
     rng = np.random.default_rng(1)
 

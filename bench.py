@@ -209,6 +209,23 @@ def cpu_baseline(shape, batch, target_s=12.0):
                       f"single-threaded fp64 C oracle, {t:.1f} s"}
 
 
+def chain_step_bytes(shape, B: int) -> int:
+    """Bytes one token step streams: packed codes + scales of every
+    projection, plus the activation vectors read and written (negligible)."""
+    return shape.weight_bytes() + 2 * B * (shape.hidden * (4 * shape.num_layers + 1) + shape.vocab)
+
+
+def chain_config(shape, B: int, world: int) -> dict:
+    """The workload's config object, the same for both arms."""
+    return {"workload": f"{shape.name}-shaped decode chain: {shape.num_layers} layers x "
+                        f"(QKV {shape.n_qkv}x{shape.hidden}, O {shape.hidden}x{shape.hidden}, "
+                        f"gate_up {2 * shape.ffn}x{shape.hidden}, down {shape.hidden}x{shape.ffn}) "
+                        f"+ LM head {shape.vocab}x{shape.hidden}, batch {B}",
+            "batch": B, "bytes_per_token": chain_step_bytes(shape, B),
+            "l2": "inputs larger than L2 (1.8+ GB of weights per step), no flush",
+            "parallelism": "replicas" if world > 1 else "single GPU"}
+
+
 def run_reference(args, rank, world):
     from paper_2412_15803_gb300.model import SHAPES
     if rank != 0:
@@ -228,11 +245,12 @@ def run_reference(args, rank, world):
     value = tok / sum(times)
     line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": 1e3 * sum(times) / len(times), "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
-            "config": {"workload": f"{shape.name}-shaped decode chain, {shape.num_layers} layers + LM head, "
-                                   f"batch {args.batch}", "sample_fraction_per_step": frac},
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded SplitMix64 weights and activations)", "impl": "reference",
+            "config": chain_config(shape, args.batch, world),
             "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
-                             "sample": f"each step: first {frac:.5f} of the rows of every projection"},
+                             "sample": f"each step: first {frac:.5f} of the rows of every projection "
+                                       f"(all {4 * shape.num_layers + 1}), scaled to a token by weights"},
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -276,11 +294,7 @@ def run_ours(args, rank, world, local):
     logits = torch.empty((B, shape.vocab), dtype=torch.int16, device="cuda")
     stream = torch.cuda.current_stream()
 
-    # bytes one token streams: packed codes + scales of every projection,
-    # plus the activation vectors read and written (negligible)
-    weight_bytes = shape.weight_bytes()
-    vec_bytes = 2 * B * (shape.hidden * (4 * shape.num_layers + 1) + shape.vocab)
-    step_bytes = weight_bytes + vec_bytes
+    step_bytes = chain_step_bytes(shape, B)
 
     for _ in range(args.warmup):
         model.decode(x, logits, stream)
@@ -341,13 +355,7 @@ def run_ours(args, rank, world, local):
             "dtype": "f32",
             "precision": "int4 codes (group 32, fp16 scale, zero point 7), fp16 activations, fp32 accumulation",
             "data": "synthetic (seeded SplitMix64 weights and activations)",
-            "config": {"workload": f"{shape.name}-shaped decode chain: {shape.num_layers} layers x "
-                                   f"(QKV {shape.n_qkv}x{shape.hidden}, O {shape.hidden}x{shape.hidden}, "
-                                   f"gate_up {2 * shape.ffn}x{shape.hidden}, down {shape.hidden}x{shape.ffn}) "
-                                   f"+ LM head {shape.vocab}x{shape.hidden}, batch {B}",
-                       "batch": B, "bytes_per_token": step_bytes,
-                       "l2": "inputs larger than L2 (1.8+ GB of weights per step), no flush",
-                       "parallelism": "replicas" if world > 1 else "single GPU"},
+            "config": chain_config(shape, B, world),
             "hbm_gbs": step_bytes * args.steps / (total_ms_max / 1e3) / 1e9,
             "hbm_frac_of_nominal_8tbs": step_bytes * args.steps / (total_ms_max / 1e3) / 1e9 / NOMINAL_HBM_GBS,
             "roofline": {"bound": "hbm", "kernel": kernel_name, "achieved": achieved, "peak": peak,
@@ -465,7 +473,8 @@ def run_attn_reference(args, rank, world):
     value = w.batch / statistics.mean(times)
     line = {"metric": ATTN_METRIC, "value": value, "unit": "sequences/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": 1e3 * statistics.mean(times), "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded SplitMix64 weights and activations)", "impl": "reference",
             "config": attn_config(w, 1),
             "cpu_baseline": {"value": value, "unit": "sequences/s", "cores": 1, "kind": "oracle",
                              "sample": f"each step: shortest sequences first for about {step_s:.1f} s of oracle "
@@ -621,7 +630,8 @@ def run_prefill_reference(args, rank, world):
     value = done / sum(times) / 1e12
     line = {"metric": PREFILL_METRIC, "value": value, "unit": "TFLOP/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": 1e3 * flops_step / (value * 1e12), "higher_is_better": True,
-            "scaling": "weak", "vs_baseline": None, "dtype": "f64", "data": "synthetic", "impl": "reference",
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded SplitMix64 weights and activations)", "impl": "reference",
             "config": {"workload": f"prefill-3b: QKV, O, gate_up, down of one 3B-shaped layer over {M} tokens"},
             "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": 1, "kind": "oracle",
                              "sample": "a few rows of every projection against up to 64 tokens, single-threaded fp64 C oracle"},

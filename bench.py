@@ -474,7 +474,7 @@ def run_attn_reference(args, rank, world):
     line = {"metric": ATTN_METRIC, "value": value, "unit": "sequences/s", "n_gpus": world, "steps": args.steps,
             "warmup": args.warmup, "ms_per_step": 1e3 * statistics.mean(times), "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64",
-            "data": "synthetic (seeded SplitMix64 weights and activations)", "impl": "reference",
+            "data": "synthetic (seeded sum4 keys, values and queries; random page tables)", "impl": "reference",
             "config": attn_config(w, 1),
             "cpu_baseline": {"value": value, "unit": "sequences/s", "cores": 1, "kind": "oracle",
                              "sample": f"each step: shortest sequences first for about {step_s:.1f} s of oracle "

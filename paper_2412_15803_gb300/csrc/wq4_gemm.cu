@@ -42,10 +42,10 @@ constexpr int kGDCol = 256;           // accumulator: TOK columns
 constexpr int kGT = 1024;             // transpose buffer: TOK tokens x 128 outputs fp16
 constexpr int kGTmemCols = 512;
 
-// Tile of TOK tokens (MMA N = 128 or 256).
+// Tile of TOK tokens (MMA N = 128, 192 or 256).
 template <int TOK>
 struct GCfg {
-    static constexpr int kSlots = TOK == 256 ? 4 : 6;
+    static constexpr int kSlots = TOK == 256 ? 4 : (TOK == 192 ? 5 : 6);
     static constexpr int kX = TOK * 64 * 2;                // activation block: TOK tokens x 64 K fp16
     static constexpr int kSlot = kX + kGCodes + kGScales;  // a multiple of 1024
     static constexpr int kRing = kGT + TOK * 128 * 2;
@@ -285,11 +285,28 @@ int gemm_attr()
     return rc;
 }
 
-// Token tile: 256 (measured: a 128-token tile costs well over half of a
-// 256-token one), 128 when the prompt has at most 128 tokens.
-int pick_tok(int M)
+// Token tile: the width whose grid rounds (tiles over the SMs, rounded up)
+// times its cost relative to a 256-token tile is least; a 128-token tile
+// costs well over half of a 256-token one, a 192-token tile more than 6/7 of
+// one (measured: 7 rounds of 192 ran slower than 6 of 256), so 0.6 and 0.9.
+// Ties go to the wider tile.  128 when the prompt has at most 128 tokens.
+int pick_tok(int N, int M, int sms)
 {
-    return M <= 128 ? 128 : 256;
+    if (M <= 128) return 128;
+    const int rt = (N + 127) / 128;
+    const int toks[3] = {256, 192, 128};
+    const double cost[3] = {1.0, 0.9, 0.6};
+    int best = 256;
+    double best_c = 1e300;
+    for (int i = 0; i < 3; ++i) {
+        const int64_t tiles = static_cast<int64_t>(rt) * ((M + toks[i] - 1) / toks[i]);
+        const double c = static_cast<double>((tiles + sms - 1) / sms) * cost[i];
+        if (c < best_c - 1e-9) {
+            best_c = c;
+            best = toks[i];
+        }
+    }
+    return best;
 }
 
 }  // namespace
@@ -311,8 +328,8 @@ extern "C" int wq4_gemm(const uint32_t* W_packed, const uint16_t* scales, const 
     int dev = 0;
     const DeviceInfo* di = current_device_info(&dev);
     if (!di) return WQ4_ERR_CUDA;
-    const int tok = pick_tok(M);
-    if ((tok == 256 ? gemm_attr<256>() : gemm_attr<128>()) != 0) return WQ4_ERR_CUDA;
+    const int tok = pick_tok(N, M, di->sm_count);
+    if ((tok == 256 ? gemm_attr<256>() : tok == 192 ? gemm_attr<192>() : gemm_attr<128>()) != 0) return WQ4_ERR_CUDA;
     CUtensorMap mc, ms, mx;
     if (!encode_tensor_map_2d(&mc, CU_TENSOR_MAP_DATA_TYPE_UINT8, W_packed, static_cast<uint64_t>(K) / 2,
                               static_cast<uint64_t>(N), static_cast<uint64_t>(K) / 2, 32, 64,
@@ -337,6 +354,8 @@ extern "C" int wq4_gemm(const uint32_t* W_packed, const uint16_t* scales, const 
     const int grid = static_cast<int>(tiles < di->sm_count ? tiles : di->sm_count);
     if (tok == 256)
         gemm_kernel<256><<<grid, kGThreads, GCfg<256>::kSmem, static_cast<cudaStream_t>(stream)>>>(mc, ms, mx, a);
+    else if (tok == 192)
+        gemm_kernel<192><<<grid, kGThreads, GCfg<192>::kSmem, static_cast<cudaStream_t>(stream)>>>(mc, ms, mx, a);
     else
         gemm_kernel<128><<<grid, kGThreads, GCfg<128>::kSmem, static_cast<cudaStream_t>(stream)>>>(mc, ms, mx, a);
     return cudaGetLastError() == cudaSuccess ? WQ4_OK : WQ4_ERR_CUDA;

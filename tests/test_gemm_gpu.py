@@ -45,6 +45,20 @@ def test_gemm_parity(N, K, M):
     check(y, W, s, x)
 
 
+@pytest.mark.parametrize("M", [380, 500])
+def test_gemm_parity_wide_token_tiles(M):
+    """76 row tiles (9728 rows): on a 152-SM GB300 the tile-width rule takes
+    192-token tiles for 380 tokens and 256-token tiles for 500 (both with a
+    ragged last token tile); every output computed, sampled rows checked."""
+    N, K = 9728, 256
+    W, s = synth.matrix(37, N, K)
+    x = synth.activations(38, M, K)
+    y = run_gemm(W, s, x, N, K, M)
+    rows = np.unique(np.concatenate([[0, 1, 127, 128, N - 1], np.random.default_rng(M).integers(0, N, 61)]))
+    check(y, W, s, x, rows)
+    assert not np.any(y == 0xFFFF)
+
+
 def test_gemm_full_size_sampled():
     """The 3B gate_up projection (16384 x 3072) over a 2048-token prompt, the
     benchmark's largest launch: every output computed, sampled rows (all

@@ -4,21 +4,22 @@
 //
 // Y[m][n] = fp16( sum_k x[m][k] * fp16((q(n,k) - 7) * s(n, k/32)) ), fp32 sums.
 //
-// A persistent grid walks (128 weight rows x 256 tokens) tiles, row tile
-// major so that the CTAs running at one time share a weight tile through L2.
-// Per 64-wide K chunk a producer warp brings the tile's codes and scales
-// (2-D tensor copies) and the 256 x 64 activation block (one 128-byte swizzled
-// box) into a 4-slot ring (small slots, so that copies stay in flight while
-// the MMAs of earlier chunks run); eight dequant warps write the 128 x 64
-// weights, dequantized to fp16 in natural K order, into one of three
-// 32-column A buffers in tensor memory (lane = weight row); one thread issues
-// 4 tcgen05.mma (kind::f16, M = 128, N = 256 tokens, K = 16: the tensor-core
-// rate, ~128 cycles each, so the dequant warps keep up) into a 256-column fp32
-// accumulator; four epilogue warps move a finished accumulator into a
-// shared-memory transpose buffer, release it, and store 256 tokens x 128
-// outputs with 16-byte stores while the next tile's MMAs run.  Every weight is
-// rounded to fp16 once (relative error <= 2^-11, accumulated in fp32): within
-// the library's accuracy contract.
+// A persistent grid walks (128 weight rows x T tokens) tiles, T = 128, 192 or
+// 256 chosen per call (pick_tok), row tile major so that the CTAs running at
+// one time share a weight tile through L2.  Per 64-wide K chunk a producer
+// warp brings the tile's codes and scales (2-D tensor copies) and the T x 64
+// activation block (one 128-byte swizzled box) into a ring of 4-6 slots
+// (small slots, so that copies stay in flight while the MMAs of earlier
+// chunks run); eight dequant warps write the 128 x 64 weights, dequantized to
+// fp16 in natural K order, into one of three 32-column A buffers in tensor
+// memory (lane = weight row); one thread issues 4 tcgen05.mma (kind::f16,
+// M = 128, N = T tokens, K = 16: at T = 256 the tensor-core rate, ~128 cycles
+// each, so the dequant warps keep up) into a T-column fp32 accumulator; four
+// epilogue warps move a finished accumulator into a shared-memory transpose
+// buffer, release it, and store T tokens x 128 outputs with 16-byte stores
+// while the next tile's MMAs run.  Every weight is rounded to fp16 once
+// (relative error <= 2^-11, accumulated in fp32): within the library's
+// accuracy contract.
 #include "wq4.h"
 #include "wq4_device.cuh"
 #include "wq4_host.h"

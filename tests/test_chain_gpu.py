@@ -101,9 +101,11 @@ def check_logits(model, logits, rows=None):
     within(logits[:, idx], y, A, "lm_head")
 
 
-@pytest.mark.parametrize("batch", [1, 2, 3, 4, 5, 8, 32])
+@pytest.mark.parametrize("batch", [1, 2, 3, 4, 5, 8, 13, 17, 32])
 def test_tiny_chain_every_stage_every_element(batch):
-    """Batch 1-4: the persistent kernel; 5-32: the graph of stage kernels."""
+    """Batch 1-2: the persistent kernel; 3-32: the graph of tensor-core stage
+    kernels (batch padded to 16 up to 16, else to 32; 13 and 17 leave a
+    partly padded group of four batch rows)."""
     model = DecodeModel(TINY, batch=batch, seed=batch)
     x = synth.activations(100 + batch, batch, TINY.hidden)
     logits = run(model, x)

@@ -208,6 +208,17 @@ def test_linearity_in_x_and_s():
     assert np.array_equal(y4, 4 * y1) and np.array_equal(A4, 4 * A1)
 
 
+def test_row_factors_scale_their_own_batch_row():
+    """Each batch row b takes its own factor r_b: with powers of two the
+    scaling is exact, so y(r)[b] = r_b y(1)[b] bit for bit."""
+    N, K, batch = 5, 128, 3
+    W, s, x = _random_case(N, K, batch, seed=9)
+    r = np.array([0.5, 4.0, 2.0 ** -3])
+    y, A, _ = oracle.gemv(W, s, x)
+    yr, Ar, _ = oracle.gemv(W, s, x, r=r)
+    assert np.array_equal(yr, r[:, None] * y) and np.array_equal(Ar, r[:, None] * A)
+
+
 @pytest.mark.parametrize("N,K,batch", [(1, 32, 1), (3, 32, 2), (4, 64, 1), (2, 64, 2), (4, 96, 3)])
 def test_brute_force_vs_dense_numpy(N, K, batch):
     W, s, x = _random_case(N, K, batch, seed=N * 100 + K + batch)
@@ -298,6 +309,31 @@ def test_chain_all_sevens_passes_the_normalised_input_through():
     for t in tr[:-1]:
         assert np.all(t["qkv"] & 0x7FFF == 0) and np.all(t["d"] & 0x7FFF == 0)
         assert np.array_equal(t["x2"], t["v"])          # o = d = 0: output = layer input
+
+
+def test_chain_gate_and_up_halves():
+    """SiLU acts on the gate half (rows [0, F)) and multiplies the up half
+    (rows [F, 2F)): with up rows weighting the input twice as much as the
+    gate rows (code 9, w = 2s, against code 8, w = s), m = silu(g) * 2g,
+    which silu(2g) * g does not match."""
+    H, F, batch, eps = 64, 64, 2, 1e-5
+    qg = np.full((2 * F, H), 7, np.uint8)
+    qg[np.arange(F), np.arange(F)] = 8          # gate row j: x1[j]
+    qg[F + np.arange(F), np.arange(F)] = 9      # up row j: 2 x1[j]
+    layers = [dict(qkv=_identity_like(2 * H, H), o=_identity_like(H, H),
+                   gate_up=(oracle.pack(qg), np.full((2 * F, H // 32), 0x3C00, np.uint16)),
+                   down=_identity_like(H, F))]
+    x = synth.activations(13, batch, H)
+    _, _, tr = ochain.token(x, layers, _identity_like(H, H), H, F, eps)
+    t = tr[0]
+    gu = t["gu"].view(np.float16).astype(np.float64)
+    g, up = gu[:, :F], gu[:, F:]
+    assert np.array_equal(up, 2 * g)            # exact: fp16 doubling
+    m = t["m"].view(np.float16).astype(np.float64)
+    expect = (g / (1.0 + np.exp(-g)) * up).astype(np.float16).astype(np.float64)
+    swapped = (up / (1.0 + np.exp(-up)) * g).astype(np.float16).astype(np.float64)
+    assert np.allclose(m, expect, rtol=2.0 ** -10, atol=2.0 ** -24)
+    assert not np.allclose(m, swapped, rtol=2.0 ** -8, atol=2.0 ** -20)
 
 
 def test_chain_wiring_with_identity_projections():

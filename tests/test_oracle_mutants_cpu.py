@@ -46,6 +46,10 @@ MUTANTS = [
     ("magnitude without abs", G, "mag += fabs(w * xv);", "mag += w * xv;", None),
     ("row factor not applied", G, "acc *= rb;", "(void)rb;", None),
     ("row factor of the first row", G, "double rb = r ? r[b] : 1.0;", "double rb = r ? r[0] : 1.0;", None),
+    ("magnitude without the row factor", G, "mag *= rb;", "(void)mag;", None),
+    ("last code of a row dropped", G, "            for (int k = 0; k < K; ++k) {\n                int q = wq4o_code",
+     "            for (int k = 0; k < K - 1; ++k) {\n                int q = wq4o_code", None),
+    ("fp16 output rounded through fp32", G, "wq4o_double_to_half(acc)", "wq4o_double_to_half((float)acc)", None),
     # chain glue
     ("RMS without eps", G, "sqrt(ss / (double)n + eps)", "sqrt(ss / (double)n)", None),
     ("RMS mean over n - 1", G, "sqrt(ss / (double)n + eps)", "sqrt(ss / (double)(n - 1) + eps)", None),
@@ -54,6 +58,8 @@ MUTANTS = [
     ("residual subtracts", G, "wq4o_half_to_double(a[i]) + wq4o_half_to_double(b[i])",
      "wq4o_half_to_double(a[i]) - wq4o_half_to_double(b[i])", None),
     # chain composition
+    ("attention stand-in from the key block", CH, "a = np.ascontiguousarray(qkv[:, :H])",
+     "a = np.ascontiguousarray(qkv[:, H:2 * H])", None),
     ("QKV without its RMS factor", CH, 'gemv(*w["qkv"], u, r1)', 'gemv(*w["qkv"], u)', None),
     ("O with the layer input's factor", CH, 'gemv(*w["o"], a, r2)', 'gemv(*w["o"], a, r1)', None),
     ("residual from u instead of v", CH, "x1 = add_fp16(v, o)", "x1 = add_fp16(u, o)", None),
@@ -64,6 +70,8 @@ MUTANTS = [
     ("second residual from v", CH, "x2 = add_fp16(x1, d)", "x2 = add_fp16(v, d)", None),
     ("LM head without its RMS factor", CH, "gemv(*lm_head, x, rf)", "gemv(*lm_head, x)", None),
     # attention
+    ("query of the kv head", AT, "const uint16_t* qj = q + (int64_t)b * q_stride + (int64_t)j * head_dim;",
+     "const uint16_t* qj = q + (int64_t)b * q_stride + (int64_t)h * head_dim;", None),
     ("kv head by modulo", AT, "const int h = j / G;", "const int h = j % n_kv_heads;", None),
     ("scale dropped in the weights", AT, "exp(scale * dot - m)", "exp(dot - m)", None),
     ("no max shift", AT, "exp(scale * dot - m)", "exp(scale * dot)", None),

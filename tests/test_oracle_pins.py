@@ -208,6 +208,24 @@ def test_linearity_in_x_and_s():
     assert np.array_equal(y4, 4 * y1) and np.array_equal(A4, 4 * A1)
 
 
+def test_fp16_output_is_one_rounding_of_the_fp64_sum():
+    """y16 = fp16_RNE(y) with y the exact fp64 sum, not a rounding through
+    fp32: y = 1 + 2^-11 + 2^-24 (codes 8, scale 1, x = 1, 2^-11, 2^-24; exact
+    in fp64) lies just above the fp16 tie between 1 and 1 + 2^-10, so it
+    rounds up to 0x3C01; rounded to fp32 first it would become the tie itself
+    (2^-24 is half an fp32 ulp at 1) and then round to even, 0x3C00."""
+    K = 32
+    q = np.full((1, K), 7, np.uint8)
+    q[0, :3] = 8
+    W = oracle.pack(q)
+    s = np.full((1, 1), 0x3C00, np.uint16)
+    x = np.zeros((1, K), np.uint16)
+    x[0, :3] = np.array([1.0, 2.0 ** -11, 2.0 ** -24]).astype(np.float16).view(np.uint16)
+    y, A, y16 = oracle.gemv(W, s, x)
+    assert y[0, 0] == 1.0 + 2.0 ** -11 + 2.0 ** -24 and A[0, 0] == y[0, 0]
+    assert y16[0, 0] == 0x3C01
+
+
 def test_row_factors_scale_their_own_batch_row():
     """Each batch row b takes its own factor r_b: with powers of two the
     scaling is exact, so y(r)[b] = r_b y(1)[b] bit for bit."""

@@ -97,6 +97,22 @@ def test_equal_scores_give_the_mean():
             assert np.array_equal(o[b, j], mean)
 
 
+def test_fp16_output_is_one_rounding_of_the_fp64_value():
+    """o16 = fp16_RNE(o) of the fp64 value, rounded once: four tokens with
+    equal scores (q = 0) and values 4, 2^-9, 2^-22, 0 in dimension 0 give
+    o = 1 + 2^-11 + 2^-24 exactly, just above the fp16 tie between 1 and
+    1 + 2^-10, so 0x3C01; a rounding through fp32 first would land on the
+    tie and round to even (0x3C00)."""
+    D, P = 128, 16
+    k = synth.sum4_fp16(5, 9, 0, P * D).reshape(1, 1, P, D)
+    v = np.zeros((1, 1, P, D), np.uint16)
+    v[0, 0, :4, 0] = _f16(np.array([4.0, 2.0 ** -9, 2.0 ** -22, 0.0]))
+    q = np.zeros((1, D), np.uint16)
+    o, _, o16 = oracle.paged_attention(q, k, v, np.array([[0]]), np.array([4]), 0.1, 1)
+    assert o[0, 0, 0] == 1.0 + 2.0 ** -11 + 2.0 ** -24
+    assert o16[0, 0, 0] == 0x3C01
+
+
 def test_two_tokens_closed_form():
     """Scores a and 0: o = (e^a v0 + v1) / (e^a + 1)."""
     D, P = 128, 16

@@ -72,6 +72,9 @@ MUTANTS = [
     # attention
     ("query of the kv head", AT, "const uint16_t* qj = q + (int64_t)b * q_stride + (int64_t)j * head_dim;",
      "const uint16_t* qj = q + (int64_t)b * q_stride + (int64_t)h * head_dim;", None),
+    ("attention output rounded through fp32", AT, "o16j[d] = wq4o_double_to_half(oj[d]);",
+     "o16j[d] = wq4o_double_to_half((float)oj[d]);", None),
+    ("maximum of the unscaled scores", AT, "const double st = scale * dot;", "const double st = dot;", None),
     ("kv head by modulo", AT, "const int h = j / G;", "const int h = j % n_kv_heads;", None),
     ("scale dropped in the weights", AT, "exp(scale * dot - m)", "exp(dot - m)", None),
     ("no max shift", AT, "exp(scale * dot - m)", "exp(scale * dot)", None),

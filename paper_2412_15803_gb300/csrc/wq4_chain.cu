@@ -5,8 +5,8 @@
 // Structure (GB300-first; the paper's WebGPU engine launches one compiled
 // kernel per operator, Section 2.3):
 //  * One CTA per SM, co-resident (cooperative launch).  Each CTA owns a fixed
-//    slice of the output rows of every stage (QKV, O, gate_up, down per layer,
-//    then the LM head).
+//    slice of the output words (two fp16 outputs each) of every stage (QKV, O,
+//    gate_up, down per layer, then the LM head).
 //  * A producer warp walks the CTA's slices of ALL stages in order and streams
 //    their packed weights through a ring of shared-memory slots with 1-D bulk
 //    copies (TMA) and mbarriers.  Weights do not depend on activations, so the
@@ -16,10 +16,19 @@
 //    computes the same factor in the same order (identical bits everywhere),
 //    applies it as a row factor of its projection, and publishes its slice of
 //    the normalised vector for the O stage's residual add.
-//  * Consumer warps stage each stage's input vector in shared memory, take
-//    two-row items (four rows for gate_up: gate j, j+1 and up j, j+1)
-//    round-robin, unpack in registers, accumulate in fp32, and apply the
-//    fused epilogue (RMS factor, residual add, SiLU(gate) * up).
+//  * Work items are (superpair, K part): a superpair is two row pairs (two
+//    output words, or gate_up's gate and up rows of one word; one row pair
+//    for very long rows), and K is cut into q equal parts chosen per stage
+//    so that the 15 consumer warps, taking items round-robin in ring order,
+//    get nearly equal work.  An item is a run of units of 256 codes; per row
+//    pair a unit is two mma.sync m16n8k16 on the legacy tensor path: A holds
+//    exact fp16 (q - 7) of 16 (row, group) combinations (two rows x eight
+//    groups of 32 codes), B holds the eight groups' activations as its eight
+//    columns (loaded once for both pairs), and the group scales multiply the
+//    diagonal of the fp32 result on the CUDA cores (no fp16 rounding of a
+//    weight or a product).  After the stage, the parts of every word are
+//    added in part order and the fused epilogue (RMS factor, residual add,
+//    SiLU(gate) * up) publishes the words.
 //  * Stage outputs travel between CTAs as 8-byte words {2 x fp16 data, 32-bit
 //    token epoch} written with single 64-bit stores; a consumer polls the
 //    words of its input until every epoch matches.  No grid-wide barrier and
@@ -58,27 +67,23 @@ constexpr int kMaxChainBatch = 2;   // larger batches take the tensor-core graph
 // item.  Only warps that own items of a chunk touch its barriers.
 constexpr uint32_t kSlotRelease = 1024;
 // Shared-memory header: mbarriers (kFullBars full, kChainMaxSlots empty) |
-// RMS partial sums | epoch | the residual
-// words of the CTA's rows (O and down stages); then the staged input vector,
-// then the weight ring.
+// RMS partial sums | epoch | stage table | warp table | residual words of the
+// CTA's words (O and down stages) | per-item partial row sums; then the
+// staged input vector, then the weight ring.
 constexpr int kHdrRed = 512;                 // float red[kMaxChainBatch][16]: per-warp sums of squares
 static_assert(8 * (kFullBars + kChainMaxSlots) <= kHdrRed, "mbarriers overlap the header");
 constexpr int kHdrEpoch = 768;               // uint32 epoch, then int vw0, vw1 (the CTA's slice of v)
 constexpr int kHdrInfo = 784;                // StageInfo info[5], one per stage type
-constexpr int kHdrWofs = 944;                // uint8 wofs[5][16]: a warp's first chunk within a stage
-constexpr int kHdrRes = 1024;                // uint32 res[kMaxResWords]: prefetched residual words
-constexpr int kMaxResWords = 1024;
-__host__ __device__ constexpr int chain_header_bytes(int, int)
-{
-    return kHdrRes + 4 * kMaxResWords;
-}
+constexpr int kHdrRes = 1152;                // uint32 res[kMaxResWords]: prefetched residual words
+constexpr int kMaxResWords = 256;
+constexpr int kHdrPart = kHdrRes + 4 * kMaxResWords;   // float4 part[superpair][K part][B]: row sums
+constexpr int kMaxPart = 384;
+constexpr int kChainHeader = kHdrPart + 16 * kMaxPart;
+static_assert(kHdrPart % 16 == 0 && kChainHeader % 128 == 0, "header alignment");
 
 // Consumer warps per CTA: with the producer warp, 16 warps (128 registers a
 // thread).
-template <int B>
-struct ChainWarps {
-    static constexpr int NW = 15;
-};
+constexpr int kChainWarps = 15;
 
 enum StageType { kQKV = 0, kO = 1, kGU = 2, kDOWN = 3, kLM = 4 };
 
@@ -91,6 +96,8 @@ struct ChainParams {
     const DevMat* mats;  // [4L + 1]: per layer qkv, o, gate_up, down; then lm_head
     int L, H, F, Nqkv, V;
     float eps;
+    int q[5];            // K parts per superpair, per stage type (divides K / 256)
+    int spw[5];          // words per superpair, per stage type (gate_up: 1)
     const uint16_t* x;   // [B][H] token input
     uint16_t* logits;    // [B][V]
     uint32_t* seq;       // token counter (workspace header)
@@ -101,6 +108,10 @@ struct ChainParams {
     uint64_t* llM;       // [L][B][F/2]   silu(gate) * up
     uint64_t* llX;       // [L+1][B][H/2] layer outputs (index 0 unused)
     uint64_t* llV;       // [L][B][H/2]   RMS-normalised layer inputs (residual of O)
+    // Every flagged vector is written twice (replica 1 at llX + rep.X etc., in
+    // uint64 words); CTA c reads replica c & 1, which halves the number of
+    // CTAs polling each line of a stage boundary.
+    struct { uint32_t A, X1, M, X, V; } rep;
     uint16_t* pV;        // [L+1][B][H]   RMS-normalised layer inputs; [L] feeds the LM head
     uint16_t* pX2;       // [L][B][H]     layer outputs
     uint16_t* pQKV;      // [L][B][Nqkv]
@@ -116,8 +127,11 @@ struct ChainParams {
     uint32_t* err;
 };
 
+// One stage: N output rows of K codes, `words` output words of rpw rows each
+// (gate_up: gate rows 2w, 2w+1 and up rows F+2w, F+2w+1; the LM head's last
+// word may hold one row).
 struct Stage {
-    int type, layer, N, K, rpi, items;
+    int type, layer, N, K, words, rpw;
     const uint32_t* W;
     const uint16_t* s;
 };
@@ -126,15 +140,15 @@ __device__ __forceinline__ Stage stage_at(const ChainParams& p, int st)
 {
     Stage g;
     if (st == 4 * p.L) {
-        g.type = kLM; g.layer = p.L; g.N = p.V; g.K = p.H; g.rpi = 4; g.items = (p.V + 3) / 4;
+        g.type = kLM; g.layer = p.L; g.N = p.V; g.K = p.H; g.rpw = 2; g.words = (p.V + 1) / 2;
     } else {
         g.layer = st >> 2;
         g.type = st & 3;
         switch (g.type) {
-            case kQKV: g.N = p.Nqkv; g.K = p.H; g.rpi = 2; g.items = p.Nqkv / 2; break;
-            case kO: g.N = p.H; g.K = p.H; g.rpi = 2; g.items = p.H / 2; break;
-            case kGU: g.N = 2 * p.F; g.K = p.H; g.rpi = 4; g.items = p.F / 2; break;
-            default: g.N = p.H; g.K = p.F; g.rpi = 2; g.items = p.H / 2; break;
+            case kQKV: g.N = p.Nqkv; g.K = p.H; g.rpw = 2; g.words = p.Nqkv / 2; break;
+            case kO: g.N = p.H; g.K = p.H; g.rpw = 2; g.words = p.H / 2; break;
+            case kGU: g.N = 2 * p.F; g.K = p.H; g.rpw = 4; g.words = p.F / 2; break;
+            default: g.N = p.H; g.K = p.F; g.rpw = 2; g.words = p.H / 2; break;
         }
     }
     g.W = p.mats[st].W;
@@ -142,22 +156,23 @@ __device__ __forceinline__ Stage stage_at(const ChainParams& p, int st)
     return g;
 }
 
-// Byte layout of one chunk (items [ia, ib) of a stage) inside a slot.
+// Byte layout of one chunk (words [wa, wb) of a stage) inside a slot: the
+// chunk's rows (gate_up: its gate rows, then its up rows), then their scales.
 struct ChunkLayout {
     int nrows;          // rows in the chunk (both halves for gate_up)
     int nh;             // rows per half (gate_up) / nrows otherwise
     uint32_t codes_bytes, scale_bytes;
 };
 
-__device__ __forceinline__ ChunkLayout chunk_layout(const Stage& g, int ia, int ib)
+__device__ __forceinline__ ChunkLayout chunk_layout(const Stage& g, int wa, int wb)
 {
     ChunkLayout c;
     if (g.type == kGU) {
-        c.nh = 2 * (ib - ia);
+        c.nh = 2 * (wb - wa);
         c.nrows = 2 * c.nh;
     } else {
-        const int r1 = min(g.rpi * ib, g.N);
-        c.nrows = r1 - g.rpi * ia;
+        const int r1 = min(2 * wb, g.N);
+        c.nrows = r1 - 2 * wa;
         c.nh = c.nrows;
     }
     c.codes_bytes = static_cast<uint32_t>(c.nrows) * (g.K / 2);
@@ -165,27 +180,38 @@ __device__ __forceinline__ ChunkLayout chunk_layout(const Stage& g, int ia, int 
     return c;
 }
 
-// What one CTA does in every stage of one type, computed once per launch so
-// that no stage pays for integer divisions: items [i0, i1), items per ring
-// slot, the number of chunks, and that number modulo the slot and barrier
-// counts (flip: parity changes of the barrier ring beyond the wrap).
+// What one CTA does in every stage of one type, computed once per launch:
+// its words [w0, w0 + nwords) = superpairs [0, nsp), words per chunk (a
+// multiple of the words per superpair, spw), the number of chunks and that
+// number modulo the slot and barrier counts (flip: parity changes of the
+// barrier ring beyond the wrap), units (256 codes) per superpair J, K parts q
+// and units per part upp.  Items are (superpair i / q, part i % q).
 struct StageInfo {
-    int i0, i1, ips, nchunks, nmod_slots, nmod_bars, flip, pad;
+    int w0, nwords, wps, nchunks, nmod_slots, nmod_bars, flip, J, spw, q, upp, nsp;
 };
-static_assert(kHdrInfo + 5 * sizeof(StageInfo) <= kHdrWofs, "stage table overlaps the header");
-static_assert(kHdrWofs + 5 * 16 <= kHdrRes, "warp table overlaps the header");
+static_assert(kHdrInfo + 5 * sizeof(StageInfo) <= kHdrRes, "stage table overlaps the header");
 
-__device__ __forceinline__ void cta_items(int items, int* i0, int* i1)
+__device__ __forceinline__ void cta_words(int words, int* w0, int* w1)
 {
-    *i0 = static_cast<int>(static_cast<int64_t>(blockIdx.x) * items / gridDim.x);
-    *i1 = static_cast<int>(static_cast<int64_t>(blockIdx.x + 1) * items / gridDim.x);
+    *w0 = static_cast<int>(static_cast<int64_t>(blockIdx.x) * words / gridDim.x);
+    *w1 = static_cast<int>(static_cast<int64_t>(blockIdx.x + 1) * words / gridDim.x);
 }
 
-__device__ __forceinline__ int items_per_slot(const ChainParams& p, const Stage& g)
+// Words per superpair (the plan's choice: 2, or 1 for large words; gate_up's
+// word already holds two row pairs).
+__device__ __forceinline__ int words_per_superpair(const ChainParams& p, const Stage& g)
 {
-    const uint32_t item_bytes = static_cast<uint32_t>(g.rpi) * (g.K / 2 + g.K / 16);
-    const int ips = static_cast<int>(p.slot_bytes / item_bytes);
-    return ips < 1 ? 1 : ips;
+    return p.spw[g.type];
+}
+
+// Words per ring slot: a whole number of superpairs (the plan's slot holds at
+// least one).
+__device__ __forceinline__ int words_per_slot(const ChainParams& p, const Stage& g)
+{
+    const uint32_t word_bytes = static_cast<uint32_t>(g.rpw) * (g.K / 2 + g.K / 16);
+    const int spw = words_per_superpair(p, g);
+    const int wps = static_cast<int>(p.slot_bytes / word_bytes) / spw * spw;
+    return wps < spw ? spw : wps;
 }
 
 // A representative stage of each type (layer 0, or the LM head).
@@ -194,12 +220,43 @@ __device__ __forceinline__ int stage_of_type(const ChainParams& p, int t)
     return t == kLM ? 4 * p.L : t;
 }
 
+// Exact floor(n / d) for 0 <= n, d < 2^24 from a float reciprocal: the
+// product is within 2^-9 of n / d for the quotients used here (< 2^14), so
+// one correction step gives the floor.  No integer division on the path.
+struct FDiv {
+    float r;
+    int d;
+};
+__device__ __forceinline__ FDiv fdiv_make(int d)
+{
+    FDiv f;
+    f.d = d;
+    f.r = __frcp_rn(static_cast<float>(d));
+    return f;
+}
+__device__ __forceinline__ int fdiv(int n, const FDiv& f)
+{
+    int q = __float2int_rz(static_cast<float>(n) * f.r);
+    if (q * f.d > n) --q;
+    else if ((q + 1) * f.d <= n) ++q;
+    return q;
+}
+
+
+
 // ------------------------------------------------------- flagged words --
 
 __device__ __forceinline__ void ll_store(uint64_t* addr, uint32_t data, uint32_t epoch)
 {
     const uint64_t v = (static_cast<uint64_t>(epoch) << 32) | data;
     asm volatile("st.relaxed.gpu.global.b64 [%0], %1;" ::"l"(addr), "l"(v) : "memory");
+}
+
+// A flagged word into both replicas of its vector (replica 1 `rep` words on).
+__device__ __forceinline__ void ll_store2(uint64_t* addr, uint32_t rep, uint32_t data, uint32_t epoch)
+{
+    ll_store(addr, data, epoch);
+    ll_store(addr + rep, data, epoch);
 }
 
 __device__ __forceinline__ void ll_load2_raw(const uint64_t* addr, uint64_t& a, uint64_t& b)
@@ -279,16 +336,6 @@ __device__ __forceinline__ uint32_t pack2(uint16_t a, uint16_t b)
 // correctly rounded fp16 sum (fp32 carries more than 2 * 11 + 2 bits).
 __device__ __forceinline__ uint16_t add_h(float a, float b) { return float_to_half_bits(a + b); }
 
-// fp16(r * v_i) for the 8 fp16 values of a chunk
-__device__ __forceinline__ uint4 scale8(uint4 v, float r)
-{
-    uint32_t w[4] = {v.x, v.y, v.z, v.w};
-#pragma unroll
-    for (int i = 0; i < 4; ++i)
-        w[i] = pack2(float_to_half_bits(r * lo_f(w[i])), float_to_half_bits(r * hi_f(w[i])));
-    return make_uint4(w[0], w[1], w[2], w[3]);
-}
-
 __device__ __forceinline__ float sum8_sq(uint4 v)
 {
     const uint32_t w[4] = {v.x, v.y, v.z, v.w};
@@ -302,86 +349,109 @@ __device__ __forceinline__ float sum8_sq(uint4 v)
     return s;
 }
 
+// Eight consecutive activations x0..x7 (four words of two) in the order the
+// MMA's B fragment takes them: (x0, x4), (x1, x5), (x2, x6), (x3, x7) -- the
+// pairing of unpack_word's outputs.
+__device__ __forceinline__ uint4 pair_permute(uint4 v)
+{
+    return make_uint4(__byte_perm(v.x, v.z, 0x5410), __byte_perm(v.x, v.z, 0x7632), __byte_perm(v.y, v.w, 0x5410),
+                      __byte_perm(v.y, v.w, 0x7632));
+}
+
+// Word w (activations 2w, 2w+1) of a pair-permuted row staged at xw (uint32).
+__device__ __forceinline__ uint32_t permuted_word(const uint32_t* xw, int w)
+{
+    const int c = w >> 2, i = w & 3;
+    const uint32_t* u = xw + 4 * c + ((i & 1) ? 2 : 0);
+    return (i & 2) ? __byte_perm(u[0], u[1], 0x7632) : __byte_perm(u[0], u[1], 0x5410);
+}
+
 // ---------------------------------------------------------- the kernel --
 
-// One group (32 codes) of every row of an item against the staged
-// activations.  crow/srow point at the lane's first group of each row, xl at
-// the lane's first group of activation row 0; `off` is the group offset
-// (a multiple of 32, so the lane's chunk swizzle `sw` does not change).  The
-// activations are loaded once and used for every row; each row's 32 products
-// go into two 16-long fp32 chains before the group's scale is applied.
-template <int B, int RPI>
-__device__ __forceinline__ void group_rows_dot(const uint4* const crow[4], const uint16_t* const srow[4],
-                                               const uint4* xl, int cpr, int sw, int off, float acc[4][B])
+// The units of one item for NP row pairs (smem code rows ca[], cb[], scale
+// rows sa[], sb[]): for each group set j (256 codes) in [j0, j1), two
+// m16n8k16 MMAs per pair over its 16 (row, group) combinations and the eight
+// groups' activations (loaded once for all pairs), then the scaled diagonal
+// into acc[pair][b] (lanes 0, 5, 10, 15 hold row a's partial sums, lanes 16,
+// 21, 26, 31 row b's).
+//
+// Lane (g, c) = (lane >> 2, lane & 3).  A row m of the MMA is (row, group
+// 8j + sigma): m = g < 4: (a, 2g); m = g + 8 < 12: (a, 2g + 1); m = g >= 4:
+// (b, 2g - 7); m = g + 8 >= 12: (b, 2g - 8).  The pairing of rows a and b with
+// odd and even groups puts the eight 16-byte rows of each ldmatrix on
+// distinct bank quads.  B column sigma holds group 8j + sigma of x, so the
+// wanted sums sit on the diagonal D[m][sigma(m)]: lanes 5g (g < 4) hold them
+// in d0 (even group) and d3 (odd group), lanes 5g - 4 (g >= 4) in d2 and d1.
+template <int B, int NP>
+__device__ __forceinline__ void item_units(const uint32_t (&ca)[NP], const uint32_t (&cb)[NP], const uint32_t (&sa)[NP],
+                                           const uint32_t (&sb)[NP], uint32_t xs, int cpr, int j0, int j1,
+                                           float (&acc)[NP][B])
 {
-    uint4 xv[B][4];
+    const int lane = threadIdx.x & 31;
+    const int g = lane >> 2, c = lane & 3;
+    const bool hi = g >= 4;
+    // this lane's ldmatrix row address: matrix lane >> 3 (0: A rows g, 1: A rows g + 8)
+    const int t = lane & 7, mi = (lane >> 3) & 1;
+    const int goff = (t < 4) ? (2 * t + mi) : (2 * (t - 4) + 1 - mi);
+    uint32_t lb[NP], sbs[NP];
 #pragma unroll
-    for (int b = 0; b < B; ++b)
+    for (int pr = 0; pr < NP; ++pr) {
+        lb[pr] = ((t < 4) ? ca[pr] : cb[pr]) + 16 * goff;
+        sbs[pr] = (hi ? sb[pr] : sa[pr]) + 4 * c;
+    }
+    const uint32_t xbase = xs + 16 * lane;
+    const float zero[4] = {0.f, 0.f, 0.f, 0.f};
+#pragma unroll(NP == 1 ? 2 : 1)
+    for (int j = j0; j < j1; ++j) {
+        uint4 xv[B];
 #pragma unroll
-        for (int j = 0; j < 4; ++j) xv[b][j] = xl[b * cpr + 4 * off + (j ^ sw)];
+        for (int b = 0; b < B; ++b) xv[b] = lds_v4(xbase + 16 * (b * cpr + 32 * j));
+        uint32_t r0[NP], r1[NP], sw[NP];
 #pragma unroll
-    for (int r = 0; r < RPI; ++r) {
-        const uint4 cw = crow[r][off];
-        const float sc = half_bits_to_float(srow[r][off]);
-        uint32_t q[16];
-        unpack_word(cw.x, q + 0);
-        unpack_word(cw.y, q + 4);
-        unpack_word(cw.z, q + 8);
-        unpack_word(cw.w, q + 12);
+        for (int pr = 0; pr < NP; ++pr) {
+            ldsm_x2(lb[pr] + 128 * j, r0[pr], r1[pr]);
+            sw[pr] = lds_u32(sbs[pr] + 16 * j);
+        }
 #pragma unroll
-        for (int b = 0; b < B; ++b) {
-            const float a01 = fma8(q + 4, xv[b][1], fma8(q + 0, xv[b][0], 0.f));
-            const float a23 = fma8(q + 12, xv[b][3], fma8(q + 8, xv[b][2], 0.f));
-            acc[r][b] = fmaf(sc, a01 + a23, acc[r][b]);
+        for (int pr = 0; pr < NP; ++pr) {
+            uint32_t pa[4], pb[4];
+            unpack_word(r0[pr], pa);
+            unpack_word(r1[pr], pb);
+            const float se = lo_f(sw[pr]), so = hi_f(sw[pr]);
+#pragma unroll
+            for (int b = 0; b < B; ++b) {
+                float d[4];
+                mma_16816(d, pa[0], pb[0], pa[1], pb[1], xv[b].x, xv[b].y, zero);
+                mma_16816(d, pa[2], pb[2], pa[3], pb[3], xv[b].z, xv[b].w, d);
+                const float ve = hi ? d[2] : d[0];
+                const float vo = hi ? d[1] : d[3];
+                acc[pr][b] = fmaf(se, ve, fmaf(so, vo, acc[pr][b]));
+            }
         }
     }
 }
 
-// Every group of the item's rows: lane l takes groups l + 32 i.  Rows of 96,
-// 128 or 256 groups (K = 3072, 4096, 8192) run fully unrolled (all loads of
-// the item can be issued ahead of its arithmetic); other lengths take a loop
-// and a tail.
-template <int B, int RPI>
-__device__ __forceinline__ void item_dot(const uint4* const crow[4], const uint16_t* const srow[4],
-                                         const uint4* xl, int cpr, int gpr, int lane, float acc[4][B])
+// Row sums of a row pair from item_units: lane 0 gets row a, lane 16 row b.
+__device__ __forceinline__ float pair_reduce(float v)
 {
-    const int sw = (lane >> 1) & 3;
-    switch (gpr) {
-        case 96:
-#pragma unroll
-            for (int i = 0; i < 3; ++i) group_rows_dot<B, RPI>(crow, srow, xl, cpr, sw, 32 * i, acc);
-            return;
-        case 128:
-#pragma unroll
-            for (int i = 0; i < 4; ++i) group_rows_dot<B, RPI>(crow, srow, xl, cpr, sw, 32 * i, acc);
-            return;
-        case 256:
-#pragma unroll
-            for (int i = 0; i < 8; ++i) group_rows_dot<B, RPI>(crow, srow, xl, cpr, sw, 32 * i, acc);
-            return;
-        default: {
-            const int full = gpr >> 5;
-#pragma unroll 2
-            for (int i = 0; i < full; ++i) group_rows_dot<B, RPI>(crow, srow, xl, cpr, sw, 32 * i, acc);
-            if (lane < (gpr & 31)) group_rows_dot<B, RPI>(crow, srow, xl, cpr, sw, 32 * full, acc);
-        }
-    }
+    v += __shfl_down_sync(0xffffffffu, v, 5);
+    v += __shfl_down_sync(0xffffffffu, v, 10);
+    return v;
 }
 
-// Fused epilogue of one item for batch row b: v0..v3 are the item's row sums
-// (rows 2it, 2it+1; gate_up: gate 2it, 2it+1 then up 2it, 2it+1; LM head:
-// rows 4it .. 4it+3); resw is
-// the item's residual word (O: the normalised layer input, down: x + o).
+// Fused epilogue of one word w for batch row b: v0..v3 are its row sums (rows
+// 2w, 2w+1; gate_up: gate 2w, 2w+1 then up 2w, 2w+1; LM head: rows 2w, 2w+1);
+// resw is the word's residual (O: the normalised layer input, down: x + o).
 template <int B>
-__device__ __forceinline__ void item_epilogue(const ChainParams& p, const Stage& g, int it, int b, float v0,
-                                              float v1, float v2, float v3, float rf, uint32_t resw, uint32_t epoch)
+__device__ __forceinline__ void word_epilogue(const ChainParams& p, const Stage& g, int w, int b, float v0, float v1,
+                                              float v2, float v3, float rf, uint32_t resw, uint32_t epoch)
 {
     const int H = p.H, F = p.F, l = g.layer;
-    const int n = 2 * it;
+    const int n = 2 * w;
     if (g.type == kQKV) {
-        const uint32_t w = pack2(float_to_half_bits(rf * v0), float_to_half_bits(rf * v1));
-        *reinterpret_cast<uint32_t*>(p.pQKV + (static_cast<size_t>(l) * B + b) * p.Nqkv + n) = w;
-        if (n < H) ll_store(p.llA + (static_cast<size_t>(l) * B + b) * (H / 2) + n / 2, w, epoch);
+        const uint32_t wd = pack2(float_to_half_bits(rf * v0), float_to_half_bits(rf * v1));
+        *reinterpret_cast<uint32_t*>(p.pQKV + (static_cast<size_t>(l) * B + b) * p.Nqkv + n) = wd;
+        if (n < H) ll_store2(p.llA + (static_cast<size_t>(l) * B + b) * (H / 2) + w, p.rep.A, wd, epoch);
     } else if (g.type == kO) {
         const uint16_t o0 = float_to_half_bits(rf * v0);
         const uint16_t o1 = float_to_half_bits(rf * v1);
@@ -389,9 +459,8 @@ __device__ __forceinline__ void item_epilogue(const ChainParams& p, const Stage&
         const size_t off = (static_cast<size_t>(l) * B + b) * H + n;
         *reinterpret_cast<uint32_t*>(p.pO + off) = pack2(o0, o1);
         *reinterpret_cast<uint32_t*>(p.pX1 + off) = x1;
-        ll_store(p.llX1 + (static_cast<size_t>(l) * B + b) * (H / 2) + n / 2, x1, epoch);
+        ll_store2(p.llX1 + (static_cast<size_t>(l) * B + b) * (H / 2) + w, p.rep.X1, x1, epoch);
     } else if (g.type == kGU) {
-        const int j = n;  // gate rows j, j+1 and up rows F+j, F+j+1
         const uint16_t g0 = float_to_half_bits(rf * v0);
         const uint16_t g1 = float_to_half_bits(rf * v1);
         const uint16_t u0 = float_to_half_bits(rf * v2);
@@ -400,26 +469,22 @@ __device__ __forceinline__ void item_epilogue(const ChainParams& p, const Stage&
         const uint16_t m0 = float_to_half_bits(gf0 / (1.f + expf(-gf0)) * half_bits_to_float(u0));
         const uint16_t m1 = float_to_half_bits(gf1 / (1.f + expf(-gf1)) * half_bits_to_float(u1));
         const size_t gu = (static_cast<size_t>(l) * B + b) * (2 * F);
-        *reinterpret_cast<uint32_t*>(p.pGU + gu + j) = pack2(g0, g1);
-        *reinterpret_cast<uint32_t*>(p.pGU + gu + F + j) = pack2(u0, u1);
+        *reinterpret_cast<uint32_t*>(p.pGU + gu + n) = pack2(g0, g1);
+        *reinterpret_cast<uint32_t*>(p.pGU + gu + F + n) = pack2(u0, u1);
         const uint32_t mw = pack2(m0, m1);
-        *reinterpret_cast<uint32_t*>(p.pM + (static_cast<size_t>(l) * B + b) * F + j) = mw;
-        ll_store(p.llM + (static_cast<size_t>(l) * B + b) * (F / 2) + j / 2, mw, epoch);
+        *reinterpret_cast<uint32_t*>(p.pM + (static_cast<size_t>(l) * B + b) * F + n) = mw;
+        ll_store2(p.llM + (static_cast<size_t>(l) * B + b) * (F / 2) + w, p.rep.M, mw, epoch);
     } else if (g.type == kDOWN) {
         const uint16_t d0 = float_to_half_bits(v0);
         const uint16_t d1 = float_to_half_bits(v1);
         const uint32_t x2 = pack2(add_h(lo_f(resw), half_bits_to_float(d0)), add_h(hi_f(resw), half_bits_to_float(d1)));
         *reinterpret_cast<uint32_t*>(p.pD + (static_cast<size_t>(l) * B + b) * H + n) = pack2(d0, d1);
         *reinterpret_cast<uint32_t*>(p.pX2 + (static_cast<size_t>(l) * B + b) * H + n) = x2;
-        ll_store(p.llX + (static_cast<size_t>(l + 1) * B + b) * (H / 2) + n / 2, x2, epoch);
+        ll_store2(p.llX + (static_cast<size_t>(l + 1) * B + b) * (H / 2) + w, p.rep.X, x2, epoch);
     } else {
-        const int n4 = 4 * it;   // the LM head's items are 4 rows
-        uint16_t* out = p.logits + static_cast<size_t>(b) * p.V + n4;
-        const int nv = p.V - n4;
+        uint16_t* out = p.logits + static_cast<size_t>(b) * p.V + n;
         out[0] = float_to_half_bits(rf * v0);
-        if (nv > 1) out[1] = float_to_half_bits(rf * v1);
-        if (nv > 2) out[2] = float_to_half_bits(rf * v2);
-        if (nv > 3) out[3] = float_to_half_bits(rf * v3);
+        if (n + 1 < p.V) out[1] = float_to_half_bits(rf * v1);
     }
 }
 
@@ -429,16 +494,15 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
     extern __shared__ __align__(1024) uint8_t smem[];
     uint64_t* full = reinterpret_cast<uint64_t*>(smem);
     uint64_t* empty = full + kFullBars;
-    float* red = reinterpret_cast<float*>(smem + kHdrRed);          // [NW][kMaxChainBatch]
+    float* red = reinterpret_cast<float*>(smem + kHdrRed);          // [kMaxChainBatch][16]
     uint32_t* epoch_sh = reinterpret_cast<uint32_t*>(smem + kHdrEpoch);
-    uint32_t* res = reinterpret_cast<uint32_t*>(smem + kHdrRes);    // [B][items of the CTA]
     StageInfo* info = reinterpret_cast<StageInfo*>(smem + kHdrInfo);
-    uint8_t* wofs_tab = smem + kHdrWofs;
-    constexpr int kHeader = chain_header_bytes(NW, B);
-    uint4* xs = reinterpret_cast<uint4*>(smem + kHeader);
-    uint8_t* slots = smem + kHeader + p.x_bytes;
+    uint32_t* res = reinterpret_cast<uint32_t*>(smem + kHdrRes);    // [B][words of the CTA]
+    float4* part = reinterpret_cast<float4*>(smem + kHdrPart);      // [word][part][B]
+    uint4* xs = reinterpret_cast<uint4*>(smem + kChainHeader);       // [B][K / 8], pair-permuted
+    uint8_t* slots = smem + kChainHeader + p.x_bytes;
     constexpr int kConsumers = NW * 32;
-    constexpr int kPoll = 2;     // input chunks a thread has in flight at once
+    constexpr int kPoll = 3;     // input chunks a thread has in flight at once
 
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int nstages = 4 * p.L + 1;
@@ -460,18 +524,21 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
         const int t = threadIdx.x - 32;
         const Stage g = stage_at(p, stage_of_type(p, t));
         StageInfo in;
-        cta_items(g.items, &in.i0, &in.i1);
-        in.ips = items_per_slot(p, g);
-        in.nchunks = (in.i1 - in.i0 + in.ips - 1) / in.ips;
+        int w0, w1;
+        cta_words(g.words, &w0, &w1);
+        in.w0 = w0;
+        in.nwords = w1 - w0;
+        in.wps = words_per_slot(p, g);
+        in.nchunks = (in.nwords + in.wps - 1) / in.wps;
         in.nmod_slots = in.nchunks % p.nslots;
         in.nmod_bars = in.nchunks % p.nbars;
         in.flip = (in.nchunks / p.nbars) & 1;
-        in.pad = 0;
+        in.J = g.K >> 8;
+        in.spw = words_per_superpair(p, g);
+        in.q = p.q[t];
+        in.upp = in.J / in.q;
+        in.nsp = (in.nwords + in.spw - 1) / in.spw;
         info[t] = in;
-    }
-    if (threadIdx.x >= 64 && threadIdx.x < 64 + 5 * 16) {
-        const int t = (threadIdx.x - 64) >> 4, w = (threadIdx.x - 64) & 15;
-        wofs_tab[t * 16 + w] = static_cast<uint8_t>(w / items_per_slot(p, stage_at(p, stage_of_type(p, t))));
     }
     __syncthreads();
     const uint32_t epoch = *epoch_sh;
@@ -486,12 +553,12 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
             for (int st = 0; st < nstages; ++st) {
                 const Stage g = stage_at(p, st);
                 const StageInfo in = info[g.type];
-                const int i0 = in.i0, i1 = in.i1, ips = in.ips;
+                const int w0 = in.w0, w1 = in.w0 + in.nwords, wps = in.wps;
                 const int wpr = g.K >> 3, gpr = g.K >> 5;
-                for (int ia = i0; ia < i1; ia += ips, ++ord) {
-                    const int ib = min(i1, ia + ips);
+                for (int wa = w0; wa < w1; wa += wps, ++ord) {
+                    const int wb = min(w1, wa + wps);
                     if (round > 0) mbar_wait(&empty[slot], (round - 1) & 1, p.err);
-                    const ChunkLayout c = chunk_layout(g, ia, ib);
+                    const ChunkLayout c = chunk_layout(g, wa, wb);
                     uint8_t* dst = slots + static_cast<size_t>(slot) * p.slot_bytes;
                     uint64_t* fb = &full[fbi];
                     if (++slot == p.nslots) {
@@ -503,14 +570,13 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
                     if (g.type == kGU) {
                         const uint32_t hc = c.codes_bytes / 2, hs = c.scale_bytes / 2;
                         const size_t up = static_cast<size_t>(p.F);
-                        bulk_g2s(dst, g.W + static_cast<size_t>(2 * ia) * wpr, hc, fb, pol);
-                        bulk_g2s(dst + hc, g.W + (up + 2 * ia) * wpr, hc, fb, pol);
-                        bulk_g2s(dst + c.codes_bytes, g.s + static_cast<size_t>(2 * ia) * gpr, hs, fb, pol);
-                        bulk_g2s(dst + c.codes_bytes + hs, g.s + (up + 2 * ia) * gpr, hs, fb, pol);
+                        bulk_g2s(dst, g.W + static_cast<size_t>(2 * wa) * wpr, hc, fb, pol);
+                        bulk_g2s(dst + hc, g.W + (up + 2 * wa) * wpr, hc, fb, pol);
+                        bulk_g2s(dst + c.codes_bytes, g.s + static_cast<size_t>(2 * wa) * gpr, hs, fb, pol);
+                        bulk_g2s(dst + c.codes_bytes + hs, g.s + (up + 2 * wa) * gpr, hs, fb, pol);
                     } else {
-                        bulk_g2s(dst, g.W + static_cast<size_t>(g.rpi * ia) * wpr, c.codes_bytes, fb, pol);
-                        bulk_g2s(dst + c.codes_bytes, g.s + static_cast<size_t>(g.rpi * ia) * gpr, c.scale_bytes,
-                                 fb, pol);
+                        bulk_g2s(dst, g.W + static_cast<size_t>(2 * wa) * wpr, c.codes_bytes, fb, pol);
+                        bulk_g2s(dst + c.codes_bytes, g.s + static_cast<size_t>(2 * wa) * gpr, c.scale_bytes, fb, pol);
                     }
                 }
             }
@@ -522,37 +588,35 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
     } else {
         // ------------------------------------------------ consumer warps
         const int H = p.H, F = p.F;
-        // slot, full barrier and barrier parity of the stage's first chunk
-        int cslot = 0, cbar = 0;
-        uint32_t cpar = 0;
+        int cord0 = 0;   // ring ordinal of the stage's first chunk
         for (int st = 0; st < nstages; ++st) {
             const Stage g = stage_at(p, st);
             const StageInfo& in = info[g.type];
-            const int i0 = in.i0, i1 = in.i1;
-            if (i1 <= i0) continue;
+            if (in.nwords <= 0) continue;
             const int l = g.layer;
-            const int K = g.K, gpr = K >> 5, cpr = K >> 3;
-            const int nit = i1 - i0;
+            const int K = g.K, cpr = K >> 3;
+            const int nwd = in.nwords, w0 = in.w0;
 
-            // -- stage the input vector (all consumer warps), its RMS factor and
-            //    the residual words of the CTA's rows
-            named_barrier_sync(1, kConsumers);   // every warp is done with the previous xs and res
+            // -- stage the input vector (all consumer warps, pair-permuted),
+            //    its RMS factor and the residual words of the CTA's words
+            named_barrier_sync(1, kConsumers);   // every warp is done with the previous xs, res and part
             {
                 const uint64_t* ll = nullptr;
                 const bool plain = (g.type == kQKV && l == 0);
-                if (g.type == kQKV) ll = p.llX + static_cast<size_t>(l) * B * (H / 2);
-                else if (g.type == kO) ll = p.llA + static_cast<size_t>(l) * B * (H / 2);
-                else if (g.type == kGU) ll = p.llX1 + static_cast<size_t>(l) * B * (H / 2);
-                else if (g.type == kDOWN) ll = p.llM + static_cast<size_t>(l) * B * (F / 2);
-                else ll = p.llX + static_cast<size_t>(p.L) * B * (H / 2);
+                const bool r1 = (blockIdx.x & 1) != 0;   // this CTA's replica
+                if (g.type == kQKV) ll = p.llX + (r1 ? p.rep.X : 0u) + static_cast<size_t>(l) * B * (H / 2);
+                else if (g.type == kO) ll = p.llA + (r1 ? p.rep.A : 0u) + static_cast<size_t>(l) * B * (H / 2);
+                else if (g.type == kGU) ll = p.llX1 + (r1 ? p.rep.X1 : 0u) + static_cast<size_t>(l) * B * (H / 2);
+                else if (g.type == kDOWN) ll = p.llM + (r1 ? p.rep.M : 0u) + static_cast<size_t>(l) * B * (F / 2);
+                else ll = p.llX + (r1 ? p.rep.X : 0u) + static_cast<size_t>(p.L) * B * (H / 2);
                 const uint64_t* rl = nullptr;
-                if (g.type == kO) rl = p.llV + static_cast<size_t>(l) * B * (H / 2);
-                else if (g.type == kDOWN) rl = p.llX1 + static_cast<size_t>(l) * B * (H / 2);
+                if (g.type == kO) rl = p.llV + (r1 ? p.rep.V : 0u) + static_cast<size_t>(l) * B * (H / 2);
+                else if (g.type == kDOWN) rl = p.llX1 + (r1 ? p.rep.X1 : 0u) + static_cast<size_t>(l) * B * (H / 2);
                 if (rl) {
 #pragma unroll
                     for (int b = 0; b < B; ++b)
-                        for (int k = threadIdx.x; k < nit; k += kConsumers)
-                            res[b * nit + k] = ll_load(rl + static_cast<size_t>(b) * (H / 2) + i0 + k, epoch, p.err, p.abort);
+                        for (int k = threadIdx.x; k < nwd; k += kConsumers)
+                            res[b * nwd + k] = ll_load(rl + static_cast<size_t>(b) * (H / 2) + w0 + k, epoch, p.err, p.abort);
                 }
                 float ss[B];
 #pragma unroll
@@ -600,8 +664,8 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
                     for (int k = 0; k < kPoll; ++k) {
                         const int i = ib + k * kConsumers;
                         if (i < total) {
-                            const int b = i / cpr, c = i - b * cpr;
-                            xs[b * cpr + x_chunk(c >> 2, c & 3)] = v[k];
+                            const int b = i / cpr;
+                            xs[i] = pair_permute(v[k]);
 #pragma unroll
                             for (int bb = 0; bb < B; ++bb)
                                 if (bb == b) ss[bb] += sum8_sq(v[k]);
@@ -625,45 +689,30 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
                                 (((d.x + d.y) + (d.z + d.w)) + ((e.x + e.y) + (e.z + e.w)));
                 rf[b] = (g.type == kDOWN) ? 1.f : rsqrtf(t * (1.f / static_cast<float>(K)) + p.eps);
             }
-            if (g.type == kQKV || g.type == kLM) {
-                // the normalised layer input v = fp16(r * u) is kept for the
-                // residual stream (and the trace): every CTA publishes its
-                // slice of it; the projections below use r as a row factor
-                const int w0 = static_cast<int>(epoch_sh[1]), w1 = static_cast<int>(epoch_sh[2]);
-                const uint32_t* xw = reinterpret_cast<const uint32_t*>(xs);
-#pragma unroll
-                for (int b = 0; b < B; ++b) {
-                    for (int w = w0 + threadIdx.x; w < w1; w += kConsumers) {
-                        const int c = w >> 2;               // chunk of the word
-                        const uint32_t u = xw[4 * (b * cpr + x_chunk(c >> 2, c & 3)) + (w & 3)];
-                        const uint32_t v = pack2(float_to_half_bits(rf[b] * lo_f(u)), float_to_half_bits(rf[b] * hi_f(u)));
-                        reinterpret_cast<uint32_t*>(p.pV + (static_cast<size_t>(l) * B + b) * H)[w] = v;
-                        if (g.type == kQKV) ll_store(p.llV + (static_cast<size_t>(l) * B + b) * (H / 2) + w, v, epoch);
-                    }
-                }
-            }
-
-            // -- stream the CTA's items of this stage: item i0 + k goes to warp
-            //    k % NW; a warp visits only the chunks that hold its items
-            const int ips = in.ips;
-            const uint4* xl = xs + 4 * lane;
-            int it = i0 + warp;
-            if (it < i1) {
-                // the warp's first chunk: wofs chunks after the stage's first
-                const int wofs = wofs_tab[g.type * 16 + warp];
-                int ia = i0 + wofs * ips, ib = min(i1, ia + ips);
-                int slot = cslot + wofs;
-                while (slot >= p.nslots) slot -= p.nslots;
-                int bar = cbar + wofs;                      // wofs < nbars
-                uint32_t par = cpar;
-                if (bar >= p.nbars) {
-                    bar -= p.nbars;
-                    par ^= 1u;
-                }
-                while (it < i1) {
+            // -- items (superpair, K part) round-robin over the warps, in ring
+            //    order: item k goes to warp k % NW; a warp visits only the
+            //    chunks that hold its items
+            const int spw = in.spw, wps = in.wps, nch = in.nchunks, q = in.q, upp = in.upp;
+            const int nsp = in.nsp, nitems = nsp * q;
+            const int sps = spw - 1;                                        // log2 of words per superpair
+            const int spc = wps >> sps;                                     // superpairs per chunk
+            const int ips = spc * q;                                        // items per chunk
+            const uint32_t xsa = smem_addr(xs);
+            const FDiv fq = fdiv_make(q), fips = fdiv_make(ips), fns = fdiv_make(p.nslots), fnb = fdiv_make(p.nbars);
+            int it = warp;
+            if (it < nitems) {
+                int k = fdiv(it, fips);                                     // chunk of the warp's first item
+                int ia = k * ips, ib = min(nitems, ia + ips);
+                int ord = cord0 + k;
+                int slot = ord - fdiv(ord, fns) * p.nslots;
+                const int qb = fdiv(ord, fnb);
+                int bar = ord - qb * p.nbars;
+                uint32_t par = static_cast<uint32_t>(qb) & 1u;
+                while (it < nitems) {
                     while (it >= ib) {                      // next chunk
+                        ++k;
                         ia += ips;
-                        ib = min(i1, ia + ips);
+                        ib = min(nitems, ia + ips);
                         if (++slot == p.nslots) slot = 0;
                         if (++bar == p.nbars) {
                             bar = 0;
@@ -671,64 +720,139 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
                         }
                     }
                     mbar_wait(&full[bar], par, p.err);
-                    const uint8_t* base = slots + static_cast<size_t>(slot) * p.slot_bytes;
-                    const ChunkLayout c = chunk_layout(g, ia, ib);
+                    const int kw0 = k * wps, kw1 = min(nwd, kw0 + wps);   // the chunk's words
+                    const ChunkLayout c = chunk_layout(g, w0 + kw0, w0 + kw1);
+                    const uint32_t cbase = smem_addr(slots + static_cast<size_t>(slot) * p.slot_bytes);
+                    const uint32_t sbase = cbase + c.codes_bytes;
                     uint32_t arrivals = (it == ia) ? kSlotRelease - static_cast<uint32_t>(ib - ia) : 0u;
                     for (; it < ib; it += NW) {
                         ++arrivals;
-                        const int ii = it - ia;        // item within the chunk
-                        const uint4* crow[4];
-                        const uint16_t* srow[4];
+                        const int sl = fdiv(it, fq);         // the item's superpair and K part
+                        const int pt = it - sl * q;
+                        const int jb = pt * upp, je = jb + upp;
+                        const int sw0 = sl << sps;           // the superpair's first word (stage-relative)
+                        const int wl = sw0 - kw0;            // ... within the chunk
+                        uint32_t ra[2], rb[2];
                         if (g.type == kGU) {
+                            // pairs (gate 2w + pr, up 2w + pr) of word w
 #pragma unroll
-                            for (int r = 0; r < 4; ++r) {
-                                const int half = r >> 1, rr = 2 * ii + (r & 1);
-                                crow[r] = reinterpret_cast<const uint4*>(base + static_cast<size_t>(half) * (c.codes_bytes / 2) +
-                                                                         static_cast<size_t>(rr) * (K / 2)) + lane;
-                                srow[r] = reinterpret_cast<const uint16_t*>(base + c.codes_bytes + half * (c.scale_bytes / 2) +
-                                                                            rr * (K / 16)) + lane;
+                            for (int pr = 0; pr < 2; ++pr) {
+                                ra[pr] = 2 * wl + pr;
+                                rb[pr] = c.nh + 2 * wl + pr;
                             }
                         } else {
-                            // rows rpi*it .. rpi*it + rpi - 1; rows past N repeat the first
-                            const int nvalid = min(g.rpi, g.N - g.rpi * it);
+                            // pairs (2w, 2w + 1) of words w, w + 1 (one-word superpairs, or
+                            // the second word missing at the end of the CTA's words: pair 0
+                            // again, not computed or ignored; rows past N -- the LM head's
+                            // last -- read row 2w again, ignored)
 #pragma unroll
-                            for (int r = 0; r < 4; ++r) {
-                                const int rr = g.rpi * ii + (r < nvalid ? r : 0);
-                                crow[r] = reinterpret_cast<const uint4*>(base + static_cast<size_t>(rr) * (K / 2)) + lane;
-                                srow[r] = reinterpret_cast<const uint16_t*>(base + c.codes_bytes + rr * (K / 16)) + lane;
+                            for (int pr = 0; pr < 2; ++pr) {
+                                const int wr = (sw0 + pr < nwd) ? wl + pr : wl;
+                                ra[pr] = 2 * wr;
+                                rb[pr] = (2 * (w0 + kw0 + wr) + 1 < g.N) ? 2 * wr + 1 : 2 * wr;
                             }
                         }
-                        float acc[4][B];
+                        uint32_t ca[2], cb2[2], sa[2], sb2[2];
 #pragma unroll
-                        for (int r = 0; r < 4; ++r)
+                        for (int pr = 0; pr < 2; ++pr) {
+                            ca[pr] = cbase + ra[pr] * (K / 2);
+                            cb2[pr] = cbase + rb[pr] * (K / 2);
+                            sa[pr] = sbase + ra[pr] * (K / 16);
+                            sb2[pr] = sbase + rb[pr] * (K / 16);
+                        }
+                        float acc[2][B];
 #pragma unroll
-                            for (int b = 0; b < B; ++b) acc[r][b] = 0.f;
-                        if (g.rpi == 4) item_dot<B, 4>(crow, srow, xl, cpr, gpr, lane, acc);
-                        else item_dot<B, 2>(crow, srow, xl, cpr, gpr, lane, acc);
+                        for (int pr = 0; pr < 2; ++pr)
 #pragma unroll
-                        for (int r = 0; r < 4; ++r)
+                            for (int b = 0; b < B; ++b) acc[pr][b] = 0.f;
+                        const bool two = g.type == kGU || spw == 2;
+                        if (two) {
+                            item_units<B, 2>(ca, cb2, sa, sb2, xsa, cpr, jb, je, acc);
+                        } else {
+                            const uint32_t ca1[1] = {ca[0]}, cb1[1] = {cb2[0]}, sa1[1] = {sa[0]}, sb1[1] = {sb2[0]};
+                            float (&acc1)[1][B] = *reinterpret_cast<float (*)[1][B]>(&acc[0]);
+                            item_units<B, 1>(ca1, cb1, sa1, sb1, xsa, cpr, jb, je, acc1);
+                        }
 #pragma unroll
-                            for (int b = 0; b < B; ++b)
-                                if (r < g.rpi) acc[r][b] = warp_sum(acc[r][b]);
+                        for (int pr = 0; pr < 2; ++pr)
 #pragma unroll
-                        for (int b = 0; b < B; ++b)
-                            if (lane == b)
-                                item_epilogue<B>(p, g, it, b, acc[0][b], acc[1][b], acc[2][b], acc[3][b], rf[b],
-                                                 (g.type == kO || g.type == kDOWN) ? res[b * nit + (it - i0)] : 0u,
-                                                 epoch);
+                            for (int b = 0; b < B; ++b) acc[pr][b] = pair_reduce(acc[pr][b]);
+                        // this item's part of the superpair's row sums: (pair 0 row a,
+                        // pair 0 row b, pair 1 row a, pair 1 row b); lane 0 holds the
+                        // a rows, lane 16 the b rows
+                        if (g.type == kLM) {
+                            // whole superpairs (one part): lane 0 writes rows 2w and
+                            // 2w + 2, lane 16 rows 2w + 1 and 2w + 3 of words w, w + 1
+                            const int n0 = 2 * (w0 + sw0) + (lane == 16 ? 1 : 0);
+#pragma unroll
+                            for (int b = 0; b < B; ++b) {
+                                uint16_t* out = p.logits + static_cast<size_t>(b) * p.V;
+                                if (lane == 0 || lane == 16) {
+                                    if (n0 < p.V) out[n0] = float_to_half_bits(rf[b] * acc[0][b]);
+                                    if (spw == 2 && sw0 + 1 < nwd && n0 + 2 < p.V)
+                                        out[n0 + 2] = float_to_half_bits(rf[b] * acc[1][b]);
+                                }
+                            }
+                        } else {
+                            float* pf = reinterpret_cast<float*>(part + (sl * q + pt) * B);
+#pragma unroll
+                            for (int b = 0; b < B; ++b) {
+                                if (lane == 0) { pf[4 * b + 0] = acc[0][b]; pf[4 * b + 2] = acc[1][b]; }
+                                if (lane == 16) { pf[4 * b + 1] = acc[0][b]; pf[4 * b + 3] = acc[1][b]; }
+                            }
+                        }
                     }
                     __syncwarp();
                     if (lane == 0) mbar_arrive_count(&empty[slot], arrivals);
                 }
             }
-            cslot += in.nmod_slots;
-            if (cslot >= p.nslots) cslot -= p.nslots;
-            cbar += in.nmod_bars;
-            cpar ^= static_cast<uint32_t>(in.flip);
-            if (cbar >= p.nbars) {
-                cbar -= p.nbars;
-                cpar ^= 1u;
+            if (g.type == kQKV || g.type == kLM) {
+                // the normalised layer input v = fp16(r * u) is kept for the
+                // residual stream (and the trace): every CTA publishes its
+                // slice of it; the projections below use r as a row factor
+                const int vw0 = static_cast<int>(epoch_sh[1]), vw1 = static_cast<int>(epoch_sh[2]);
+                const uint32_t* xw = reinterpret_cast<const uint32_t*>(xs);
+#pragma unroll
+                for (int b = 0; b < B; ++b) {
+                    for (int w = vw0 + threadIdx.x; w < vw1; w += kConsumers) {
+                        const uint32_t u = permuted_word(xw + 4 * b * cpr, w);
+                        const uint32_t v = pack2(float_to_half_bits(rf[b] * lo_f(u)), float_to_half_bits(rf[b] * hi_f(u)));
+                        reinterpret_cast<uint32_t*>(p.pV + (static_cast<size_t>(l) * B + b) * H)[w] = v;
+                        if (g.type == kQKV) ll_store2(p.llV + (static_cast<size_t>(l) * B + b) * (H / 2) + w, p.rep.V, v, epoch);
+                    }
+                }
             }
+
+            // -- every part of every word is in: add the parts in part order and
+            //    publish the words, one thread per (superpair, batch row) on the
+            //    first warps (spreading the entries over all warps, one lane
+            //    each, measured 0.2 ms a token slower)
+            if (g.type != kLM) named_barrier_sync(1, kConsumers);
+            for (int e = threadIdx.x; g.type != kLM && e < nsp * B; e += kConsumers) {
+                const int sl = e / B, b = e - sl * B;
+                const float4* pp = part + sl * q * B + b;
+                float4 sum = pp[0];
+                for (int r = 1; r < q; ++r) {
+                    const float4 t4 = pp[r * B];
+                    sum.x += t4.x; sum.y += t4.y; sum.z += t4.z; sum.w += t4.w;
+                }
+                const int wc = sl << sps;                     // first word (stage-relative)
+#pragma unroll
+                for (int bb = 0; bb < B; ++bb) {
+                    if (bb != b) continue;
+                    if (g.type == kGU) {
+                        word_epilogue<B>(p, g, w0 + wc, bb, sum.x, sum.z, sum.y, sum.w, rf[bb], 0u, epoch);
+                    } else {
+                        const bool resid = (g.type == kO || g.type == kDOWN);
+                        word_epilogue<B>(p, g, w0 + wc, bb, sum.x, sum.y, 0.f, 0.f, rf[bb],
+                                         resid ? res[bb * nwd + wc] : 0u, epoch);
+                        if (spw == 2 && wc + 1 < nwd)
+                            word_epilogue<B>(p, g, w0 + wc + 1, bb, sum.z, sum.w, 0.f, 0.f, rf[bb],
+                                             resid ? res[bb * nwd + wc + 1] : 0u, epoch);
+                    }
+                }
+            }
+            cord0 += nch;
         }
     }
 
@@ -800,11 +924,11 @@ Layout make_layout(const Dims& d)
     y.header = take(256);
     y.mats = take(sizeof(DevMat) * (4 * L + 1));
     y.ll_begin = o;
-    y.llA = take(8 * L * B * (H / 2));
-    y.llX1 = take(8 * L * B * (H / 2));
-    y.llM = take(8 * L * B * (F / 2));
-    y.llX = take(8 * (L + 1) * B * (H / 2));
-    y.llV = take(8 * L * B * (H / 2));
+    y.llA = take(8 * 2 * L * B * (H / 2));        // two replicas each
+    y.llX1 = take(8 * 2 * L * B * (H / 2));
+    y.llM = take(8 * 2 * L * B * (F / 2));
+    y.llX = take(8 * 2 * (L + 1) * B * (H / 2));
+    y.llV = take(8 * 2 * L * B * (H / 2));
     y.ll_end = o;
     y.pV = take(2 * (L + 1) * B * H);
     y.pX2 = take(2 * L * B * H);
@@ -843,6 +967,8 @@ struct Plan {
     uint32_t slot_bytes, x_bytes;
     size_t smem;
     int nw;
+    int q[5];                // K parts per superpair, per stage type
+    int spw[5];              // words per superpair, per stage type
     cudaGraphExec_t graph;   // graph path (batch > kMaxChainBatch), else null
 };
 
@@ -863,41 +989,60 @@ bool mat_ok(const wq4_mat& m)
 template <int B>
 cudaError_t set_chain_attr(int smem)
 {
-    return cudaFuncSetAttribute(chain_kernel<B, ChainWarps<B>::NW>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    return cudaFuncSetAttribute(chain_kernel<B, kChainWarps>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
 }
 
-int chain_warps(int B)
+// Bytes of one output word of each stage type (two rows; gate_up four).
+void word_bytes(const Dims& d, size_t out[5])
 {
-    switch (B) {
-        case 1: return ChainWarps<1>::NW;
-        case 2: return ChainWarps<2>::NW;
-        default: return ChainWarps<2>::NW;
-    }
-}
-
-
-// Slot size: a multiple of 128 bytes holding at least one item of every
-// stage, chosen to waste the least ring space over the chain's byte mix.
-uint32_t choose_slot_bytes(const Dims& d)
-{
-    struct S { size_t item, bytes; };
     const size_t rowH = static_cast<size_t>(d.H) / 2 + d.H / 16, rowF = static_cast<size_t>(d.F) / 2 + d.F / 16;
-    const S st[5] = {{2 * rowH, static_cast<size_t>(d.Nqkv) * rowH},
-                     {2 * rowH, static_cast<size_t>(d.H) * rowH},
-                     {4 * rowH, static_cast<size_t>(2) * d.F * rowH},
-                     {2 * rowF, static_cast<size_t>(d.H) * rowF},
-                     {4 * rowH, static_cast<size_t>(d.V) * rowH}};
+    out[0] = 2 * rowH;   // QKV
+    out[1] = 2 * rowH;   // O
+    out[2] = 4 * rowH;   // gate_up
+    out[3] = 2 * rowF;   // down
+    out[4] = 2 * rowH;   // LM head
+}
+
+// Words of each stage type.
+void stage_words(const Dims& d, int out[5])
+{
+    out[0] = d.Nqkv / 2;
+    out[1] = d.H / 2;
+    out[2] = d.F / 2;
+    out[3] = d.H / 2;
+    out[4] = (d.V + 1) / 2;
+}
+
+// Words per superpair of each stage type: two words (four rows sharing the
+// activations) unless that is more than kMaxSuperpairBytes of weights;
+// gate_up's word already holds two row pairs.
+constexpr size_t kMaxSuperpairBytes = 20 * 1024;
+void choose_spw(const Dims& d, int spw[5])
+{
+    size_t wb[5];
+    word_bytes(d, wb);
+    for (int t = 0; t < 5; ++t) spw[t] = (t == 2 || 2 * wb[t] > kMaxSuperpairBytes) ? 1 : 2;
+}
+
+// Slot size: a multiple of 128 bytes holding at least one superpair of every
+// stage, chosen to waste the least ring space over the chain's byte mix.
+uint32_t choose_slot_bytes(const Dims& d, const int spw[5])
+{
+    size_t wb[5];
+    word_bytes(d, wb);
+    int words[5];
+    stage_words(d, words);
     size_t max_item = 0;
-    for (const S& s : st) max_item = s.item > max_item ? s.item : max_item;
+    for (int t = 0; t < 5; ++t) max_item = wb[t] * spw[t] > max_item ? wb[t] * spw[t] : max_item;
     size_t lo = align_up(max_item, 128);
     if (lo < 16384) lo = 16384;
     size_t best = lo;
     double best_waste = 1e300;
     for (size_t sb = lo; sb <= lo + 8192; sb += 128) {
         double waste = 0;
-        for (const S& s : st) {
-            const size_t ips = sb / s.item;
-            waste += static_cast<double>(s.bytes) * (1.0 - static_cast<double>(ips * s.item) / sb);
+        for (int t = 0; t < 5; ++t) {
+            const size_t wps = sb / wb[t] / spw[t] * spw[t];
+            waste += static_cast<double>(words[t]) * wb[t] * (1.0 - static_cast<double>(wps * wb[t]) / sb);
         }
         if (waste < best_waste) {
             best_waste = waste;
@@ -912,15 +1057,60 @@ int full_bars(int nslots)
     return (kFullBars / nslots) * nslots;
 }
 
-// True when no consumer wait on the ring can alias: for every stage,
-// nslots + ceil(NW / items per slot) <= the number of full barriers.
-bool ring_ok(const Dims& d, int nslots, uint32_t slot_bytes, int nw)
+// K parts per superpair for each stage type: a divisor q of the stage's
+// 256-code group sets that gives the least per-warp time when the CTA's
+// superpairs x q items are taken round-robin by the consumer warps: rounds x
+// (units x unit cost + item cost), with the costs measured on this kernel
+// (a unit of two row pairs ~300 cycles, one row pair ~200, an item ~1200:
+// the first unit's latency, the reduction and the chunk hand-over).  The
+// items the warps run at once must sit in at most nslots - 2 chunks, or the
+// last warps wait for slots; the partial sums of all the CTA's superpairs
+// must fit in shared memory.  The LM head keeps whole superpairs (q = 1, no
+// partial sums).  Returns false if some stage has no admissible q.
+bool choose_parts(const Dims& d, int grid, int nw, const int spw[5], int nslots, uint32_t slot_bytes, int q[5])
 {
-    const size_t rowH = static_cast<size_t>(d.H) / 2 + d.H / 16, rowF = static_cast<size_t>(d.F) / 2 + d.F / 16;
-    const size_t items[5] = {2 * rowH, 2 * rowH, 4 * rowH, 2 * rowF, 4 * rowH};
-    for (size_t item : items) {
-        size_t ips = slot_bytes / item;
-        if (ips < 1) ips = 1;
+    int words[5];
+    stage_words(d, words);
+    size_t wb[5];
+    word_bytes(d, wb);
+    const int J[5] = {d.H / 256, d.H / 256, d.H / 256, d.F / 256, d.H / 256};
+    q[4] = 1;
+    for (int t = 0; t < 4; ++t) {
+        q[t] = 0;
+        const long wmax = (words[t] + grid - 1) / grid;
+        const long spmax = (wmax + spw[t] - 1) / spw[t];
+        size_t spc = slot_bytes / wb[t] / spw[t];
+        if (spc < 1) spc = 1;
+        const bool two = t == 2 || spw[t] == 2;
+        const double unit = two ? 300.0 * (1.0 + 0.5 * (d.B - 1)) : 200.0 * (1.0 + 0.5 * (d.B - 1));
+        double best = 1e300;
+        for (int c = 1; c <= J[t]; ++c) {
+            if (J[t] % c || spmax * c * d.B > kMaxPart) continue;
+            const size_t ips = spc * static_cast<size_t>(c);
+            if ((static_cast<size_t>(nw) + ips - 1) / ips > static_cast<size_t>(nslots > 3 ? nslots - 2 : 1)) continue;
+            const long rounds = (spmax * c + nw - 1) / nw;
+            const double cost = static_cast<double>(rounds) * ((J[t] / c) * unit + 1200.0);
+            if (cost <= best) {   // ties: more, shorter items (measured faster)
+                best = cost;
+                q[t] = c;
+            }
+        }
+        if (q[t] == 0) return false;
+    }
+    return true;
+}
+
+// True when no consumer wait on the ring can alias: for every stage,
+// nslots + ceil(NW / items per slot) <= the number of full barriers (items
+// per slot = superpairs per slot x K parts).
+bool ring_ok(const Dims& d, int nslots, uint32_t slot_bytes, int nw, const int spw[5], const int q[5])
+{
+    size_t wb[5];
+    word_bytes(d, wb);
+    for (int t = 0; t < 5; ++t) {
+        size_t sps = slot_bytes / wb[t] / spw[t];
+        if (sps < 1) sps = 1;
+        const size_t ips = sps * static_cast<size_t>(q[t]);
         if (static_cast<size_t>(nslots) + (nw + ips - 1) / ips > static_cast<size_t>(full_bars(nslots))) return false;
     }
     return true;
@@ -1013,14 +1203,20 @@ int build_plan(const wq4_layer_table* t, Plan* pl, cudaStream_t stream)
     }
     if (!di->coop_launch) return WQ4_ERR_UNSUPPORTED;
     const uint32_t x_bytes = static_cast<uint32_t>(align_up(static_cast<size_t>(d.B) * 2 * (d.H > d.F ? d.H : d.F), 128));
-    const uint32_t slot_bytes = choose_slot_bytes(d);
-    const int header = chain_header_bytes(chain_warps(d.B), d.B);
+    // the residual words of a CTA's words must fit in shared memory
+    if (static_cast<long>((d.H / 2 + di->sm_count - 1) / di->sm_count) * d.B > kMaxResWords) return WQ4_ERR_UNSUPPORTED;
+    int spw[5];
+    choose_spw(d, spw);
+    const uint32_t slot_bytes = choose_slot_bytes(d, spw);
+    const int header = kChainHeader;
     const long avail = static_cast<long>(di->smem_optin) - header - static_cast<long>(x_bytes);
     int nslots = avail > 0 ? static_cast<int>(avail / slot_bytes) : 0;
     if (nslots > kChainMaxSlots) nslots = kChainMaxSlots;
+    int q[5];
+    if (!choose_parts(d, di->sm_count, kChainWarps, spw, nslots, slot_bytes, q)) return WQ4_ERR_UNSUPPORTED;
     // fewer slots give more full barriers per slot: take the deepest ring
     // whose barriers cannot alias
-    while (nslots >= 2 && !ring_ok(d, nslots, slot_bytes, chain_warps(d.B))) --nslots;
+    while (nslots >= 2 && !ring_ok(d, nslots, slot_bytes, kChainWarps, spw, q)) --nslots;
     if (nslots < 2) return WQ4_ERR_UNSUPPORTED;
     const size_t smem = header + x_bytes + static_cast<size_t>(nslots) * slot_bytes;
     // The limit is a property of the kernel, shared by every plan: set it to
@@ -1062,9 +1258,9 @@ int build_plan(const wq4_layer_table* t, Plan* pl, cudaStream_t stream)
     pl->slot_bytes = slot_bytes;
     pl->x_bytes = x_bytes;
     pl->smem = smem;
-    pl->nw = chain_warps(d.B);
-    // the residual words of a CTA's rows must fit in shared memory
-    if (static_cast<long>((d.H / 2 + pl->grid - 1) / pl->grid) * d.B > kMaxResWords) return WQ4_ERR_UNSUPPORTED;
+    pl->nw = kChainWarps;
+    for (int t = 0; t < 5; ++t) pl->q[t] = q[t];
+    for (int t = 0; t < 5; ++t) pl->spw[t] = spw[t];
     return WQ4_OK;
 }
 
@@ -1102,6 +1298,15 @@ int launch_chain(const Plan& pl, const uint16_t* x, uint16_t* logits, cudaStream
     p.llM = reinterpret_cast<uint64_t*>(ws + y.llM);
     p.llX = reinterpret_cast<uint64_t*>(ws + y.llX);
     p.llV = reinterpret_cast<uint64_t*>(ws + y.llV);
+    {
+        const uint32_t L = static_cast<uint32_t>(pl.dims.L), B = static_cast<uint32_t>(pl.dims.B);
+        const uint32_t H = static_cast<uint32_t>(pl.dims.H), F = static_cast<uint32_t>(pl.dims.F);
+        p.rep.A = L * B * (H / 2);
+        p.rep.X1 = L * B * (H / 2);
+        p.rep.M = L * B * (F / 2);
+        p.rep.X = (L + 1) * B * (H / 2);
+        p.rep.V = L * B * (H / 2);
+    }
     p.pV = reinterpret_cast<uint16_t*>(ws + y.pV);
     p.pX2 = reinterpret_cast<uint16_t*>(ws + y.pX2);
     p.pQKV = reinterpret_cast<uint16_t*>(ws + y.pQKV);
@@ -1114,6 +1319,8 @@ int launch_chain(const Plan& pl, const uint16_t* x, uint16_t* logits, cudaStream
     p.nbars = pl.nbars;
     p.slot_bytes = pl.slot_bytes;
     p.x_bytes = pl.x_bytes;
+    for (int t = 0; t < 5; ++t) p.q[t] = pl.q[t];
+    for (int t = 0; t < 5; ++t) p.spw[t] = pl.spw[t];
     p.err = status_word();
     if (!p.err) return WQ4_ERR_CUDA;
 
@@ -1129,9 +1336,8 @@ int launch_chain(const Plan& pl, const uint16_t* x, uint16_t* logits, cudaStream
     cfg.numAttrs = 1;
     cudaError_t e;
     switch (pl.dims.B) {
-        case 1: e = cudaLaunchKernelEx(&cfg, chain_kernel<1, ChainWarps<1>::NW>, p); break;
-        case 2: e = cudaLaunchKernelEx(&cfg, chain_kernel<2, ChainWarps<2>::NW>, p); break;
-        default: e = cudaLaunchKernelEx(&cfg, chain_kernel<2, ChainWarps<2>::NW>, p); break;
+        case 1: e = cudaLaunchKernelEx(&cfg, chain_kernel<1, kChainWarps>, p); break;
+        default: e = cudaLaunchKernelEx(&cfg, chain_kernel<2, kChainWarps>, p); break;
     }
     return e == cudaSuccess ? WQ4_OK : WQ4_ERR_CUDA;
 }

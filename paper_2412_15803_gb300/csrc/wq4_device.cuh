@@ -229,6 +229,44 @@ __device__ __forceinline__ void group_dot_smem(uint4 cw, float sc, const uint4* 
     }
 }
 
+// ------------------------------------------------ legacy tensor-core path --
+
+// Two 8x8 b16 matrices from shared memory: lane t (t < 16) supplies the
+// address of row t & 7 of matrix t >> 3 (16-byte aligned); lane (g, c) =
+// (lane >> 2, lane & 3) receives bytes 4c..4c+3 of row g of each matrix.
+__device__ __forceinline__ void ldsm_x2(uint32_t addr, uint32_t& r0, uint32_t& r1)
+{
+    asm volatile("ldmatrix.sync.aligned.m8n8.x2.shared.b16 {%0, %1}, [%2];" : "=r"(r0), "=r"(r1) : "r"(addr) : "memory");
+}
+
+__device__ __forceinline__ uint32_t lds_u32(uint32_t addr)
+{
+    uint32_t v;
+    asm volatile("ld.shared.b32 %0, [%1];" : "=r"(v) : "r"(addr) : "memory");
+    return v;
+}
+
+__device__ __forceinline__ uint4 lds_v4(uint32_t addr)
+{
+    uint4 v;
+    asm volatile("ld.shared.v4.b32 {%0, %1, %2, %3}, [%4];" : "=r"(v.x), "=r"(v.y), "=r"(v.z), "=r"(v.w) : "r"(addr) : "memory");
+    return v;
+}
+
+// D = A (16x16, fp16, row-major fragment a[0..3]) * B (16x8, fp16, column
+// fragment b0, b1) + C, fp32 accumulation.  Fragments of lane (g, c):
+// a = {A[g][2c..2c+1], A[g+8][2c..2c+1], A[g][2c+8..2c+9], A[g+8][2c+8..2c+9]},
+// b0 = B[2c..2c+1][g], b1 = B[2c+8..2c+9][g],
+// d = {D[g][2c], D[g][2c+1], D[g+8][2c], D[g+8][2c+1]}.
+// fp16 x fp16 products are exact in fp32.
+__device__ __forceinline__ void mma_16816(float d[4], uint32_t a0, uint32_t a1, uint32_t a2, uint32_t a3, uint32_t b0,
+                                          uint32_t b1, const float c[4])
+{
+    asm("mma.sync.aligned.m16n8k16.row.col.f32.f16.f16.f32 {%0,%1,%2,%3}, {%4,%5,%6,%7}, {%8,%9}, {%10,%11,%12,%13};"
+        : "=f"(d[0]), "=f"(d[1]), "=f"(d[2]), "=f"(d[3])
+        : "r"(a0), "r"(a1), "r"(a2), "r"(a3), "r"(b0), "r"(b1), "f"(c[0]), "f"(c[1]), "f"(c[2]), "f"(c[3]));
+}
+
 __device__ __forceinline__ float warp_sum(float v)
 {
 #pragma unroll

@@ -56,6 +56,10 @@ enum wq4_status {
 /* Largest batch (rows of x) any call accepts. */
 #define WQ4_MAX_BATCH 32
 
+/* Largest scale magnitude of the paths that round the dequantized weight
+ * (q - 7) * s to fp16 (wq4_gemm, wq4_decode_chain at batch 3-32). */
+#define WQ4_MAX_FP16_SCALE 8188.0f
+
 /*
  * y[b][n] = fp16( sum_k (q(n,k) - 7) * scales[n][k/32] * x[b][k] )
  * for b < batch, n < N: the fused dequantize-and-multiply projection of one
@@ -80,7 +84,11 @@ int wq4_gemv(const uint32_t* W_packed, const uint16_t* scales, const uint16_t* x
  * prompt through one projection), on the tensor cores:
  *   Y[m][n] = fp16( sum_k x[m][k] * fp16((q(n,k) - 7) * scales[n][k/32]) )
  * for m < M, n < N, sums in fp32.  Each dequantized weight is rounded to fp16
- * once (relative error <= 2^-11), so the accuracy contract above holds.
+ * once (relative error <= 2^-11), so the accuracy contract above holds for
+ * every scale with |s| <= 8188 (WQ4_MAX_FP16_SCALE; 8 * 8188 = 65504, the
+ * fp16 maximum).  A larger scale makes some (q - 7) s overflow fp16: the call
+ * still runs, sets bit 6 of the device status word (wq4_device_status) and
+ * the outputs of those rows are not valid; wq4_gemv has no such limit.
  *   W_packed, scales : as wq4_gemv, both 16-byte aligned.
  *   x : fp16 bits [M][K], 16-byte aligned.   y : fp16 bits [M][N], 16-byte
  *       aligned, must not overlap x, W or scales.
@@ -120,8 +128,9 @@ const char* wq4_status_string(int status);
  * another CTA's activations gave up; wq4_attn.h calls add bit 3 = a sequence
  * length beyond its page table (clamped), bit 4 = a page id outside the pool
  * (zeros read in its place), bit 5 = an append with a bad position or page
- * id (nothing written).  Returns WQ4_ERR_TIMEOUT if any bit was set, WQ4_OK
- * otherwise, WQ4_ERR_CUDA on a CUDA failure.
+ * id (nothing written); bit 6 = wq4_gemm met a scale beyond
+ * WQ4_MAX_FP16_SCALE (its outputs are not valid).  Returns WQ4_ERR_TIMEOUT if
+ * any bit was set, WQ4_OK otherwise, WQ4_ERR_CUDA on a CUDA failure.
  */
 int wq4_device_status(void* stream, int* flags_out);
 
@@ -188,17 +197,22 @@ size_t wq4_chain_workspace_bytes(const wq4_layer_table* table);
  * residual stream.
  *   x      : fp16 [batch][hidden] device, 16-byte aligned
  *   logits : fp16 [batch][vocab]  device, 2-byte aligned
- * Batch 1-2 runs as the persistent kernel above.  Batch 3-32 runs as a CUDA
- * graph, captured once per table, of one tensor-core kernel per projection
- * (dequantized fp16 weights w = fp16((q - 7) s) times the batch's inputs,
- * tcgen05 MMAs with fp32 accumulation, the chain's row factors, residual adds
- * and SiLU fused into each stage's epilogue); each call copies x into the
- * workspace, replays the graph and copies the logits out (all on `stream`).
- * The first call for a table (or after its contents changed) validates it and
- * uploads its pointer table into the workspace (cudaMemcpyAsync on `stream`);
- * later calls only launch.  Rebuilding the plan of a batch 3-32 table
- * synchronizes `stream` before freeing the old graph.  Calls on one table must
- * not overlap on the GPU.
+ * Batch 1-2 runs as the persistent kernel above (exact dequantization, any
+ * fp16 scale).  Batch 3-32 runs as a CUDA graph, captured once per table, of
+ * one tensor-core kernel per projection (dequantized fp16 weights
+ * w = fp16((q - 7) s) times the batch's inputs, tcgen05 MMAs with fp32
+ * accumulation, the chain's row factors, residual adds and SiLU fused into
+ * each stage's epilogue); each call copies x into the workspace, replays the
+ * graph and copies the logits out (all on `stream`).
+ * The first call for a table (or after its contents changed) builds its plan:
+ * at batch 1-2 it validates the table and uploads its pointer table into the
+ * workspace (cudaMemcpyAsync on `stream`); at batch 3-32 it also scans every
+ * scale (a table with a scale beyond WQ4_MAX_FP16_SCALE is rejected with
+ * WQ4_ERR_UNSUPPORTED), synchronizes `stream`, and captures and instantiates
+ * the CUDA graph (driver-side resources, no device memory of this library);
+ * rebuilding a batch 3-32 plan also synchronizes `stream` before freeing the
+ * old graph.  Later calls only launch.  Calls on one table must not overlap
+ * on the GPU.
  * Returns WQ4_OK, WQ4_ERR_INVALID, WQ4_ERR_ALIGN, WQ4_ERR_UNSUPPORTED or
  * WQ4_ERR_CUDA (including a GPU that cannot co-schedule the persistent grid).
  */
@@ -237,7 +251,13 @@ int wq4_decode_chain_host(const wq4_layer_table* table, const uint16_t* x_host,
  *     before any stream capture.
  *   - All calls on a device share the one array, which keeps the last call's
  *     contents; the first call for a table, or a call with a different table
- *     than the previous one, clears the array's counters and flags again.
+ *     than the previous one, rebuilds the plan and clears the array's
+ *     counters and flags again.  A rebuild enqueues copies on `stream`; at
+ *     batch 3-32 (the tables that fit: the tiny and small shapes) it also
+ *     scans the scales, synchronizes `stream` and captures and instantiates
+ *     a CUDA graph (driver-side resources, but no device memory).  Make every
+ *     call that switches tables outside stream capture: a rebuild requested
+ *     while `stream` is capturing returns WQ4_ERR_UNSUPPORTED.
  *     Calls that overlap on the GPU race on the array: serialize them.
  *   - A table whose wq4_chain_workspace_bytes exceeds
  *     WQ4_NOALLOC_SCRATCH_BYTES is rejected with WQ4_ERR_UNSUPPORTED before
@@ -247,7 +267,9 @@ int wq4_decode_chain_noalloc(const wq4_layer_table* table, const uint16_t* x,
                              uint16_t* logits, void* stream);
 
 /* Releases the cached plan of `table` (host-side state only; the workspace
- * stays the caller's).  Returns WQ4_ERR_INVALID if no plan exists. */
+ * stays the caller's).  A batch 3-32 plan owns a CUDA graph: synchronize every
+ * stream that ran the table before calling this.  Returns WQ4_ERR_INVALID if
+ * no plan exists. */
 int wq4_chain_plan_destroy(const wq4_layer_table* table);
 
 /*

@@ -70,8 +70,9 @@ constexpr uint32_t kSlotRelease = 1024;
 // RMS partial sums | epoch | stage table | warp table | residual words of the
 // CTA's words (O and down stages) | per-item partial row sums; then the
 // staged input vector, then the weight ring.
-constexpr int kHdrRed = 512;                 // float red[kMaxChainBatch][16]: per-warp sums of squares
+constexpr int kHdrRed = 512;                 // float red[kMaxChainBatch][32]: per-warp sums of squares
 static_assert(8 * (kFullBars + kChainMaxSlots) <= kHdrRed, "mbarriers overlap the header");
+static_assert(kHdrRed + 4 * 2 * 32 <= 768, "RMS partial sums overlap the header");
 constexpr int kHdrEpoch = 768;               // uint32 epoch, then int vw0, vw1 (the CTA's slice of v)
 constexpr int kHdrInfo = 784;                // StageInfo info[5], one per stage type
 constexpr int kHdrRes = 1152;                // uint32 res[kMaxResWords]: prefetched residual words
@@ -494,7 +495,7 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
     extern __shared__ __align__(1024) uint8_t smem[];
     uint64_t* full = reinterpret_cast<uint64_t*>(smem);
     uint64_t* empty = full + kFullBars;
-    float* red = reinterpret_cast<float*>(smem + kHdrRed);          // [kMaxChainBatch][16]
+    float* red = reinterpret_cast<float*>(smem + kHdrRed);          // [kMaxChainBatch][32]
     uint32_t* epoch_sh = reinterpret_cast<uint32_t*>(smem + kHdrEpoch);
     StageInfo* info = reinterpret_cast<StageInfo*>(smem + kHdrInfo);
     uint32_t* res = reinterpret_cast<uint32_t*>(smem + kHdrRes);    // [B][words of the CTA]
@@ -519,7 +520,7 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
         epoch_sh[1] = static_cast<int>(static_cast<int64_t>(blockIdx.x) * nw / gridDim.x);
         epoch_sh[2] = static_cast<int>(static_cast<int64_t>(blockIdx.x + 1) * nw / gridDim.x);
     }
-    if (threadIdx.x < kMaxChainBatch * 16) red[threadIdx.x] = 0.f;   // warps >= NW stay zero
+    if (threadIdx.x < kMaxChainBatch * 32) red[threadIdx.x] = 0.f;   // warps >= NW stay zero
     if (threadIdx.x >= 32 && threadIdx.x < 32 + 5) {
         const int t = threadIdx.x - 32;
         const Stage g = stage_at(p, stage_of_type(p, t));
@@ -675,7 +676,7 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
 #pragma unroll
                 for (int b = 0; b < B; ++b) {
                     const float v = warp_sum(ss[b]);
-                    if (lane == 0) red[b * 16 + warp] = v;
+                    if (lane == 0) red[b * 32 + warp] = v;
                 }
             }
             named_barrier_sync(1, kConsumers);
@@ -683,10 +684,14 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
 #pragma unroll
             for (int b = 0; b < B; ++b) {
                 // the same sum, in the same order, in every warp and every CTA
-                const float4* r4 = reinterpret_cast<const float4*>(red + b * 16);
-                const float4 a = r4[0], c = r4[1], d = r4[2], e = r4[3];
-                const float t = (((a.x + a.y) + (a.z + a.w)) + ((c.x + c.y) + (c.z + c.w))) +
-                                (((d.x + d.y) + (d.z + d.w)) + ((e.x + e.y) + (e.z + e.w)));
+                const float4* r4 = reinterpret_cast<const float4*>(red + b * 32);
+                float q4[8];
+#pragma unroll
+                for (int i = 0; i < 8; ++i) {
+                    const float4 a = r4[i];
+                    q4[i] = (a.x + a.y) + (a.z + a.w);
+                }
+                const float t = ((q4[0] + q4[1]) + (q4[2] + q4[3])) + ((q4[4] + q4[5]) + (q4[6] + q4[7]));
                 rf[b] = (g.type == kDOWN) ? 1.f : rsqrtf(t * (1.f / static_cast<float>(K)) + p.eps);
             }
             // -- items (superpair, K part) round-robin over the warps, in ring
@@ -1116,6 +1121,47 @@ bool ring_ok(const Dims& d, int nslots, uint32_t slot_bytes, int nw, const int s
     return true;
 }
 
+// Largest |scale| (as fp16 bits without the sign) of n scales into *out.
+__global__ void scale_max_kernel(const uint16_t* s, size_t n, uint32_t* out)
+{
+    uint32_t m = 0;
+    for (size_t i = static_cast<size_t>(blockIdx.x) * blockDim.x + threadIdx.x; i < n;
+         i += static_cast<size_t>(gridDim.x) * blockDim.x) {
+        const uint32_t b = s[i] & 0x7FFFu;
+        m = b > m ? b : m;
+    }
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) {
+        const uint32_t t = __shfl_xor_sync(0xffffffffu, m, o);
+        m = t > m ? t : m;
+    }
+    if ((threadIdx.x & 31) == 0) atomicMax(out, m);
+}
+
+// The batched path rounds each dequantized weight (q - 7) s to fp16: every
+// scale of the table must be within +-8188.  Scans all scales once (at plan
+// build) and synchronizes `stream` to read the result.
+int check_scales_fp16(const wq4_layer_table* t, const Dims& d, uint32_t* scratch_word, cudaStream_t stream)
+{
+    if (cudaMemsetAsync(scratch_word, 0, 4, stream) != cudaSuccess) return WQ4_ERR_CUDA;
+    auto scan = [&](const wq4_mat& m, size_t n) {
+        scale_max_kernel<<<64, 256, 0, stream>>>(m.s, n, scratch_word);
+        return cudaGetLastError() == cudaSuccess;
+    };
+    const size_t H = d.H, F = d.F;
+    for (int l = 0; l < d.L; ++l) {
+        const wq4_layer& ly = t->layers[l];
+        if (!scan(ly.qkv, static_cast<size_t>(d.Nqkv) * (H / 32)) || !scan(ly.o, H * (H / 32)) ||
+            !scan(ly.gate_up, 2 * F * (H / 32)) || !scan(ly.down, H * (F / 32)))
+            return WQ4_ERR_CUDA;
+    }
+    if (!scan(t->lm_head, static_cast<size_t>(d.V) * (H / 32))) return WQ4_ERR_CUDA;
+    uint32_t m = 0;
+    if (cudaMemcpyAsync(&m, scratch_word, 4, cudaMemcpyDeviceToHost, stream) != cudaSuccess) return WQ4_ERR_CUDA;
+    if (cudaStreamSynchronize(stream) != cudaSuccess) return WQ4_ERR_CUDA;
+    return m > kMaxFp16ScaleBits ? WQ4_ERR_UNSUPPORTED : WQ4_OK;
+}
+
 // Records one token of the graph path on `cs`: every stage kernel of every
 // layer, reading the token input from the workspace staging area and writing
 // the logits to the workspace logits area.
@@ -1123,9 +1169,9 @@ int build_graph_plan(const wq4_layer_table* t, const Dims& d, const Layout& lay,
                      Plan* pl, cudaStream_t stream)
 {
     uint8_t* ws = static_cast<uint8_t*>(t->workspace);
-    // the split stages' arrival counters start at zero (each stage leaves them so)
-    if (cudaMemsetAsync(ws + lay.cnt, 0, 4 * static_cast<size_t>(kTcCounterWords), stream) != cudaSuccess)
-        return WQ4_ERR_CUDA;
+    // scales beyond +-8188 would overflow the fp16 dequantized weights
+    const int rs = check_scales_fp16(t, d, reinterpret_cast<uint32_t*>(ws + lay.header) + 3, stream);
+    if (rs != WQ4_OK) return rs;
     auto U16 = [&](size_t off) { return reinterpret_cast<uint16_t*>(ws + off); };
     TcBuffers buf;
     buf.x_stage = U16(lay.x_stage);
@@ -1156,7 +1202,12 @@ int build_graph_plan(const wq4_layer_table* t, const Dims& d, const Layout& lay,
     cudaGraphExec_t exec = nullptr;
     rc = WQ4_ERR_CUDA;
     if (cudaStreamBeginCapture(cs, cudaStreamCaptureModeThreadLocal) == cudaSuccess) {
-        const int rrec = tc_record_token(tc, cs);
+        // every token starts with zero arrival counters (a stage whose waits gave
+        // up may leave some non-zero; the next token must not inherit them)
+        int rrec = cudaMemsetAsync(ws + lay.cnt, 0, 4 * static_cast<size_t>(kTcCounterWords), cs) == cudaSuccess
+                       ? WQ4_OK
+                       : WQ4_ERR_CUDA;
+        if (rrec == WQ4_OK) rrec = tc_record_token(tc, cs);
         if (cudaStreamEndCapture(cs, &graph) == cudaSuccess && graph && rrec == WQ4_OK &&
             cudaGraphInstantiate(&exec, graph, 0) == cudaSuccess)
             rc = WQ4_OK;
@@ -1342,8 +1393,10 @@ int launch_chain(const Plan& pl, const uint16_t* x, uint16_t* logits, cudaStream
     return e == cudaSuccess ? WQ4_OK : WQ4_ERR_CUDA;
 }
 
-// Finds (or builds) the plan of `t`; returns a copy to launch from.
-int get_plan(const wq4_layer_table* t, Plan* out, cudaStream_t stream)
+// Finds (or builds) the plan of `t`; returns a copy to launch from.  With
+// no_rebuild_in_capture, a plan that would have to be (re)built while
+// `stream` is capturing is refused with WQ4_ERR_UNSUPPORTED.
+int get_plan(const wq4_layer_table* t, Plan* out, cudaStream_t stream, bool no_rebuild_in_capture = false)
 {
     if (!t) return WQ4_ERR_INVALID;
     Dims d;
@@ -1355,6 +1408,11 @@ int get_plan(const wq4_layer_table* t, Plan* out, cudaStream_t stream)
     if (it != g_plans.end() && it->second.device == dev && same_contents(it->second, t)) {
         *out = it->second;
         return WQ4_OK;
+    }
+    if (no_rebuild_in_capture) {
+        cudaStreamCaptureStatus cs = cudaStreamCaptureStatusNone;
+        if (cudaStreamIsCapturing(stream, &cs) != cudaSuccess) return WQ4_ERR_CUDA;
+        if (cs != cudaStreamCaptureStatusNone) return WQ4_ERR_UNSUPPORTED;
     }
     Plan pl;
     const int rc = build_plan(t, &pl, stream);
@@ -1501,7 +1559,7 @@ extern "C" int wq4_decode_chain_noalloc(const wq4_layer_table* table, const uint
     nd.table.workspace = nd.scratch;
     nd.table.workspace_bytes = kNoAllocScratchBytes;
     Plan pl;
-    const int rc = get_plan(&nd.table, &pl, st);
+    const int rc = get_plan(&nd.table, &pl, st, true);
     if (rc != WQ4_OK) return rc;
     const size_t lb = static_cast<size_t>(pl.dims.B) * pl.dims.V * 2;
     if (overlaps(logits, lb, x, static_cast<size_t>(pl.dims.B) * pl.dims.H * 2)) return WQ4_ERR_INVALID;

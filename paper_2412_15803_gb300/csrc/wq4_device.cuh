@@ -20,6 +20,12 @@ constexpr uint32_t kErrFlagTimeout = 2u;   // a wait on another CTA's data gave 
 constexpr uint32_t kErrSeqLen = 8u;        // attention: a length beyond the page table (clamped)
 constexpr uint32_t kErrPageId = 16u;       // attention: a page id outside the pool (zeros read)
 constexpr uint32_t kErrAppend = 32u;       // append: bad position or page id (row not written)
+constexpr uint32_t kErrScale = 64u;        // a scale beyond +-8188 met an fp16 dequantized-weight path
+
+// Largest fp16 scale magnitude whose dequantized weights (q - 7) s, |q - 7|
+// <= 8, stay finite in fp16 (8 * 8188 = 65504, the fp16 maximum; the next
+// fp16 value, 8192, overflows).  As the bits of |s|: 0x6FFF.
+constexpr uint32_t kMaxFp16ScaleBits = 0x6FFFu;
 
 // Every spin-wait gives up after this long (a legitimate wait lasts
 // microseconds); the kernel then records the error and runs to its end.

@@ -199,6 +199,8 @@ __global__ void __launch_bounds__(kGThreads, 1)
                 const uint8_t* crow = base + row * 32;
                 // scale of group 2 (c & 3) + jg of the 8 loaded for this 256-wide block
                 const uint32_t sh = *reinterpret_cast<const uint16_t*>(base + kGCodes + row * 16 + 4 * (c & 3) + 2 * jg);
+                // (q - 7) s is rounded to fp16 below: a larger scale would overflow
+                if ((sh & 0x7FFFu) > kMaxFp16ScaleBits) atomicOr(err, kErrScale);
                 {
                     const int j = jg;   // 16-byte chunk of the 32-byte row, 32-byte swizzle
                     const uint4 cw = *reinterpret_cast<const uint4*>(crow + ((j ^ ((row >> 2) & 1)) << 4));

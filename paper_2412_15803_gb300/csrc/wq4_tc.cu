@@ -437,6 +437,8 @@ __global__ void __launch_bounds__(kTcThreads, 1)
                     const uint4 cw = *reinterpret_cast<const uint4*>(crow + ((j ^ (row & 7)) << 4));
                     const uint32_t sh = (jj & 1) ? (sw[jj >> 1] >> 16) : (sw[jj >> 1] & 0xFFFFu);
                     const uint32_t s2 = sh | (sh << 16);
+                    // (q - 7) s is rounded to fp16 here: a larger scale would overflow
+                    if ((sh & 0x7FFFu) > kMaxFp16ScaleBits) atomicOr(err, kErrScale);
                     uint32_t q[16];
                     unpack_word(cw.x, q + 0);
                     unpack_word(cw.y, q + 4);

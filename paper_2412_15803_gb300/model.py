@@ -66,11 +66,17 @@ def fill_matrix(W, s, N: int, K: int, seed: int, layer: int, mat: int, symmetric
 
 
 class DecodeModel:
-    """A synthetic decoder resident in device memory plus its wq4 layer table."""
+    """A synthetic decoder resident in device memory plus its wq4 layer table.
 
-    def __init__(self, shape: ModelShape, batch: int = 1, seed: int = 0, eps: float = 1e-5, device=None):
+    symmetric: codes drawn on 0..14 (the default, zero-mean q - 7, so that deep
+    chains stay within fp16) or, with False, uniform on 0..15 (every code value,
+    including 15, reaches every kernel; fine for a few layers)."""
+
+    def __init__(self, shape: ModelShape, batch: int = 1, seed: int = 0, eps: float = 1e-5, device=None,
+                 symmetric: bool = True):
         import torch
         self.shape, self.batch, self.seed, self.eps = shape, batch, seed, eps
+        self.symmetric = symmetric
         dev = torch.device("cuda") if device is None else torch.device(device)
         self.weights = []          # per layer: dict name -> (W tensor, s tensor)
         self._keep = []
@@ -80,14 +86,14 @@ class DecodeModel:
             for name, N, K, mat in shape.mats(l):
                 W = torch.empty((N, K // 8), dtype=torch.int32, device=dev)
                 s = torch.empty((N, K // 32), dtype=torch.int16, device=dev)
-                fill_matrix(W, s, N, K, seed, l, mat, symmetric=True)
+                fill_matrix(W, s, N, K, seed, l, mat, symmetric=symmetric)
                 d[name] = (W, s)
                 setattr(layers[l], name, _w.wq4_mat(W.data_ptr(), s.data_ptr()))
             self.weights.append(d)
         V, H = shape.vocab, shape.hidden
         W = torch.empty((V, H // 8), dtype=torch.int32, device=dev)
         s = torch.empty((V, H // 32), dtype=torch.int16, device=dev)
-        fill_matrix(W, s, V, H, seed, shape.num_layers, synth.MAT_LM_HEAD, symmetric=True)
+        fill_matrix(W, s, V, H, seed, shape.num_layers, synth.MAT_LM_HEAD, symmetric=symmetric)
         self.lm_head = (W, s)
         self._layers = layers
         t = _w.wq4_layer_table()
@@ -141,4 +147,4 @@ class DecodeModel:
             N, K, mat, lay = sh.vocab, sh.hidden, synth.MAT_LM_HEAD, sh.num_layers
         else:
             (N, K, mat), lay = [(N, K, m) for nm, N, K, m in sh.mats(layer) if nm == name][0], layer
-        return synth.matrix(self.seed, N, K, lay, mat, row_start, nrows, symmetric=True)
+        return synth.matrix(self.seed, N, K, lay, mat, row_start, nrows, symmetric=self.symmetric)

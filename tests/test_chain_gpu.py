@@ -121,6 +121,20 @@ def test_tiny_chain_every_stage_every_element(batch):
     assert rel < 2e-2, rel
 
 
+@pytest.mark.parametrize("shape,batch", [(TINY, 1), (TINY, 2), (TINY, 3), (TINY, 8), (TINY, 32), (SMALL, 1), (SMALL, 4)])
+def test_chain_full_range_codes_every_element(shape, batch):
+    """Codes uniform on 0..15 (every code value, code 15 = weight 8 s, on
+    every path: the persistent kernel's exact tensor-path dequantization at
+    batch 1-2, the fp16 dequantized weights of the stage graph at 3-32);
+    every stage, every element, and the logits."""
+    model = DecodeModel(shape, batch=batch, seed=40 + batch, symmetric=False)
+    x = synth.activations(140 + batch, batch, shape.hidden)
+    logits = run(model, x)
+    for l in range(shape.num_layers):
+        check_stages(model, l, u=x if l == 0 else None)
+    check_logits(model, logits)
+
+
 def test_tiny_chain_repeat_and_host_variant():
     model = DecodeModel(TINY, batch=2, seed=9)
     x = synth.activations(7, 2, TINY.hidden)
@@ -190,12 +204,13 @@ def test_3b_chain_full_size_sampled():
     assert np.array_equal(run(model, x), logits)
 
 
-@pytest.mark.parametrize("batch", [1, 4])
+@pytest.mark.parametrize("batch", [1, 2, 4, 8, 16, 32])
 def test_8b_chain_full_size_sampled(batch):
-    """The 32-layer 8B-shaped chain at batch 1 (persistent CUDA-core kernel:
-    the longest rows, K = 14336 in the down projection) and at batch 4
-    (tensor-core stage graph).  Sampled rows of three layers and of the LM
-    head, and twenty tokens with identical bits."""
+    """The 32-layer 8B-shaped chain over the batch sweep: batch 1-2 on the
+    persistent kernel (the longest rows, K = 14336 in the down projection,
+    one row pair per item), 4-32 on the tensor-core stage graph (batch 17-32:
+    32-column tiles and 8-part K splits at K = 14336).  Sampled rows of three
+    layers and of the LM head, and twenty tokens with identical bits."""
     sh = SHAPE_8B
     model = DecodeModel(sh, batch=batch, seed=3)
     x = synth.activations(5, batch, sh.hidden)

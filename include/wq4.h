@@ -161,7 +161,8 @@ typedef struct {
  *   is the stand-in attention output, see wq4_decode_chain).
  *   workspace  : device buffer of at least wq4_chain_workspace_bytes(table)
  *                bytes, 256-byte aligned, used only by this table's chain.
- *   hidden and ffn must be multiples of 256, vocab any >= 1, batch 1..32.
+ *   hidden and ffn must be multiples of 256, vocab any >= 1, batch 1..32;
+ *   batch 1-2 takes at most 128 layers (WQ4_ERR_UNSUPPORTED beyond).
  */
 typedef struct {
     int num_layers, hidden, ffn, n_q_heads, n_kv_heads, head_dim, vocab, batch;
@@ -268,8 +269,13 @@ int wq4_decode_chain_noalloc(const wq4_layer_table* table, const uint16_t* x,
 
 /* Releases the cached plan of `table` (host-side state only; the workspace
  * stays the caller's).  A batch 3-32 plan owns a CUDA graph: synchronize every
- * stream that ran the table before calling this.  Returns WQ4_ERR_INVALID if
- * no plan exists. */
+ * stream that ran the table before calling this.  Plans are cached by the
+ * table's address and contents: release a table's plan before freeing any
+ * buffer it names, or a later table at the same address with the same
+ * pointers reuses the plan without re-initialising its workspace.  (The batch
+ * 1-2 kernel takes the weight pointers in its launch parameters, so such a
+ * reuse reads no pointer from the workspace.)  Returns WQ4_ERR_INVALID if no
+ * plan exists. */
 int wq4_chain_plan_destroy(const wq4_layer_table* table);
 
 /*
@@ -290,6 +296,28 @@ typedef struct {
 } wq4_chain_trace;
 
 int wq4_chain_trace_offsets(const wq4_layer_table* table, int layer, wq4_chain_trace* out);
+
+/*
+ * Test hook of the bounded device waits (no counterpart in the paper: the
+ * paper's kernels run as separate launches and never wait on one another).
+ * Sets, for every later launch of the batch 1-2 chain kernel in this process
+ * (wq4_decode_chain, _host, _noalloc; a CUDA graph that captured a launch
+ * keeps the values of its capture):
+ *   wait_limit_ns : how long one wait on another CTA's activations polls
+ *                   before it gives up (1 .. 500,000,000; the default is
+ *                   500,000,000 = 0.5 s).  The weight pipeline's mbarrier
+ *                   waits keep the default.
+ *   stall_stage   : -1 (default) for none, else the stage 4*layer + t
+ *                   (t = 0 QKV, 1 O, 2 gate_up, 3 down; 4*n_layers = LM head)
+ *                   whose input waits poll for an epoch that no CTA writes,
+ *                   so that they run out.  Stage 0 reads x directly and has
+ *                   no such wait.
+ * After a stalled stage the kernel still finishes (its outputs are not
+ * valid), every access stays within the workspace, and wq4_device_status
+ * reports bit 1.  Returns WQ4_ERR_INVALID for a limit of 0 or above the
+ * default, or a stage below -1.
+ */
+int wq4_test_chain_waits(uint64_t wait_limit_ns, int stall_stage);
 
 #ifdef __cplusplus
 }

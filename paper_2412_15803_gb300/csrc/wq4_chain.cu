@@ -45,6 +45,7 @@
 
 #include <cmath>
 #include <cstring>
+#include <atomic>
 #include <map>
 #include <mutex>
 #include <vector>
@@ -93,8 +94,12 @@ struct DevMat {
     const uint16_t* s;
 };
 
+// Largest layer count of the persistent chain: its weight pointers travel in
+// the launch parameters (a __grid_constant__ struct), not in the workspace, so
+// no plan depends on device memory the caller could have freed or zeroed.
+constexpr int kChainMaxLayers = 128;
+
 struct ChainParams {
-    const DevMat* mats;  // [4L + 1]: per layer qkv, o, gate_up, down; then lm_head
     int L, H, F, Nqkv, V;
     float eps;
     int q[5];            // K parts per superpair, per stage type (divides K / 256)
@@ -126,7 +131,11 @@ struct ChainParams {
     uint32_t slot_bytes;
     uint32_t x_bytes;
     uint32_t* err;
+    uint64_t wait_ns;    // limit of a wait on flagged words (kWaitTimeoutNs unless a test sets it)
+    int stall_stage;     // test hook: this stage waits for an epoch nobody writes (-1: none)
+    DevMat mats[4 * kChainMaxLayers + 1];   // [4L + 1]: per layer qkv, o, gate_up, down; then lm_head
 };
+static_assert(sizeof(ChainParams) <= 32764, "kernel parameter space");
 
 // One stage: N output rows of K codes, `words` output words of rpw rows each
 // (gate_up: gate rows 2w, 2w+1 and up rows F+2w, F+2w+1; the LM head's last
@@ -272,12 +281,12 @@ __device__ __forceinline__ uint64_t ll_load1_raw(const uint64_t* addr)
     return a;
 }
 
-// A wait gives up after kWaitTimeoutNs, or at once when another CTA already
-// gave up on this token; the first to give up records the token in *abort.
-__device__ __forceinline__ bool gave_up(uint64_t t0, uint32_t epoch, uint32_t* abort)
+// A wait gives up after limit_ns, or at once when another CTA already gave
+// up on this token (epoch); the first to give up records the token in *abort.
+__device__ __forceinline__ bool gave_up(uint64_t t0, uint32_t epoch, uint32_t* abort, uint64_t limit_ns)
 {
     if (*reinterpret_cast<const volatile uint32_t*>(abort) == epoch) return true;
-    if (globaltimer_ns() - t0 > kWaitTimeoutNs) {
+    if (globaltimer_ns() - t0 > limit_ns) {
         atomicExch(abort, epoch);
         return true;
     }
@@ -285,22 +294,24 @@ __device__ __forceinline__ bool gave_up(uint64_t t0, uint32_t epoch, uint32_t* a
 }
 
 // Four consecutive flagged words (8 fp16 values) at a 32-byte aligned address;
-// polls until all four carry `epoch`.
-__device__ __forceinline__ uint4 ll_load4(const uint64_t* addr, uint32_t epoch, uint32_t* err, uint32_t* abort)
+// polls until all four carry `tag` (the token's epoch, or under the stall test
+// hook an epoch that no CTA writes during the token).
+__device__ __forceinline__ uint4 ll_load4(const uint64_t* addr, uint32_t tag, uint32_t epoch, uint32_t* err,
+                                         uint32_t* abort, uint64_t limit_ns)
 {
     uint64_t a, b, c, d;
     ll_load2_raw(addr, a, b);
     ll_load2_raw(addr + 2, c, d);
-    if (static_cast<uint32_t>(a >> 32) != epoch || static_cast<uint32_t>(b >> 32) != epoch ||
-        static_cast<uint32_t>(c >> 32) != epoch || static_cast<uint32_t>(d >> 32) != epoch) {
+    if (static_cast<uint32_t>(a >> 32) != tag || static_cast<uint32_t>(b >> 32) != tag ||
+        static_cast<uint32_t>(c >> 32) != tag || static_cast<uint32_t>(d >> 32) != tag) {
         const uint64_t t0 = globaltimer_ns();
         for (uint32_t it = 0;; ++it) {
             ll_load2_raw(addr, a, b);
             ll_load2_raw(addr + 2, c, d);
-            if (static_cast<uint32_t>(a >> 32) == epoch && static_cast<uint32_t>(b >> 32) == epoch &&
-                static_cast<uint32_t>(c >> 32) == epoch && static_cast<uint32_t>(d >> 32) == epoch)
+            if (static_cast<uint32_t>(a >> 32) == tag && static_cast<uint32_t>(b >> 32) == tag &&
+                static_cast<uint32_t>(c >> 32) == tag && static_cast<uint32_t>(d >> 32) == tag)
                 break;
-            if ((it & 63) == 63 && gave_up(t0, epoch, abort)) {
+            if ((it & 63) == 63 && gave_up(t0, epoch, abort, limit_ns)) {
                 atomicOr(err, kErrFlagTimeout);
                 break;
             }
@@ -310,15 +321,16 @@ __device__ __forceinline__ uint4 ll_load4(const uint64_t* addr, uint32_t epoch, 
                       static_cast<uint32_t>(d));
 }
 
-__device__ __forceinline__ uint32_t ll_load(const uint64_t* addr, uint32_t epoch, uint32_t* err, uint32_t* abort)
+__device__ __forceinline__ uint32_t ll_load(const uint64_t* addr, uint32_t tag, uint32_t epoch, uint32_t* err,
+                                           uint32_t* abort, uint64_t limit_ns)
 {
     uint64_t a = ll_load1_raw(addr);
-    if (static_cast<uint32_t>(a >> 32) != epoch) {
+    if (static_cast<uint32_t>(a >> 32) != tag) {
         const uint64_t t0 = globaltimer_ns();
         for (uint32_t it = 0;; ++it) {
             a = ll_load1_raw(addr);
-            if (static_cast<uint32_t>(a >> 32) == epoch) break;
-            if ((it & 63) == 63 && gave_up(t0, epoch, abort)) {
+            if (static_cast<uint32_t>(a >> 32) == tag) break;
+            if ((it & 63) == 63 && gave_up(t0, epoch, abort, limit_ns)) {
                 atomicOr(err, kErrFlagTimeout);
                 break;
             }
@@ -490,7 +502,7 @@ __device__ __forceinline__ void word_epilogue(const ChainParams& p, const Stage&
 }
 
 template <int B, int NW>
-__global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainParams p)
+__global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const __grid_constant__ ChainParams p)
 {
     extern __shared__ __align__(1024) uint8_t smem[];
     uint64_t* full = reinterpret_cast<uint64_t*>(smem);
@@ -600,6 +612,9 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
 
             // -- stage the input vector (all consumer warps, pair-permuted),
             //    its RMS factor and the residual words of the CTA's words
+            //    (the stall test hook makes one stage wait for an epoch that no
+            //    producer writes: its waits run out, bounded)
+            const uint32_t want = (st == p.stall_stage) ? (epoch + 0x80000000u) : epoch;
             named_barrier_sync(1, kConsumers);   // every warp is done with the previous xs, res and part
             {
                 const uint64_t* ll = nullptr;
@@ -617,7 +632,7 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
 #pragma unroll
                     for (int b = 0; b < B; ++b)
                         for (int k = threadIdx.x; k < nwd; k += kConsumers)
-                            res[b * nwd + k] = ll_load(rl + static_cast<size_t>(b) * (H / 2) + w0 + k, epoch, p.err, p.abort);
+                            res[b * nwd + k] = ll_load(rl + static_cast<size_t>(b) * (H / 2) + w0 + k, want, epoch, p.err, p.abort, p.wait_ns);
                 }
                 float ss[B];
 #pragma unroll
@@ -650,13 +665,13 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
                             if (i < total) {
                                 bool ok = true;
 #pragma unroll
-                                for (int j = 0; j < 4; ++j) ok = ok && static_cast<uint32_t>(w[k][j] >> 32) == epoch;
+                                for (int j = 0; j < 4; ++j) ok = ok && static_cast<uint32_t>(w[k][j] >> 32) == want;
                                 if (ok) {
                                     v[k] = make_uint4(static_cast<uint32_t>(w[k][0]), static_cast<uint32_t>(w[k][1]),
                                                       static_cast<uint32_t>(w[k][2]), static_cast<uint32_t>(w[k][3]));
                                 } else {
                                     const int b = i / cpr, c = i - b * cpr;
-                                    v[k] = ll_load4(ll + static_cast<size_t>(b) * (K / 2) + 4 * c, epoch, p.err, p.abort);
+                                    v[k] = ll_load4(ll + static_cast<size_t>(b) * (K / 2) + 4 * c, want, epoch, p.err, p.abort, p.wait_ns);
                                 }
                             }
                         }
@@ -884,7 +899,7 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const ChainPara
 // ---------------------------------------------------------------- host --
 
 struct Layout {
-    size_t header, mats, llA, llX1, llM, llX, llV, pV, pX2, pQKV, pO, pX1, pGU, pM, pD, x_stage, logits_stage, rfac,
+    size_t header, llA, llX1, llM, llX, llV, pV, pX2, pQKV, pO, pX1, pGU, pM, pD, x_stage, logits_stage, rfac,
         xpH0, xpH1, xpF, cnt, part, total;
     size_t ll_begin, ll_end;
 };
@@ -927,7 +942,6 @@ Layout make_layout(const Dims& d)
     };
     const size_t B = d.B, L = d.L, H = d.H, F = d.F;
     y.header = take(256);
-    y.mats = take(sizeof(DevMat) * (4 * L + 1));
     y.ll_begin = o;
     y.llA = take(8 * 2 * L * B * (H / 2));        // two replicas each
     y.llX1 = take(8 * 2 * L * B * (H / 2));
@@ -979,6 +993,13 @@ struct Plan {
 
 std::mutex g_plan_mu;
 std::map<const wq4_layer_table*, Plan> g_plans;
+
+// Test hook state (wq4_test_chain_waits): the limit of the chain kernel's
+// waits on flagged words and the stage whose input waits can never be
+// satisfied.  The mbarrier waits of the weight ring keep kWaitTimeoutNs: a
+// producer that gave up early would refill a slot that is still being read.
+std::atomic<uint64_t> g_wait_ns{kWaitTimeoutNs};
+std::atomic<int> g_stall_stage{-1};
 
 bool same_contents(const Plan& pl, const wq4_layer_table* t)
 {
@@ -1253,6 +1274,7 @@ int build_plan(const wq4_layer_table* t, Plan* pl, cudaStream_t stream)
         return build_graph_plan(t, d, lay, dev, di, pl, stream);
     }
     if (!di->coop_launch) return WQ4_ERR_UNSUPPORTED;
+    if (d.L > kChainMaxLayers) return WQ4_ERR_UNSUPPORTED;
     const uint32_t x_bytes = static_cast<uint32_t>(align_up(static_cast<size_t>(d.B) * 2 * (d.H > d.F ? d.H : d.F), 128));
     // the residual words of a CTA's words must fit in shared memory
     if (static_cast<long>((d.H / 2 + di->sm_count - 1) / di->sm_count) * d.B > kMaxResWords) return WQ4_ERR_UNSUPPORTED;
@@ -1280,23 +1302,10 @@ int build_plan(const wq4_layer_table* t, Plan* pl, cudaStream_t stream)
     }
     if (e != cudaSuccess) return WQ4_ERR_CUDA;
 
-    std::vector<DevMat> mats(4 * static_cast<size_t>(d.L) + 1);
-    for (int l = 0; l < d.L; ++l) {
-        const wq4_layer& ly = t->layers[l];
-        mats[4 * l + 0] = {ly.qkv.W, ly.qkv.s};
-        mats[4 * l + 1] = {ly.o.W, ly.o.s};
-        mats[4 * l + 2] = {ly.gate_up.W, ly.gate_up.s};
-        mats[4 * l + 3] = {ly.down.W, ly.down.s};
-    }
-    mats[4 * d.L] = {t->lm_head.W, t->lm_head.s};
     uint8_t* ws = static_cast<uint8_t*>(t->workspace);
     // header (token counter) and every flagged word start at zero: epoch 0 never matches
     if (cudaMemsetAsync(ws + lay.header, 0, 256, stream) != cudaSuccess) return WQ4_ERR_CUDA;
     if (cudaMemsetAsync(ws + lay.ll_begin, 0, lay.ll_end - lay.ll_begin, stream) != cudaSuccess) return WQ4_ERR_CUDA;
-    // pageable source: the call returns once the bytes are staged
-    if (cudaMemcpyAsync(ws + lay.mats, mats.data(), sizeof(DevMat) * mats.size(), cudaMemcpyHostToDevice, stream) !=
-        cudaSuccess)
-        return WQ4_ERR_CUDA;
 
     pl->table = *t;
     pl->layers.assign(t->layers, t->layers + d.L);
@@ -1331,8 +1340,15 @@ int launch_chain(const Plan& pl, const uint16_t* x, uint16_t* logits, cudaStream
             return WQ4_ERR_CUDA;
         return WQ4_OK;
     }
-    ChainParams p;
-    p.mats = reinterpret_cast<const DevMat*>(ws + y.mats);
+    ChainParams p = {};
+    for (int l = 0; l < pl.dims.L; ++l) {
+        const wq4_layer& ly = pl.layers[l];
+        p.mats[4 * l + 0] = {ly.qkv.W, ly.qkv.s};
+        p.mats[4 * l + 1] = {ly.o.W, ly.o.s};
+        p.mats[4 * l + 2] = {ly.gate_up.W, ly.gate_up.s};
+        p.mats[4 * l + 3] = {ly.down.W, ly.down.s};
+    }
+    p.mats[4 * pl.dims.L] = {pl.table.lm_head.W, pl.table.lm_head.s};
     p.L = pl.dims.L;
     p.H = pl.dims.H;
     p.F = pl.dims.F;
@@ -1374,6 +1390,8 @@ int launch_chain(const Plan& pl, const uint16_t* x, uint16_t* logits, cudaStream
     for (int t = 0; t < 5; ++t) p.spw[t] = pl.spw[t];
     p.err = status_word();
     if (!p.err) return WQ4_ERR_CUDA;
+    p.wait_ns = g_wait_ns.load();
+    p.stall_stage = g_stall_stage.load();
 
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(pl.grid);
@@ -1481,6 +1499,14 @@ extern "C" int wq4_chain_plan_destroy(const wq4_layer_table* table)
     if (it == g_plans.end()) return WQ4_ERR_INVALID;
     if (it->second.graph) cudaGraphExecDestroy(it->second.graph);
     g_plans.erase(it);
+    return WQ4_OK;
+}
+
+extern "C" int wq4_test_chain_waits(uint64_t wait_limit_ns, int stall_stage)
+{
+    if (wait_limit_ns == 0 || wait_limit_ns > kWaitTimeoutNs || stall_stage < -1) return WQ4_ERR_INVALID;
+    g_wait_ns.store(wait_limit_ns);
+    g_stall_stage.store(stall_stage);
     return WQ4_OK;
 }
 

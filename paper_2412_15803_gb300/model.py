@@ -9,6 +9,7 @@ computation goes through the C ABI.
 """
 from __future__ import annotations
 
+import weakref
 from dataclasses import dataclass
 
 import numpy as np
@@ -65,6 +66,12 @@ def fill_matrix(W, s, N: int, K: int, seed: int, layer: int, mat: int, symmetric
                         synth.SCALE_LO, synth.SCALE_HI, stream)
 
 
+def _release_plan(table) -> None:
+    import torch
+    torch.cuda.synchronize()          # a batched plan's graph may still run
+    _w.wq4_chain_plan_destroy(table)
+
+
 class DecodeModel:
     """A synthetic decoder resident in device memory plus its wq4 layer table.
 
@@ -112,6 +119,10 @@ class DecodeModel:
         t.workspace = aligned
         t.workspace_bytes = nbytes
         self.table = t
+        # the library caches a plan per table: release it with the model, before
+        # its buffers can come back at the same addresses under another table
+        fin = weakref.finalize(self, _release_plan, t)
+        fin.atexit = False
 
     # --- decoding -------------------------------------------------------
     def decode(self, x, logits, stream=None, check=True) -> int:

@@ -92,6 +92,7 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
     L.wq4_chain_plan_destroy.argtypes = [ctypes.POINTER(wq4_layer_table)]
     L.wq4_chain_trace_offsets.argtypes = [ctypes.POINTER(wq4_layer_table), _I,
                                           ctypes.POINTER(wq4_chain_trace)]
+    L.wq4_test_chain_waits.argtypes = [_U64, _I]
     L.wq4_synth_codes.argtypes = [_P, _I64, _I64, _U64, _U64, _I, _P]
     L.wq4_synth_scales.argtypes = [_P, _I64, _I64, _U64, _U64, ctypes.c_double, ctypes.c_double, _P]
     L.wq4_synth_sum4.argtypes = [_P, _I64, _I64, _U64, _U64, _P]
@@ -108,6 +109,7 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
 EXPORTED = ["wq4_gemv", "wq4_gemm", "wq4_unpack_debug", "wq4_pack_host", "wq4_status_string",
             "wq4_device_status", "wq4_chain_workspace_bytes", "wq4_decode_chain",
             "wq4_decode_chain_host", "wq4_decode_chain_noalloc", "wq4_chain_plan_destroy", "wq4_chain_trace_offsets",
+            "wq4_test_chain_waits",
             "wq4_synth_codes", "wq4_synth_scales", "wq4_synth_sum4",
             "wq4_paged_attention_workspace_bytes", "wq4_paged_attention", "wq4_kv_append"]
 
@@ -202,6 +204,12 @@ def wq4_chain_trace_offsets(table: wq4_layer_table, layer: int) -> wq4_chain_tra
     out = wq4_chain_trace()
     _check("wq4_chain_trace_offsets", load().wq4_chain_trace_offsets(ctypes.byref(table), layer, ctypes.byref(out)))
     return out
+
+
+def wq4_test_chain_waits(wait_limit_ns: int, stall_stage: int = -1) -> None:
+    """Test hook: limit of the chain kernel's device waits and a stage whose
+    input waits are made to run out (-1: none)."""
+    _check("wq4_test_chain_waits", load().wq4_test_chain_waits(wait_limit_ns, stall_stage))
 
 
 def wq4_synth_codes(W, word_start: int, nwords: int, seed: int, sid: int, symmetric: bool = False,

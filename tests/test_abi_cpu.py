@@ -208,3 +208,11 @@ def test_kv_append_rejects_bad_arguments():
     assert L.wq4_kv_append(ctypes.byref(c), 200 * A16 + 8, 210 * A16, 256, 220 * A16, 1, None) == wq4.WQ4_ERR_ALIGN
     c64 = _cache(head_dim=64)
     assert L.wq4_kv_append(ctypes.byref(c64), 200 * A16, 210 * A16, 256, 220 * A16, 1, None) == wq4.WQ4_ERR_UNSUPPORTED
+
+
+def test_chain_wait_hook_rejects_bad_values():
+    lib = wq4.load()
+    assert lib.wq4_test_chain_waits(0, -1) == wq4.WQ4_ERR_INVALID
+    assert lib.wq4_test_chain_waits(500_000_001, -1) == wq4.WQ4_ERR_INVALID
+    assert lib.wq4_test_chain_waits(1000, -2) == wq4.WQ4_ERR_INVALID
+    assert lib.wq4_test_chain_waits(500_000_000, -1) == wq4.WQ4_OK

@@ -279,3 +279,17 @@ def test_small_chain_graph_path_repeat_and_rebuild(batch):
     assert np.array_equal(lh, a)
     model.destroy_plan()
     assert np.array_equal(run(model, x), a)          # a new plan and graph give the same bits
+
+
+@pytest.mark.parametrize("batch", [1, 2, 3])
+def test_cached_plan_on_a_zeroed_workspace(batch):
+    """A table whose workspace was freed and came back zero-filled at the same
+    address (same table contents, so the cached plan is reused without
+    re-initialisation) decodes the same token again: the batch 1-2 kernel
+    takes its weight pointers from the launch, not from the workspace."""
+    model = DecodeModel(TINY, batch=batch, seed=90 + batch)
+    x = synth.activations(91, batch, TINY.hidden)
+    first = run(model, x)
+    model.workspace.zero_()
+    torch.cuda.synchronize()
+    assert np.array_equal(run(model, x), first)

@@ -84,3 +84,23 @@ def test_noalloc_switching_models_and_oversize_rejection():
     out = torch.zeros((4, 128256), dtype=torch.int16, device="cuda")
     rc = wq4.load().wq4_decode_chain_noalloc(ctypes.byref(big), x.data_ptr(), out.data_ptr(), None)
     assert rc == wq4.WQ4_ERR_UNSUPPORTED
+
+
+def test_noalloc_3b_batch2_full_size_sampled():
+    """The largest model shape the array holds at batch 2 (3B: 14.1 MiB):
+    bit-identical to the allocated-workspace chain; LM head rows sampled at
+    the start, middle and end of the vocabulary against the oracle."""
+    sh = SHAPE_3B
+    model = DecodeModel(sh, batch=2, seed=24)
+    assert wq4.wq4_chain_workspace_bytes(model.table) <= 16 << 20
+    x = synth.activations(52, 2, sh.hidden)
+    ref, lm_in, outs = _logits_pair(model, x)
+    for out in outs:
+        assert np.array_equal(out, ref)
+    from oracle import chain as ochain
+    r = ochain.rms_factors(lm_in, model.eps)
+    for r0 in (0, sh.vocab // 2 - 128, sh.vocab - 256):
+        W, s = model.host_rows(sh.num_layers, "lm_head", r0, 256)
+        y, A, _ = oracle.gemv(W, s, lm_in, r)
+        err = np.abs(oracle.half_to_double(ref[:, r0:r0 + 256]) - y)
+        assert np.all(err <= oracle.tolerance(y, A))

@@ -13,6 +13,7 @@ than L2 (129 MB), so no L2 flush is needed between steps.
                     [--workload 3b|8b|phi3.5] [--batch B]
     python bench.py --workload attn-8b|attn-3b|attn-8b-b1     (decode attention)
     python bench.py --workload prefill-3b [--tokens M]         (prefill-shaped GEMMs)
+    python bench.py --workload gemv-2048|gemv-3b-layer         (single wq4_gemv calls)
 
 The attn-* workloads time decode attention of one layer over a paged
 key/value cache instead (wq4_paged_attention, one launch per step): 32
@@ -48,6 +49,7 @@ PERSISTENT_MAX_BATCH = 2      # larger batches run the tensor-core graph path
 # Chrome on an Apple M3 Max, 4-bit weights): another machine's numbers, context only
 PAPER_DECODE_TOKS = {"8b": 41.1, "phi3.5": 71.1}
 FALLBACK_HBM_GBS = 6800.0
+L2_BYTES = 129 * 1024 * 1024
 
 
 def parse():
@@ -56,7 +58,8 @@ def parse():
     ap.add_argument("--steps", type=int, default=2000)
     ap.add_argument("--warmup", type=int, default=20)
     ap.add_argument("--impl", choices=["ours", "reference"], default="ours")
-    ap.add_argument("--workload", choices=["3b", "8b", "phi3.5", "attn-8b", "attn-3b", "attn-8b-b1", "prefill-3b"],
+    ap.add_argument("--workload", choices=["3b", "8b", "phi3.5", "attn-8b", "attn-3b", "attn-8b-b1", "prefill-3b",
+                                           "gemv-2048", "gemv-3b-layer"],
                     default="3b")
     ap.add_argument("--tokens", type=int, default=2048, help="prompt tokens of the prefill workload")
     ap.add_argument("--batch", type=int, default=1)
@@ -164,10 +167,64 @@ class ClockSampler:
 
 # ---------------------------------------------------------------- oracle --
 
-def oracle_sample(shape, batch: int, fraction: float, seed: int = 0):
+def host_info() -> dict:
+    """The host the CPU baselines ran on: cores this process may use, CPU model."""
+    import platform
+    try:
+        nproc = len(os.sched_getaffinity(0))
+    except Exception:
+        nproc = os.cpu_count() or 1
+    model = None
+    try:
+        out = subprocess.run(["lscpu"], capture_output=True, text=True, timeout=10).stdout
+        for line in out.splitlines():
+            if line.strip().lower().startswith("model name"):
+                model = line.split(":", 1)[1].strip()
+                break
+    except Exception:
+        pass
+    if not model:
+        try:
+            with open("/proc/cpuinfo") as f:
+                for line in f:
+                    if line.lower().startswith("model name"):
+                        model = line.split(":", 1)[1].strip()
+                        break
+        except Exception:
+            pass
+    return {"nproc": nproc, "cpu_model": model or "unknown", "machine": platform.machine()}
+
+
+class RowPool:
+    """Runs the oracle's GEMV over row blocks on `threads` threads.  The C
+    routine releases the GIL, so the blocks run on separate cores; every row
+    is computed by the same code as in a single call."""
+
+    def __init__(self, threads: int):
+        from concurrent.futures import ThreadPoolExecutor
+        self.threads = max(1, threads)
+        self.ex = ThreadPoolExecutor(self.threads) if self.threads > 1 else None
+
+    def gemv(self, W, s, x):
+        import oracle
+        N = W.shape[0]
+        if self.ex is None or N < 2 * self.threads:
+            oracle.gemv(W, s, x)
+            return
+        cuts = [N * i // self.threads for i in range(self.threads + 1)]
+        list(self.ex.map(lambda i: oracle.gemv(W[cuts[i]:cuts[i + 1]], s[cuts[i]:cuts[i + 1]], x),
+                         range(self.threads)))
+
+    def close(self):
+        if self.ex is not None:
+            self.ex.shutdown()
+
+
+def oracle_sample(shape, batch: int, fraction: float, seed: int = 0, pool: RowPool | None = None):
     """Times the fp64 oracle on the first ceil(fraction * N) rows of every
-    projection of the chain (all layers and the LM head).  Returns
-    (seconds, weights processed)."""
+    projection of the chain (all layers and the LM head); with a pool, each
+    block's rows are split over its threads.  Returns (seconds, weights
+    processed)."""
     import oracle
     from paper_2412_15803_gb300 import synth
     x = {K: synth.activations(seed, batch, K) for K in {shape.hidden, shape.ffn}}
@@ -181,7 +238,10 @@ def oracle_sample(shape, batch: int, fraction: float, seed: int = 0):
         n = max(1, int(np.ceil(fraction * N)))
         W, s = synth.matrix(seed, N, K, l, mat, 0, n, symmetric=True)
         t0 = time.perf_counter()
-        oracle.gemv(W, s, x[K])
+        if pool is None:
+            oracle.gemv(W, s, x[K])
+        else:
+            pool.gemv(W, s, x[K])
         total_t += time.perf_counter() - t0
         total_w += n * K
     return total_t, total_w
@@ -198,15 +258,28 @@ def oracle_rate_estimate(shape, batch):
     return (time.perf_counter() - t0) / (256 * shape.hidden)
 
 
+def all_core_line(value: float, unit: str, threads: int, sample: str) -> dict:
+    return {"value": value, "unit": unit, "cores": threads,
+            "kind": f"oracle, row-parallel: the same fp64 C routine over {threads} row blocks on {threads} threads",
+            "sample": sample}
+
+
 def cpu_baseline(shape, batch, target_s=12.0):
     per_w = oracle_rate_estimate(shape, batch)
     frac = min(1.0, target_s / max(per_w * shape.weight_count(), 1e-9))
     t, w = oracle_sample(shape, batch, frac)
     tokens = batch * w / shape.weight_count()
+    host = host_info()
+    pool = RowPool(host["nproc"])
+    tp, wp = oracle_sample(shape, batch, frac, pool=pool)
+    pool.close()
     return {"value": tokens / t, "unit": "tokens/s", "cores": 1, "kind": "oracle",
             "sample": f"first {frac:.4f} of the rows of all {4 * shape.num_layers + 1} projections "
                       f"({w} weights = {w / shape.weight_count():.4f} of a token), batch {batch}, "
-                      f"single-threaded fp64 C oracle, {t:.1f} s"}
+                      f"single-threaded fp64 C oracle, {t:.1f} s",
+            **host,
+            "all_core": all_core_line(batch * wp / shape.weight_count() / tp, "tokens/s", pool.threads,
+                                      f"the same rows, {tp:.1f} s")}
 
 
 def chain_step_bytes(shape, B: int) -> int:
@@ -223,6 +296,10 @@ def chain_config(shape, B: int, world: int) -> dict:
                         f"+ LM head {shape.vocab}x{shape.hidden}, batch {B}",
             "batch": B, "bytes_per_token": chain_step_bytes(shape, B),
             "l2": "inputs larger than L2 (1.8+ GB of weights per step), no flush",
+            "codes": "drawn uniform on 0..14 (zero-mean q - 7), not 0..15: with 0..15 the mean offset of "
+                     "+0.5 per weight compounds through 28-32 layers and overflows fp16 in the oracle's own "
+                     "chain; the kernels' work and timing do not depend on the code values, and every code "
+                     "value 0..15 runs through the chain in the full-range parity tests",
             "parallelism": "replicas" if world > 1 else "single GPU"}
 
 
@@ -250,7 +327,8 @@ def run_reference(args, rank, world):
             "config": chain_config(shape, args.batch, world),
             "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
                              "sample": f"each step: first {frac:.5f} of the rows of every projection "
-                                       f"(all {4 * shape.num_layers + 1}), scaled to a token by weights"},
+                                       f"(all {4 * shape.num_layers + 1}), scaled to a token by weights",
+                             **host_info()},
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -379,10 +457,280 @@ def run_ours(args, rank, world, local):
         dist.destroy_process_group()
 
 
+# ------------------------------------------------------------------ gemv --
+
+# Single wq4_gemv calls: one 2048 x 2048 matrix, and the four projections of
+# one 3B-shaped layer, at batch 1; codes uniform on 0..15, scales uniform on
+# [0.005, 0.02], x ~ N(0, 1), seed 0 (copy 0 of the rotation is exactly that
+# matrix set; copy c draws the streams of layer c).
+GEMV_WORKLOADS = {
+    "gemv-2048": [("gemv", 2048, 2048)],
+    "gemv-3b-layer": [("qkv", 5120, 3072), ("o", 3072, 3072), ("gate_up", 16384, 3072), ("down", 3072, 8192)],
+}
+
+
+def gemv_set_bytes(mats) -> int:
+    """Algorithmic bytes of one pass over the set: packed codes + scales
+    (the activations, 2 B per K and N, are added separately)."""
+    return sum(N * K // 2 + N * K // 16 for _, N, K in mats)
+
+
+def gemv_copies(mats) -> int:
+    """Copies of the set in rotation: together more than 4x L2."""
+    return -(-4 * L2_BYTES // gemv_set_bytes(mats)) + 1
+
+
+def gemv_io_bytes(mats, B: int) -> int:
+    return sum(2 * B * (N + K) for _, N, K in mats)
+
+
+def gemv_source_sha() -> str:
+    h = hashlib.sha256()
+    for f in ("wq4_gemv.cu", "wq4_device.cuh"):
+        h.update(open(os.path.join(ROOT, "paper_2412_15803_gb300", "csrc", f), "rb").read())
+    return h.hexdigest()[:16]
+
+
+def gemv_profiled_traffic(workload: str):
+    path = os.path.join(ROOT, "profiles", f"gemv_tma_kernel_{workload}.md")
+    if not os.path.exists(path):
+        return None
+    text = open(path).read()
+    m = re.search(r"traffic_bytes_per_set:\s*(\d+)", text)
+    h = re.search(r"source_sha:\s*([0-9a-f]+)", text)
+    if not m or not h or h.group(1) != gemv_source_sha():
+        return None
+    return int(m.group(1))
+
+
+def gemv_config(workload: str, mats, B: int, copies: int) -> dict:
+    desc = ", ".join(f"{n} {N}x{K}" for n, N, K in mats)
+    return {"workload": f"{workload}: wq4_gemv at batch {B} ({desc}), one launch per matrix",
+            "batch": B, "bytes_per_set": gemv_set_bytes(mats) + gemv_io_bytes(mats, B),
+            "codes": "uniform on 0..15", "scales": "uniform on [0.005, 0.02]", "x": "N(0, 1) fp16",
+            "l2": f"{copies} copies of the set in rotation ({copies * gemv_set_bytes(mats) / 1e6:.0f} MB, more "
+                  "than 4x L2), one CUDA graph replay runs every copy once",
+            "parallelism": "single GPU"}
+
+
+def gemv_oracle_step(mats, B: int, step_s: float, pool: RowPool | None = None):
+    """The oracle on the first rows of every matrix of the set, sized to about
+    step_s seconds.  Returns (seconds, bytes of weights processed)."""
+    import oracle
+    from paper_2412_15803_gb300 import synth
+    W, sc = synth.matrix(0, 64, mats[0][2])
+    x = synth.activations(0, B, mats[0][2])
+    t0 = time.perf_counter()
+    oracle.gemv(W, sc, x)
+    per_w = (time.perf_counter() - t0) / (64 * mats[0][2])
+    total_w = sum(N * K for _, N, K in mats)
+    est = max(per_w * total_w, 1e-9)           # seconds of one whole set
+    frac = min(1.0, step_s / est)
+    reps = max(1, int(step_s / est)) if frac >= 1.0 else 1
+    t, nbytes = 0.0, 0
+    for i, (_, N, K) in enumerate(mats):
+        n = max(1, int(np.ceil(frac * N)))
+        W, sc = synth.matrix(0, N, K, 0, i, 0, n)
+        x = synth.activations(0, B, K)
+        t0 = time.perf_counter()
+        for _ in range(reps):
+            if pool is None:
+                oracle.gemv(W, sc, x)
+            else:
+                pool.gemv(W, sc, x)
+        t += time.perf_counter() - t0
+        nbytes += reps * (n * K // 2 + n * K // 16)
+    what = f"{reps} passes over every matrix" if reps > 1 or frac >= 1.0 else \
+        f"first {frac:.4f} of the rows of every matrix"
+    return t, nbytes, what
+
+
+def run_gemv_reference(args, rank, world):
+    if rank != 0:
+        return
+    mats = GEMV_WORKLOADS[args.workload]
+    B = args.batch
+    nsteps = args.steps + args.warmup
+    step_s = min(5.0, 120.0 / max(nsteps, 1))
+    times, nb, what = [], 0, ""
+    for i in range(nsteps):
+        t, b, what = gemv_oracle_step(mats, B, step_s)
+        if i >= args.warmup:
+            times.append(t)
+            nb += b
+    value = nb / sum(times) / 1e9
+    copies = gemv_copies(mats)
+    step_b = copies * (gemv_set_bytes(mats) + gemv_io_bytes(mats, B))
+    line = {"metric": METRIC, "value": value, "unit": "GB/s", "n_gpus": world, "steps": args.steps,
+            "warmup": args.warmup, "ms_per_step": 1e3 * step_b / (value * 1e9), "higher_is_better": True,
+            "scaling": "weak", "vs_baseline": None, "dtype": "f64",
+            "data": "synthetic (seeded SplitMix64 weights and activations)", "impl": "reference",
+            "config": gemv_config(args.workload, mats, B, copies),
+            "cpu_baseline": {"value": value, "unit": "GB/s", "cores": 1, "kind": "oracle",
+                             "sample": f"each step: {what}, single-threaded fp64 C oracle; ms_per_step "
+                                       f"scales its rate to the {copies} sets of one step",
+                             **host_info()},
+            "e2e": {"value": value, "unit": "GB/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
+    print(json.dumps(line), flush=True)
+
+
+def run_gemv(args, rank, world, local):
+    import torch
+    import torch.distributed as dist
+    from paper_2412_15803_gb300 import synth, wq4
+    from paper_2412_15803_gb300.model import fill_matrix
+
+    torch.cuda.set_device(local)
+    if world > 1:
+        dist.init_process_group("nccl", device_id=torch.device("cuda", local))
+    mats = GEMV_WORKLOADS[args.workload]
+    B = args.batch
+    set_b = gemv_set_bytes(mats)
+    io_b = gemv_io_bytes(mats, B)
+    copies = gemv_copies(mats)
+    weights = []
+    for c in range(copies):
+        ws = []
+        for i, (_, N, K) in enumerate(mats):
+            W = torch.empty((N, K // 8), dtype=torch.int32, device="cuda")
+            sc = torch.empty((N, K // 32), dtype=torch.int16, device="cuda")
+            fill_matrix(W, sc, N, K, 0, c, i, symmetric=False)
+            ws.append((W, sc))
+        weights.append(ws)
+    xs = {K: torch.from_numpy(synth.activations(0, B, K).view(np.int16)).cuda() for _, _, K in mats}
+    ys = [torch.empty((B, N), dtype=torch.int16, device="cuda") for _, N, _ in mats]
+
+    def one_set(c, stream):
+        for i, (_, N, K) in enumerate(mats):
+            W, sc = weights[c][i]
+            wq4.wq4_gemv(W, sc, xs[K], ys[i], N, K, B, stream)
+
+    stream = torch.cuda.Stream()
+    with torch.cuda.stream(stream):
+        one_set(0, stream)
+        stream.synchronize()
+        graph = torch.cuda.CUDAGraph()
+        with torch.cuda.graph(graph, stream=stream):
+            for c in range(copies):
+                one_set(c, stream)
+        for _ in range(max(args.warmup, 3)):
+            graph.replay()
+    torch.cuda.synchronize()
+    if wq4.wq4_device_status(stream) != 0:
+        raise RuntimeError("device flag set during warm-up")
+
+    starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
+    sampler = ClockSampler(local)
+    sampler.start()
+    time.sleep(0.3)
+    if world > 1:
+        dist.barrier()
+    torch.cuda.synchronize()
+    with torch.cuda.stream(stream):
+        for i in range(args.steps):
+            starts[i].record(stream)
+            graph.replay()
+            ends[i].record(stream)
+    torch.cuda.synchronize()
+    if world > 1:
+        dist.barrier()
+    clocks = sampler.stop()
+    total_ms = starts[0].elapsed_time(ends[-1])
+    replay_ms = [s.elapsed_time(e) for s, e in zip(starts, ends)]
+
+    # single-set latency, one launch per matrix from a cold L2 (a 2x L2 buffer
+    # is written before each), and the same warm (the set just ran)
+    flush = torch.empty(2 * L2_BYTES, dtype=torch.uint8, device="cuda")
+    cold, warm = [], []
+    with torch.cuda.stream(stream):
+        for rep in range(20):
+            flush.fill_(rep & 0xFF)
+            e0, e1, e2 = (torch.cuda.Event(enable_timing=True) for _ in range(3))
+            e0.record(stream)
+            one_set(0, stream)
+            e1.record(stream)
+            one_set(0, stream)
+            e2.record(stream)
+            stream.synchronize()
+            cold.append(e0.elapsed_time(e1))
+            warm.append(e1.elapsed_time(e2))
+    del flush
+
+    # end to end through the C ABI call: x from pinned host memory, the set's
+    # GEMVs, y back to pinned host memory, every step
+    x_host = {K: v.cpu().pin_memory() for K, v in xs.items()}
+    y_host = [torch.empty_like(y, device="cpu").pin_memory() for y in ys]
+    e2e_steps = max(20, min(args.steps * copies, 2000))
+    with torch.cuda.stream(stream):
+        for i in range(e2e_steps + 5):
+            if i == 5:
+                t0 = time.perf_counter()
+            for K, v in xs.items():
+                v.copy_(x_host[K], non_blocking=True)
+            one_set(i % copies, stream)
+            for y, yh in zip(ys, y_host):
+                yh.copy_(y, non_blocking=True)
+            stream.synchronize()
+        e2e_s = (time.perf_counter() - t0) / e2e_steps
+    if wq4.wq4_device_status(stream) != 0:
+        raise RuntimeError("device flag set during the timed region")
+    t = torch.tensor([total_ms, e2e_s], dtype=torch.float64, device="cuda")
+    if world > 1:
+        dist.all_reduce(t, op=dist.ReduceOp.MAX)
+    job_ms, e2e_step = float(t[0]), float(t[1])
+    if rank == 0:
+        peak, src = measured_peak()
+        per_set_ms = statistics.mean(replay_ms) / copies
+        step_bytes = set_b + io_b
+        achieved = step_bytes / (per_set_ms * 1e-3) / 1e9
+        traffic = gemv_profiled_traffic(args.workload)
+        line = {
+            "metric": METRIC, "value": world * step_bytes * copies * args.steps / (job_ms * 1e-3) / 1e9,
+            "unit": "GB/s", "n_gpus": world, "steps": args.steps, "warmup": args.warmup,
+            "ms_per_step": job_ms / args.steps, "higher_is_better": True, "scaling": "weak",
+            "vs_baseline": None, "dtype": "f32",
+            "precision": "int4 codes (group 32, fp16 scale, zero point 7), fp16 activations, fp32 accumulation",
+            "data": "synthetic (seeded SplitMix64 weights and activations)",
+            "config": gemv_config(args.workload, mats, B, copies),
+            "step": f"one CUDA graph replay: {copies} sets x {len(mats)} launches",
+            "per_set_us": per_set_ms * 1e3,
+            "per_launch_us": per_set_ms * 1e3 / len(mats),
+            "single_set_latency_us": {"cold_l2_median": 1e3 * statistics.median(cold),
+                                      "warm_l2_median": 1e3 * statistics.median(warm),
+                                      "launches": len(mats)},
+            "hbm_frac_of_nominal_8tbs": achieved / NOMINAL_HBM_GBS,
+            "roofline": {"bound": "hbm", "kernel": "gemv_tma_kernel", "achieved": achieved, "peak": peak,
+                         "peak_source": src, "unit": "GB/s", "frac": achieved / peak,
+                         "traffic": traffic, "traffic_unit": "bytes per set (ncu, cold L2)",
+                         "algorithmic_bytes_per_set": step_bytes, "avg_set_ms": per_set_ms},
+            "e2e": {"value": step_bytes / e2e_step / 1e9, "unit": "GB/s",
+                    "h2d_bytes_per_step": sum(2 * B * K for K in xs),
+                    "d2h_bytes_per_step": sum(2 * B * N for _, N, _ in mats),
+                    "step": "one set through wq4_gemv with host copies"},
+            "gpu_launches": args.steps * copies * len(mats),
+            "clocks": clocks,
+        }
+        if world == 1 and not args.no_cpu_baseline:
+            t1, b1, what = gemv_oracle_step(mats, B, 10.0)
+            host = host_info()
+            pool = RowPool(host["nproc"])
+            tp, bp, what_p = gemv_oracle_step(mats, B, 10.0 * min(pool.threads, 8), pool)
+            pool.close()
+            line["cpu_baseline"] = {
+                "value": b1 / t1 / 1e9, "unit": "GB/s", "cores": 1, "kind": "oracle",
+                "sample": f"{what}, single-threaded fp64 C oracle, {t1:.1f} s",
+                **host,
+                "all_core": all_core_line(bp / tp / 1e9, "GB/s", pool.threads,
+                                          f"{what_p}, {tp:.1f} s")}
+        print(json.dumps(line), flush=True)
+    if world > 1:
+        dist.destroy_process_group()
+
+
 # -------------------------------------------------------------- attention --
 
 ATTN_METRIC = "paged decode attention sequences/s (one decode step per sequence) and achieved HBM GB/s"
-L2_BYTES = 129 * 1024 * 1024
 
 
 def attn_source_sha() -> str:
@@ -404,10 +752,12 @@ def attn_profiled_traffic(workload: str):
     return int(m.group(1))
 
 
-def attn_oracle_sample(w, seed: int, target_s: float):
+def attn_oracle_sample(w, seed: int, target_s: float, threads: int = 1, nseq_fixed: int = 0):
     """Times the fp64 oracle on whole sequences of the workload (shortest
     first, sequences regenerated on the host) until about target_s seconds
-    have been spent; returns (seconds, tokens of context processed, sequences)."""
+    have been spent, or on the first nseq_fixed sequences spread over
+    `threads` threads; returns (seconds, tokens of context processed,
+    sequences)."""
     import oracle
     from paper_2412_15803_gb300 import synth
     sh = w.shape
@@ -416,8 +766,7 @@ def attn_oracle_sample(w, seed: int, target_s: float):
     num_pages = int(((lens.astype(np.int64) + P - 1) // P).sum())
     table = synth.page_table(seed, lens, P, num_pages)
     per = sh.n_kv_heads * P * D
-    spent, toks, nseq = 0.0, 0, 0
-    for b in np.argsort(lens, kind="stable"):
+    def inputs(b):
         T = int(lens[b])
         n = (T + P - 1) // P
         pages = table[b, :n]
@@ -426,11 +775,30 @@ def attn_oracle_sample(w, seed: int, target_s: float):
         k = k.reshape(n, sh.n_kv_heads, P, D)
         v = v.reshape(n, sh.n_kv_heads, P, D)
         q = synth.sum4_fp16(seed, synth.stream_id(synth.KIND_Q, 0, 0), int(b) * sh.n_q_heads * D, sh.n_q_heads * D)
-        t0 = time.perf_counter()
+        return q, k, v, n, T
+
+    def call(a):
+        q, k, v, n, T = a
         oracle.paged_attention(q[None, :], k, v, np.arange(n, dtype=np.int32)[None, :], np.array([T], np.int32),
                                1.0 / np.sqrt(D), sh.n_q_heads)
+
+    order = np.argsort(lens, kind="stable")
+    if threads > 1 and nseq_fixed:
+        # the same sequences, one per thread at a time (the C routine releases the GIL)
+        from concurrent.futures import ThreadPoolExecutor
+        args = [inputs(b) for b in order[:nseq_fixed]]
+        with ThreadPoolExecutor(threads) as ex:
+            t0 = time.perf_counter()
+            list(ex.map(call, args))
+            spent = time.perf_counter() - t0
+        return spent, sum(a[4] for a in args), len(args)
+    spent, toks, nseq = 0.0, 0, 0
+    for b in order:
+        a = inputs(b)
+        t0 = time.perf_counter()
+        call(a)
         spent += time.perf_counter() - t0
-        toks += T
+        toks += a[4]
         nseq += 1
         if spent >= target_s:
             break
@@ -441,9 +809,19 @@ def attn_cpu_line(w, seed: int, target_s: float):
     t, toks, nseq = attn_oracle_sample(w, seed, target_s)
     total_toks = int(w.lens(seed).astype(np.int64).sum())
     est = t * total_toks / max(toks, 1)
-    return {"value": w.batch / est, "unit": "sequences/s", "cores": 1, "kind": "oracle",
+    host = host_info()
+    line = {"value": w.batch / est, "unit": "sequences/s", "cores": 1, "kind": "oracle",
             "sample": f"{nseq} of the {w.batch} sequences (shortest first, {toks} of {total_toks} context "
-                      f"tokens), single-threaded fp64 C oracle, {t:.1f} s, scaled to the whole batch"}
+                      f"tokens), single-threaded fp64 C oracle, {t:.1f} s, scaled to the whole batch", **host}
+    threads = host["nproc"]
+    if threads > 1 and nseq >= 2:
+        tp, toksp, nseqp = attn_oracle_sample(w, seed, target_s, threads=threads, nseq_fixed=nseq)
+        line["all_core"] = {"value": w.batch / (tp * total_toks / max(toksp, 1)), "unit": "sequences/s",
+                            "cores": threads,
+                            "kind": f"oracle, sequence-parallel: the same fp64 C routine, one sequence per "
+                                    f"thread on {threads} threads",
+                            "sample": f"the same {nseqp} sequences, {tp:.1f} s, scaled to the whole batch"}
+    return line
 
 
 def attn_config(w, layers: int):
@@ -478,7 +856,7 @@ def run_attn_reference(args, rank, world):
             "config": attn_config(w, 1),
             "cpu_baseline": {"value": value, "unit": "sequences/s", "cores": 1, "kind": "oracle",
                              "sample": f"each step: shortest sequences first for about {step_s:.1f} s of oracle "
-                                       "time, scaled to the whole batch"},
+                                       "time, scaled to the whole batch", **host_info()},
             "e2e": {"value": value, "unit": "sequences/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -634,7 +1012,8 @@ def run_prefill_reference(args, rank, world):
             "data": "synthetic (seeded SplitMix64 weights and activations)", "impl": "reference",
             "config": {"workload": f"prefill-3b: QKV, O, gate_up, down of one 3B-shaped layer over {M} tokens"},
             "cpu_baseline": {"value": value, "unit": "TFLOP/s", "cores": 1, "kind": "oracle",
-                             "sample": "a few rows of every projection against up to 64 tokens, single-threaded fp64 C oracle"},
+                             "sample": "a few rows of every projection against up to 64 tokens, single-threaded fp64 C oracle",
+                             **host_info()},
             "e2e": {"value": value, "unit": "TFLOP/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
 
@@ -766,10 +1145,25 @@ def run_prefill(args, rank, world, local):
                 oracle.gemv(W, sc, xs)
                 n += 1
             dt = time.perf_counter() - t0
+            host = host_info()
+            pool = RowPool(host["nproc"])
+            rows = 16 * pool.threads
+            Wp, scp = synth.matrix(0, rows, shape.hidden)
+            t0 = time.perf_counter()
+            npar = 0
+            while time.perf_counter() - t0 < 5.0:
+                pool.gemv(Wp, scp, xs)
+                npar += 1
+            dtp = time.perf_counter() - t0
+            pool.close()
             line["cpu_baseline"] = {"value": n * 2 * 16 * shape.hidden * 64 / dt / 1e12, "unit": "TFLOP/s", "cores": 1,
                                     "kind": "oracle",
                                     "sample": f"16 rows x {shape.hidden} x 64 tokens repeated for {dt:.1f} s, "
-                                              "single-threaded fp64 C oracle"}
+                                              "single-threaded fp64 C oracle", **host,
+                                    "all_core": all_core_line(npar * 2 * rows * shape.hidden * 64 / dtp / 1e12,
+                                                              "TFLOP/s", pool.threads,
+                                                              f"{rows} rows x {shape.hidden} x 64 tokens repeated "
+                                                              f"for {dtp:.1f} s")}
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()
@@ -778,6 +1172,9 @@ def run_prefill(args, rank, world, local):
 def main():
     args = parse()
     rank, world, local = dist_env()
+    if args.workload.startswith("gemv"):
+        (run_gemv_reference(args, rank, world) if args.impl == "reference" else run_gemv(args, rank, world, local))
+        return
     if args.workload.startswith("prefill"):
         (run_prefill_reference(args, rank, world) if args.impl == "reference" else run_prefill(args, rank, world, local))
         return

@@ -175,6 +175,30 @@ def rms_normalize(u, eps: float) -> np.ndarray:
     return v
 
 
+def rope(x, positions, head_dim: int, theta: float):
+    """Rotary position embedding of the heads of each row (the paper names no
+    positional encoding; its models, Llama-3.1 and Phi-3.5, rotate q and k).
+    Reading: within each head, the adjacent pair (x_2i, x_2i+1) is the
+    complex number x_2i + i x_2i+1 multiplied by exp(i pos w_i), with
+    w_i = theta^(-2i / head_dim) and pos = positions[b] (the token's place in
+    its sequence).  Inputs are fp16 bits [batch][n_heads * head_dim]; the
+    rotation is exact in fp64 on the fp16 values and rounded once.
+
+    Returns (fp64 [batch][n], fp16 bits [batch][n])."""
+    x = np.atleast_2d(_c(x, np.uint16))
+    batch, n = x.shape
+    assert n % head_dim == 0 and head_dim % 2 == 0
+    pos = np.asarray(positions, np.float64).reshape(batch, 1, 1)
+    i = np.arange(head_dim // 2, dtype=np.float64)
+    w = np.power(float(theta), -2.0 * i / head_dim)            # [head_dim / 2]
+    ang = pos * w[None, None, :]                                # [batch][1][head_dim / 2]
+    c, s = np.cos(ang), np.sin(ang)
+    v = half_to_double(x).reshape(batch, n // head_dim, head_dim // 2, 2)
+    re, im = v[..., 0], v[..., 1]
+    out = np.stack([re * c - im * s, re * s + im * c], axis=-1).reshape(batch, n)
+    return out, double_to_half(out)
+
+
 def silu_mul(g, u):
     """-> (m fp64, m16 fp16 bits) with m = silu(g) * u."""
     g = _c(g, np.uint16)

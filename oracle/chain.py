@@ -4,9 +4,15 @@ TEST INFRASTRUCTURE ONLY (see the package docstring).
 
 The paper's workload is token decoding of 4-bit quantized transformer models
 (Section 3, Table 1); the weight stream of every projection of every layer is
-read once per token.  Attention itself (PagedAttention / FlashAttention,
-Section 2.3) is not part of this chain: the query block of the fused QKV
-output stands in for the attention output.
+read once per token.  Without an attention description (``attn=None``) the
+query block of the fused QKV output stands in for the attention output;
+with one, each layer runs the decode step's attention (PagedAttention /
+FlashAttention, Section 2.3) on rotary-embedded queries and keys:
+
+    q, k = rope(qkv[:, :H]), rope(qkv[:, H:H + Hkv D])    fp16, see oracle.rope
+    v    = qkv[:, H + Hkv D:]
+    the cache of the layer gets k, v at positions[b]     (oracle.kv_append)
+    a    = fp16( attention(q, cache, positions + 1) )    (oracle.paged_attention)
 
 Layer l takes u (fp16 [batch][H]: the token input for l = 0, else the previous
 layer's output) and re-feeds it after RMS normalisation; every stage output
@@ -36,7 +42,7 @@ from __future__ import annotations
 
 import numpy as np
 
-from . import add_fp16, gemv, rms_factor, rms_normalize, silu_mul
+from . import add_fp16, gemv, kv_append, paged_attention, rms_factor, rms_normalize, rope, silu_mul
 
 
 def rms_factors(v, eps):
@@ -44,8 +50,29 @@ def rms_factors(v, eps):
     return np.array([rms_factor(row, eps) for row in v])
 
 
-def layer(u, w, H: int, F: int, eps: float):
-    """One layer.  w = dict(qkv=(W, s), o=..., gate_up=..., down=...).
+def attention_step(qkv, H: int, attn: dict, t: dict):
+    """The decode step's attention of one layer (see the module docstring).
+
+    attn: n_q_heads, n_kv_heads, head_dim, theta, scale, positions (int32
+    [batch]), and this layer's k_cache, v_cache (modified in place) and
+    page_table.  Returns a (fp16 bits [batch][H]) and records the steps in t."""
+    D, Hkv, nq = attn["head_dim"], attn["n_kv_heads"], attn["n_q_heads"]
+    pos = np.asarray(attn["positions"], np.int32)
+    q64, q = rope(np.ascontiguousarray(qkv[:, :H]), pos, D, attn["theta"])
+    k64, k = rope(np.ascontiguousarray(qkv[:, H:H + Hkv * D]), pos, D, attn["theta"])
+    v = np.ascontiguousarray(qkv[:, H + Hkv * D:H + 2 * Hkv * D])
+    kv_append(k, v, attn["k_cache"], attn["v_cache"], attn["page_table"], pos)
+    o, A, o16 = paged_attention(q, attn["k_cache"], attn["v_cache"], attn["page_table"], pos + 1,
+                                attn["scale"], nq)
+    a = o16.reshape(qkv.shape[0], H)
+    t.update(q_rot=q, q_rot_ref=q64, k_rot=k, k_rot_ref=k64, v_new=v, attn=a, attn_ref=o.reshape(a.shape),
+             attn_A=A.reshape(a.shape))
+    return a
+
+
+def layer(u, w, H: int, F: int, eps: float, attn: dict | None = None):
+    """One layer.  w = dict(qkv=(W, s), o=..., gate_up=..., down=...); attn as
+    attention_step's, or None for the stand-in.
 
     Returns (x2, trace) where trace holds every stage's fp16 output and the
     fp64 values with their magnitudes A for the projections."""
@@ -55,7 +82,10 @@ def layer(u, w, H: int, F: int, eps: float):
     t["v"] = v
     y, A, qkv = gemv(*w["qkv"], u, r1)
     t.update(r_u=r1, qkv=qkv, qkv_ref=y, qkv_A=A)
-    a = np.ascontiguousarray(qkv[:, :H])
+    if attn is None:
+        a = np.ascontiguousarray(qkv[:, :H])
+    else:
+        a = attention_step(qkv, H, attn, t)
     r2 = rms_factors(a, eps)
     y, A, o = gemv(*w["o"], a, r2)
     t.update(r_a=r2, o=o, o_ref=y, o_A=A)
@@ -73,13 +103,14 @@ def layer(u, w, H: int, F: int, eps: float):
     return x2, t
 
 
-def token(x, layers, lm_head, H: int, F: int, eps: float):
-    """Whole token: all layers, final RMS normalisation and LM head.
+def token(x, layers, lm_head, H: int, F: int, eps: float, attn: list | None = None):
+    """Whole token: all layers, final RMS normalisation and LM head; attn:
+    one attention_step description per layer, or None for the stand-in.
 
     Returns (logits fp16 bits, logits fp64, traces)."""
     traces = []
-    for w in layers:
-        x, t = layer(x, w, H, F, eps)
+    for l, w in enumerate(layers):
+        x, t = layer(x, w, H, F, eps, None if attn is None else attn[l])
         traces.append(t)
     rf = rms_factors(x, eps)
     y, A, logits = gemv(*lm_head, x, rf)

@@ -17,11 +17,13 @@ from concurrent.futures import ThreadPoolExecutor
 import pytest
 
 ROOT = os.path.dirname(os.path.dirname(os.path.abspath(__file__)))
-PIN_SUITES = ["tests/test_oracle_pins.py", "tests/test_synth_and_golden.py", "tests/test_attention_oracle.py"]
+PIN_SUITES = ["tests/test_oracle_pins.py", "tests/test_synth_and_golden.py", "tests/test_attention_oracle.py",
+              "tests/test_rope_oracle.py"]
 
 G = "oracle/wq4_oracle.c"
 AT = "oracle/attention_oracle.c"
 CH = "oracle/chain.py"
+PY = "oracle/__init__.py"
 
 # (name, file, text, replacement, occurrence of the text: None = it must be unique)
 MUTANTS = [
@@ -90,6 +92,27 @@ MUTANTS = [
      "const uint16_t* vt = cache_row(v_cache, n_kv_heads, page_size, head_dim, 0, h, t % page_size);", None),
     ("append row shifted", AT, "pos % page_size) * head_dim", "(pos + 1) % page_size) * head_dim", None),
     ("append copies head 0 everywhere", AT, "(int64_t)h * head_dim;", "(int64_t)0 * head_dim;", None),
+    # rotary embedding
+    ("RoPE cross-term sign", PY, "re * c - im * s", "re * c + im * s", None),
+    ("RoPE frequency exponent halved", PY, "-2.0 * i / head_dim", "-1.0 * i / head_dim", None),
+    ("RoPE rotate-half pairing", PY,
+     "v = half_to_double(x).reshape(batch, n // head_dim, head_dim // 2, 2)",
+     "v = half_to_double(x).reshape(batch, n // head_dim, 2, head_dim // 2).swapaxes(-1, -2)", None),
+    ("RoPE position of row 0 for every row", PY,
+     "pos = np.asarray(positions, np.float64).reshape(batch, 1, 1)",
+     "pos = np.full((batch, 1, 1), float(np.asarray(positions).reshape(-1)[0]))", None),
+    ("RoPE position off by one", PY, "pos = np.asarray(positions, np.float64)",
+     "pos = 1.0 + np.asarray(positions, np.float64)", None),
+    # the chain's attention step
+    ("queries not rotated", CH, 'q64, q = rope(np.ascontiguousarray(qkv[:, :H]), pos, D, attn["theta"])',
+     'q = np.ascontiguousarray(qkv[:, :H]); q64 = None', None),
+    ("keys not rotated", CH, 'k64, k = rope(np.ascontiguousarray(qkv[:, H:H + Hkv * D]), pos, D, attn["theta"])',
+     'k = np.ascontiguousarray(qkv[:, H:H + Hkv * D]); k64 = None', None),
+    ("values from the key block", CH, "v = np.ascontiguousarray(qkv[:, H + Hkv * D:H + 2 * Hkv * D])",
+     "v = np.ascontiguousarray(qkv[:, H:H + Hkv * D])", None),
+    ("sequence without the new token", CH, "pos + 1,", "pos,", None),
+    ("O on the query block", CH, "a = attention_step(qkv, H, attn, t)",
+     "attention_step(qkv, H, attn, t); a = np.ascontiguousarray(qkv[:, :H])", None),
 ]
 
 

@@ -282,7 +282,10 @@ int wq4_chain_plan_destroy(const wq4_layer_table* table);
  * Byte offsets into the workspace of the plain fp16 copies of one layer's
  * stage outputs, each [batch][len] row-major, for inspection after a call
  * (layer in [0, num_layers)); layer == num_layers gives the LM head's input
- * in x_in and 0 in the other fields.
+ * in x_in and 0 in the other fields.  q_rot, k_rot and attn are written only
+ * by wq4_decode_step and lie beyond wq4_chain_workspace_bytes (inside
+ * wq4_decode_step_workspace_bytes); they are 0 when the table's heads do not
+ * allow the decode step.
  */
 typedef struct {
     size_t x_in;     /* [batch][hidden]  v: layer input after RMS norm */
@@ -293,6 +296,9 @@ typedef struct {
     size_t act;      /* [batch][ffn]     silu(gate) * up              */
     size_t down;     /* [batch][hidden]  down projection              */
     size_t x_out;    /* [batch][hidden]  x2: layer output (not normalised) */
+    size_t q_rot;    /* [batch][hidden]  rotated queries (decode step)   */
+    size_t k_rot;    /* [batch][n_kv_heads*head_dim] rotated keys (idem) */
+    size_t attn;     /* [batch][hidden]  attention output = O input (idem) */
 } wq4_chain_trace;
 
 int wq4_chain_trace_offsets(const wq4_layer_table* table, int layer, wq4_chain_trace* out);

@@ -32,6 +32,8 @@
 #include <stddef.h>
 #include <stdint.h>
 
+#include "wq4.h"
+
 #ifdef __cplusplus
 extern "C" {
 #endif
@@ -102,6 +104,73 @@ int wq4_paged_attention(const wq4_kv_cache* cache, const uint16_t* q, int q_stri
  */
 int wq4_kv_append(const wq4_kv_cache* cache, const uint16_t* new_k, const uint16_t* new_v, int new_stride,
                   const int32_t* positions, int batch, void* stream);
+
+/* ------------------------------------------------------------------------ */
+/* Decode step with attention                                               */
+/* ------------------------------------------------------------------------ */
+
+/*
+ * The attention of one decode step (Section 2.3: the compiled models run
+ * PagedAttention and FlashAttention between their projections).  The paper
+ * names no positional encoding; its models (Llama-3.1, Phi-3.5) rotate q and
+ * k, and this library's reading of that rotation is: within each head the
+ * adjacent pair (x_2i, x_2i+1) turns by pos * rope_theta^(-2i / head_dim),
+ * computed in fp64 on the fp16 values and rounded once to fp16.
+ *   layers     : HOST array of num_layers caches (device pointers inside),
+ *                all with the table's n_kv_heads, head_dim 128 and one common
+ *                page_size (a multiple of 16); page tables [batch][stride].
+ *                Sequences of a batch must not map their new positions to
+ *                the same cache row.
+ *   positions  : device int32 [batch]: the new token's place in its sequence
+ *                (the number of tokens already cached).
+ *   rope_theta : rotary base (> 1; Llama-3.x 500000, Phi-3.5 10000).
+ *   scale      : attention score scale (> 0, normally 1/sqrt(head_dim)).
+ */
+typedef struct {
+    const wq4_kv_cache* layers;
+    const int32_t* positions;
+    double rope_theta;
+    float scale;
+} wq4_decode_attn;
+
+/* Workspace bytes (table->workspace_bytes) wq4_decode_step needs: the chain's
+ * workspace plus the attention buffers (for batch 3-32 it includes
+ * wq4_paged_attention's workspace, which depends on the current device).
+ * 0 if the table is invalid or its heads are unsupported (head_dim != 128,
+ * n_q_heads / n_kv_heads not a whole number <= 8). */
+size_t wq4_decode_step_workspace_bytes(const wq4_layer_table* table);
+
+/*
+ * One decode step of every sequence of the batch: the chain of wq4_decode_chain
+ * with the query-block stand-in replaced by attention.  For layer l and row b,
+ * after the QKV projection:
+ *   q = rope(qkv[:, :H]), k = rope(qkv[:, H:H + Hkv*128]), v = qkv[:, H + Hkv*128:]
+ *   layers[l] gets k, v at position positions[b] (as wq4_kv_append)
+ *   a = fp16( attention(q, layers[l], positions[b] + 1 tokens) )
+ * and a is the O projection's input (o = r(a) W_o . a).  Batch 1-2 runs the
+ * attention inside the persistent chain kernel (split over the GPU's blocks,
+ * fp32 scores and softmax); batch 3-32 records wq4_paged_attention and a
+ * rotation/append kernel into its CUDA graph.  Accuracy: rotated q and k
+ * within one fp16 ulp of the exact rotation of the fp16 projection outputs;
+ * a within the attention contract of wq4_paged_attention; the projections as
+ * in wq4_decode_chain.  Device-side problems are flagged in the status word
+ * (bit 5: a position or page id that makes the append impossible, nothing
+ * written; bit 3: a length beyond the page table, clamped; bit 4: a page id
+ * outside the pool, zeros read).  The plan is built at the first call (and
+ * rebuilt when the table or this description changes) as for
+ * wq4_decode_chain; table->workspace must hold
+ * wq4_decode_step_workspace_bytes(table) bytes.
+ * Returns WQ4_OK, WQ4_ERR_INVALID, WQ4_ERR_ALIGN, WQ4_ERR_UNSUPPORTED or
+ * WQ4_ERR_CUDA.
+ */
+int wq4_decode_step(const wq4_layer_table* table, const wq4_decode_attn* attn, const uint16_t* x,
+                    uint16_t* logits, void* stream);
+
+/* The same step with HOST buffers (x_host fp16 [batch][hidden], logits_host
+ * fp16 [batch][vocab]): copies x in, runs the step, copies the logits out and
+ * synchronizes `stream`. */
+int wq4_decode_step_host(const wq4_layer_table* table, const wq4_decode_attn* attn, const uint16_t* x_host,
+                         uint16_t* logits_host, void* stream);
 
 #ifdef __cplusplus
 }

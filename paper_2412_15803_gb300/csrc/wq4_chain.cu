@@ -40,13 +40,16 @@
 #include "wq4_host.h"
 #include "wq4_tc_host.h"
 #include "wq4.h"
+#include "wq4_attn.h"
 
 #include <cuda_runtime.h>
 
+#include <algorithm>
 #include <cmath>
 #include <cstring>
 #include <atomic>
 #include <map>
+#include <type_traits>
 #include <mutex>
 #include <vector>
 
@@ -136,6 +139,47 @@ struct ChainParams {
     DevMat mats[4 * kChainMaxLayers + 1];   // [4L + 1]: per layer qkv, o, gate_up, down; then lm_head
 };
 static_assert(sizeof(ChainParams) <= 32764, "kernel parameter space");
+
+// ------------------------------------------------- decode step (attention) --
+//
+// With attention (wq4_decode_step) the QKV epilogue rotates q and k (rotary
+// embedding, adjacent pairs, fp64 rotation of the fp16 outputs), appends the
+// new k and v to the layer's paged cache and publishes them as flagged words;
+// at the start of the O stage every CTA computes its splits of the decode
+// attention (a (row, kv head, token range) each, fp32 online softmax over the
+// cached tokens plus the new one), the last split of each (row, kv head) to
+// arrive merges the partials and publishes the attention output, which the O
+// stage stages in place of the query block.
+constexpr int kAttnD = 128;          // head dimension
+constexpr int kAttnMaxGroup = 8;     // query heads per kv head
+constexpr int kAttnMaxSplits = 32;   // token ranges per (row, kv head)
+constexpr int kAttnPart = kAttnD + 4;   // floats of one split partial: o[128], m, l, pad
+
+struct KvLayer {
+    uint16_t* k;          // [num_pages][Hkv][P][128]
+    uint16_t* v;
+    const int32_t* pt;    // [B][pt_stride]
+    int pt_stride, num_pages;
+};
+
+struct ChainParamsA : ChainParams {
+    int Hkv, G, P, S;              // kv heads, query heads per kv head, page size, splits per (row, kv head)
+    float scale;                   // score scale
+    const int32_t* positions;      // [B] place of the new token
+    uint64_t* llK;                 // [L][B][Hkv 128 / 2] the new token's rotated keys (flagged)
+    uint64_t* llVn;                // [L][B][Hkv 128 / 2] its values (flagged)
+    uint64_t* llAt;                // [L][B][H / 2] attention output (flagged), two replicas
+    uint32_t repAt;
+    uint32_t rope_off;             // shared-memory byte offset of the rotation table and positions
+    uint16_t* pQr;                 // [L][B][H] rotated queries
+    uint16_t* pKr;                 // [L][B][Hkv 128] rotated keys
+    uint16_t* pAt;                 // [L][B][H] attention output
+    float* apart;                  // [L][B][Hkv][S][G][kAttnPart] split partials
+    uint32_t* acnt;                // [L][B][Hkv] splits arrived
+    double inv_freq[kAttnD / 2];   // theta^(-2i / 128)
+    KvLayer kv[kChainMaxLayers];
+};
+static_assert(sizeof(ChainParamsA) <= 32764, "kernel parameter space");
 
 // One stage: N output rows of K codes, `words` output words of rpw rows each
 // (gate_up: gate rows 2w, 2w+1 and up rows F+2w, F+2w+1; the LM head's last
@@ -501,8 +545,279 @@ __device__ __forceinline__ void word_epilogue(const ChainParams& p, const Stage&
     }
 }
 
+// fp16 bits of v rounded once (round to nearest even) from fp64.
+__device__ __forceinline__ uint16_t double_to_half_bits(double v)
+{
+    uint16_t h;
+    asm("cvt.rn.f16.f64 %0, %1;" : "=h"(h) : "d"(v));
+    return h;
+}
+
+// The new token's cache row of kv head `kh` (of Hkv, pages of P tokens) in
+// `pool` for batch row b, or null when its position or page id is outside
+// the page table.
+__device__ __forceinline__ uint16_t* append_row(const KvLayer& kv, int P, int Hkv, uint16_t* pool, int b, int pos, int kh)
+{
+    if (pos < 0) return nullptr;
+    const int pi = pos / P;
+    if (pi >= kv.pt_stride) return nullptr;
+    const int page = kv.pt[static_cast<size_t>(b) * kv.pt_stride + pi];
+    if (page < 0 || page >= kv.num_pages) return nullptr;
+    return pool + ((static_cast<size_t>(page) * Hkv + kh) * P + (pos - pi * P)) * kAttnD;
+}
+
+// QKV epilogue of the decode step for word w (rows n = 2w, 2w + 1) of batch
+// row b: the plain fp16 output for the trace; q and k pairs rotated by the
+// token's angle (rope: cos, sin of pos * theta^(-2i/128) for i = (n % 128) / 2),
+// q published for the attention, k and v appended to the cache and published
+// as the new token's key and value.
+template <int B>
+__device__ __noinline__ void qkv_epilogue_attn(const ChainParamsA& p, int l, int w, int b, float v0, float v1,
+                                                  float rf, uint32_t epoch, const double2* rope, const int* pos_sh)
+{
+    const int H = p.H, n = 2 * w, KD = p.Hkv * kAttnD;
+    const uint16_t h0 = float_to_half_bits(rf * v0), h1 = float_to_half_bits(rf * v1);
+    *reinterpret_cast<uint32_t*>(p.pQKV + (static_cast<size_t>(l) * B + b) * p.Nqkv + n) = pack2(h0, h1);
+    const int pos = pos_sh[b];
+    if (n < H + KD) {
+        const double2 cs = rope[b * (kAttnD / 2) + ((n & (kAttnD - 1)) >> 1)];
+        const double a = half_bits_to_float(h0), c = half_bits_to_float(h1);
+        const uint32_t rw = pack2(double_to_half_bits(a * cs.x - c * cs.y), double_to_half_bits(a * cs.y + c * cs.x));
+        if (n < H) {
+            *reinterpret_cast<uint32_t*>(p.pQr + (static_cast<size_t>(l) * B + b) * H + n) = rw;
+            ll_store2(p.llA + (static_cast<size_t>(l) * B + b) * (H / 2) + w, p.rep.A, rw, epoch);
+        } else {
+            const int kn = n - H;
+            *reinterpret_cast<uint32_t*>(p.pKr + (static_cast<size_t>(l) * B + b) * KD + kn) = rw;
+            ll_store(p.llK + (static_cast<size_t>(l) * B + b) * (KD / 2) + kn / 2, rw, epoch);
+            uint16_t* row = append_row(p.kv[l], p.P, p.Hkv, p.kv[l].k, b, pos, kn / kAttnD);
+            if (row) *reinterpret_cast<uint32_t*>(row + (kn & (kAttnD - 1))) = rw;
+            else if ((kn & (kAttnD - 1)) == 0) atomicOr(p.err, kErrAppend);
+        }
+    } else {
+        const int vn = n - H - KD;
+        const uint32_t vw = pack2(h0, h1);
+        ll_store(p.llVn + (static_cast<size_t>(l) * B + b) * (KD / 2) + vn / 2, vw, epoch);
+        uint16_t* row = append_row(p.kv[l], p.P, p.Hkv, p.kv[l].v, b, pos, vn / kAttnD);
+        if (row) *reinterpret_cast<uint32_t*>(row + (vn & (kAttnD - 1))) = vw;
+    }
+}
+
+// The rotation table of the token: cos, sin of pos_b * theta^(-2i/128) in
+// fp64 (a separate function: fp64 sincos needs registers the kernel's main
+// loop should not pay for).
+template <int B>
+__device__ __noinline__ void rope_table(const ChainParamsA& p, double2* rope)
+{
+    for (int e = threadIdx.x; e < B * (kAttnD / 2); e += blockDim.x) {
+        const int b = e / (kAttnD / 2), i = e - b * (kAttnD / 2);
+        const int pos = __ldg(p.positions + b);
+        double sn, cn;
+        sincos(static_cast<double>(pos < 0 ? 0 : pos) * p.inv_freq[i], &sn, &cn);
+        rope[e] = make_double2(cn, sn);
+    }
+}
+
+// Sum over the 32 lanes, every lane gets it.
+__device__ __forceinline__ float warp_allsum(float v)
+{
+#pragma unroll
+    for (int o = 16; o > 0; o >>= 1) v += __shfl_xor_sync(0xffffffffu, v, o);
+    return v;
+}
+
+// The decode attention of layer l, run by the consumer warps of every CTA at
+// the start of the O stage.  Split u = blockIdx.x + k * gridDim.x is (row b,
+// kv head h, token range c of S); its warps take U consecutive tokens at a
+// time (lane: dimensions 4 lane .. 4 lane + 3), keep a running maximum, sum
+// and weighted value sum per query head of the group, combine the warps in
+// shared memory (one head at a time) and store the split's (o, m, l).  The
+// last split of (b, h) to arrive merges all S of them in split order and
+// publishes a = o / l.  scratch: qs[G][128] then per-warp partials
+// [NW][kAttnPart] floats (inside the staging area, free at this point).
+template <int B, int NW, int G>
+__device__ __noinline__ void attention_phase(const ChainParamsA& p, int l, uint32_t epoch, float* scratch, const int* pos_sh,
+                                int* flag_sh)
+{
+    constexpr int kConsumers = NW * 32;
+    constexpr int U = G <= 4 ? 8 : 4;          // tokens a warp has in flight
+    const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
+    const int H = p.H, Hkv = p.Hkv, S = p.S, KD = Hkv * kAttnD;
+    const KvLayer& kv = p.kv[l];
+    float* qs = scratch;
+    float* wp = scratch + G * kAttnD;
+    const int nunits = B * Hkv * S;
+    const uint64_t* qsrc = p.llA + ((blockIdx.x & 1) ? p.rep.A : 0u) + static_cast<size_t>(l) * B * (H / 2);
+    for (int u = blockIdx.x; u < nunits; u += gridDim.x) {
+        const int b = u / (Hkv * S);
+        const int rr = u - b * (Hkv * S);
+        const int h = rr / S, c = rr - h * S;
+        const int pos = pos_sh[b];
+        int T = pos + 1;                                        // 0 for an invalid position
+        const int cap = kv.pt_stride * p.P;
+        if (T > cap) {
+            T = cap;
+            if (threadIdx.x == 0 && c == 0) atomicOr(p.err, kErrSeqLen);
+        }
+        const int t0 = static_cast<int>(static_cast<int64_t>(c) * T / S);
+        const int t1 = static_cast<int>(static_cast<int64_t>(c + 1) * T / S);
+        named_barrier_sync(1, kConsumers);                      // scratch free
+        for (int e = threadIdx.x; e < G * (kAttnD / 2); e += kConsumers) {
+            const int j = e / (kAttnD / 2), w = e - j * (kAttnD / 2);
+            const uint32_t qw = ll_load(qsrc + static_cast<size_t>(b) * (H / 2) + (h * G + j) * (kAttnD / 2) + w, epoch,
+                                        epoch, p.err, p.abort, p.wait_ns);
+            qs[j * kAttnD + 2 * w] = lo_f(qw);
+            qs[j * kAttnD + 2 * w + 1] = hi_f(qw);
+        }
+        named_barrier_sync(1, kConsumers);
+        float4 qv[G];
+#pragma unroll
+        for (int j = 0; j < G; ++j) qv[j] = reinterpret_cast<const float4*>(qs + j * kAttnD)[lane];
+        float m[G], ls[G], o[G][4];
+#pragma unroll
+        for (int j = 0; j < G; ++j) {
+            m[j] = -INFINITY;
+            ls[j] = 0.f;
+            o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
+        }
+        const uint64_t* knew = p.llK + (static_cast<size_t>(l) * B + b) * (KD / 2) + h * (kAttnD / 2) + 2 * lane;
+        const uint64_t* vnew = p.llVn + (static_cast<size_t>(l) * B + b) * (KD / 2) + h * (kAttnD / 2) + 2 * lane;
+        for (int base = t0 + warp * U; base < t1; base += NW * U) {
+            uint2 kr[U], vr[U];
+#pragma unroll
+            for (int uu = 0; uu < U; ++uu) {
+                const int t = base + uu;
+                kr[uu] = make_uint2(0u, 0u);
+                vr[uu] = make_uint2(0u, 0u);
+                if (t < t1 && t != pos) {
+                    const int pi = t / p.P;
+                    const int page = kv.pt[static_cast<size_t>(b) * kv.pt_stride + pi];
+                    if (page >= 0 && page < kv.num_pages) {
+                        const size_t row = ((static_cast<size_t>(page) * Hkv + h) * p.P + (t - pi * p.P)) * kAttnD;
+                        kr[uu] = __ldg(reinterpret_cast<const uint2*>(kv.k + row) + lane);
+                        vr[uu] = __ldg(reinterpret_cast<const uint2*>(kv.v + row) + lane);
+                    } else if (lane == 0) {
+                        atomicOr(p.err, kErrPageId);
+                    }
+                } else if (t == pos && t < t1) {
+                    // the new token: the QKV epilogue's flagged words
+                    kr[uu].x = ll_load(knew, epoch, epoch, p.err, p.abort, p.wait_ns);
+                    kr[uu].y = ll_load(knew + 1, epoch, epoch, p.err, p.abort, p.wait_ns);
+                    vr[uu].x = ll_load(vnew, epoch, epoch, p.err, p.abort, p.wait_ns);
+                    vr[uu].y = ll_load(vnew + 1, epoch, epoch, p.err, p.abort, p.wait_ns);
+                }
+            }
+#pragma unroll
+            for (int uu = 0; uu < U; ++uu) {
+                if (base + uu >= t1) break;
+                const float k0 = lo_f(kr[uu].x), k1 = hi_f(kr[uu].x), k2 = lo_f(kr[uu].y), k3 = hi_f(kr[uu].y);
+                const float w0 = lo_f(vr[uu].x), w1 = hi_f(vr[uu].x), w2 = lo_f(vr[uu].y), w3 = hi_f(vr[uu].y);
+                float sc[G];
+#pragma unroll
+                for (int j = 0; j < G; ++j) sc[j] = fmaf(qv[j].x, k0, fmaf(qv[j].y, k1, fmaf(qv[j].z, k2, qv[j].w * k3)));
+#pragma unroll
+                for (int j = 0; j < G; ++j) sc[j] = warp_allsum(sc[j]) * p.scale;
+#pragma unroll
+                for (int j = 0; j < G; ++j) {
+                    const float mn = fmaxf(m[j], sc[j]);
+                    const float corr = expf(m[j] - mn);
+                    const float pw = expf(sc[j] - mn);
+                    ls[j] = fmaf(ls[j], corr, pw);
+                    o[j][0] = fmaf(o[j][0], corr, pw * w0);
+                    o[j][1] = fmaf(o[j][1], corr, pw * w1);
+                    o[j][2] = fmaf(o[j][2], corr, pw * w2);
+                    o[j][3] = fmaf(o[j][3], corr, pw * w3);
+                    m[j] = mn;
+                }
+            }
+        }
+        // combine the warps, one query head at a time; store the split's partial
+        float* dst = p.apart + ((((static_cast<size_t>(l) * B + b) * Hkv + h) * S + c) * G) * kAttnPart;
+#pragma unroll
+        for (int j = 0; j < G; ++j) {
+            float* mine = wp + warp * kAttnPart;
+            reinterpret_cast<float4*>(mine)[lane] = make_float4(o[j][0], o[j][1], o[j][2], o[j][3]);
+            if (lane == 0) {
+                mine[kAttnD] = m[j];
+                mine[kAttnD + 1] = ls[j];
+            }
+            named_barrier_sync(1, kConsumers);
+            if (threadIdx.x < kAttnD) {
+                const int d = threadIdx.x;
+                float M = -INFINITY;
+                for (int w = 0; w < NW; ++w) M = fmaxf(M, wp[w * kAttnPart + kAttnD]);
+                float Ls = 0.f, Od = 0.f;
+                if (M != -INFINITY) {
+                    for (int w = 0; w < NW; ++w) {
+                        const float f = expf(wp[w * kAttnPart + kAttnD] - M);   // 0 for a warp without tokens
+                        Ls = fmaf(f, wp[w * kAttnPart + kAttnD + 1], Ls);
+                        Od = fmaf(f, wp[w * kAttnPart + d], Od);
+                    }
+                }
+                dst[j * kAttnPart + d] = Od;
+                if (d == 0) {
+                    dst[j * kAttnPart + kAttnD] = M;
+                    dst[j * kAttnPart + kAttnD + 1] = Ls;
+                }
+                __threadfence();
+            }
+            named_barrier_sync(1, kConsumers);
+        }
+        if (threadIdx.x == 0) {
+            __threadfence();
+            const uint32_t prev = atomicAdd(p.acnt + (static_cast<size_t>(l) * B + b) * Hkv + h, 1u);
+            *flag_sh = (prev == static_cast<uint32_t>(S - 1)) ? 1 : 0;
+            __threadfence();
+        }
+        named_barrier_sync(1, kConsumers);
+        if (*flag_sh) {
+            // every split of (b, h) is in: merge them in split order
+            const float* src = p.apart + (((static_cast<size_t>(l) * B + b) * Hkv + h) * S) * G * kAttnPart;
+            for (int e = threadIdx.x; e < G * (kAttnD / 2); e += kConsumers) {
+                const int j = e / (kAttnD / 2), w = e - j * (kAttnD / 2);
+                float M = -INFINITY;
+                for (int cc = 0; cc < S; ++cc) M = fmaxf(M, __ldcg(src + (cc * G + j) * kAttnPart + kAttnD));
+                float Ls = 0.f, O0 = 0.f, O1 = 0.f;
+                if (M != -INFINITY) {
+                    for (int cc = 0; cc < S; ++cc) {
+                        const float* pc = src + (cc * G + j) * kAttnPart;
+                        const float f = expf(__ldcg(pc + kAttnD) - M);
+                        Ls = fmaf(f, __ldcg(pc + kAttnD + 1), Ls);
+                        O0 = fmaf(f, __ldcg(pc + 2 * w), O0);
+                        O1 = fmaf(f, __ldcg(pc + 2 * w + 1), O1);
+                    }
+                }
+                const float a0 = Ls > 0.f ? O0 / Ls : 0.f, a1 = Ls > 0.f ? O1 / Ls : 0.f;
+                const uint32_t aw = pack2(float_to_half_bits(a0), float_to_half_bits(a1));
+                const int n = (h * G + j) * kAttnD + 2 * w;
+                *reinterpret_cast<uint32_t*>(p.pAt + (static_cast<size_t>(l) * B + b) * H + n) = aw;
+                ll_store2(p.llAt + (static_cast<size_t>(l) * B + b) * (H / 2) + n / 2, p.repAt, aw, epoch);
+            }
+            if (threadIdx.x == 0) p.acnt[(static_cast<size_t>(l) * B + b) * Hkv + h] = 0u;   // for the next token
+        }
+    }
+    named_barrier_sync(1, kConsumers);                          // scratch free for the staging
+}
+
 template <int B, int NW>
-__global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const __grid_constant__ ChainParams p)
+__device__ __forceinline__ void attention_dispatch(const ChainParamsA& p, int l, uint32_t epoch, float* scratch,
+                                                   const int* pos_sh, int* flag_sh)
+{
+    switch (p.G) {
+        case 1: attention_phase<B, NW, 1>(p, l, epoch, scratch, pos_sh, flag_sh); break;
+        case 2: attention_phase<B, NW, 2>(p, l, epoch, scratch, pos_sh, flag_sh); break;
+        case 3: attention_phase<B, NW, 3>(p, l, epoch, scratch, pos_sh, flag_sh); break;
+        case 4: attention_phase<B, NW, 4>(p, l, epoch, scratch, pos_sh, flag_sh); break;
+        case 5: attention_phase<B, NW, 5>(p, l, epoch, scratch, pos_sh, flag_sh); break;
+        case 6: attention_phase<B, NW, 6>(p, l, epoch, scratch, pos_sh, flag_sh); break;
+        case 7: attention_phase<B, NW, 7>(p, l, epoch, scratch, pos_sh, flag_sh); break;
+        default: attention_phase<B, NW, 8>(p, l, epoch, scratch, pos_sh, flag_sh); break;
+    }
+}
+
+template <int B, int NW, bool ATT>
+__global__ void __launch_bounds__((NW + 1) * 32, 1)
+    chain_kernel(const __grid_constant__ typename std::conditional<ATT, ChainParamsA, ChainParams>::type p)
 {
     extern __shared__ __align__(1024) uint8_t smem[];
     uint64_t* full = reinterpret_cast<uint64_t*>(smem);
@@ -533,6 +848,21 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const __grid_co
         epoch_sh[2] = static_cast<int>(static_cast<int64_t>(blockIdx.x + 1) * nw / gridDim.x);
     }
     if (threadIdx.x < kMaxChainBatch * 32) red[threadIdx.x] = 0.f;   // warps >= NW stay zero
+    // decode step: the rotation table (cos, sin of pos * theta^(-2i/128) per
+    // row, fp64) and the rows' positions (-1 for an invalid one)
+    double2* rope = nullptr;
+    int* pos_sh = nullptr;
+    int* flag_sh = nullptr;
+    if constexpr (ATT) {
+        rope = reinterpret_cast<double2*>(smem + p.rope_off);
+        pos_sh = reinterpret_cast<int*>(smem + p.rope_off + B * (kAttnD / 2) * sizeof(double2));
+        flag_sh = pos_sh + kMaxChainBatch;
+        rope_table<B>(p, rope);
+        if (threadIdx.x < B) {
+            const int pos = __ldg(p.positions + threadIdx.x);
+            pos_sh[threadIdx.x] = pos < 0 ? -1 : pos;
+        }
+    }
     if (threadIdx.x >= 32 && threadIdx.x < 32 + 5) {
         const int t = threadIdx.x - 32;
         const Stage g = stage_at(p, stage_of_type(p, t));
@@ -605,6 +935,11 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const __grid_co
         for (int st = 0; st < nstages; ++st) {
             const Stage g = stage_at(p, st);
             const StageInfo& in = info[g.type];
+            if constexpr (ATT) {
+                // every CTA takes its splits of the layer's attention, words or not
+                if (g.type == kO)
+                    attention_dispatch<B, NW>(p, g.layer, epoch, reinterpret_cast<float*>(xs), pos_sh, flag_sh);
+            }
             if (in.nwords <= 0) continue;
             const int l = g.layer;
             const int K = g.K, cpr = K >> 3;
@@ -621,7 +956,10 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const __grid_co
                 const bool plain = (g.type == kQKV && l == 0);
                 const bool r1 = (blockIdx.x & 1) != 0;   // this CTA's replica
                 if (g.type == kQKV) ll = p.llX + (r1 ? p.rep.X : 0u) + static_cast<size_t>(l) * B * (H / 2);
-                else if (g.type == kO) ll = p.llA + (r1 ? p.rep.A : 0u) + static_cast<size_t>(l) * B * (H / 2);
+                else if (g.type == kO) {
+                    if constexpr (ATT) ll = p.llAt + (r1 ? p.repAt : 0u) + static_cast<size_t>(l) * B * (H / 2);
+                    else ll = p.llA + (r1 ? p.rep.A : 0u) + static_cast<size_t>(l) * B * (H / 2);
+                }
                 else if (g.type == kGU) ll = p.llX1 + (r1 ? p.rep.X1 : 0u) + static_cast<size_t>(l) * B * (H / 2);
                 else if (g.type == kDOWN) ll = p.llM + (r1 ? p.rep.M : 0u) + static_cast<size_t>(l) * B * (F / 2);
                 else ll = p.llX + (r1 ? p.rep.X : 0u) + static_cast<size_t>(p.L) * B * (H / 2);
@@ -860,6 +1198,14 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const __grid_co
 #pragma unroll
                 for (int bb = 0; bb < B; ++bb) {
                     if (bb != b) continue;
+                    if constexpr (ATT) {
+                        if (g.type == kQKV) {
+                            qkv_epilogue_attn<B>(p, l, w0 + wc, bb, sum.x, sum.y, rf[bb], epoch, rope, pos_sh);
+                            if (spw == 2 && wc + 1 < nwd)
+                                qkv_epilogue_attn<B>(p, l, w0 + wc + 1, bb, sum.z, sum.w, rf[bb], epoch, rope, pos_sh);
+                            continue;
+                        }
+                    }
                     if (g.type == kGU) {
                         word_epilogue<B>(p, g, w0 + wc, bb, sum.x, sum.z, sum.y, sum.w, rf[bb], 0u, epoch);
                     } else {
@@ -896,17 +1242,89 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1) chain_kernel(const __grid_co
 // kernels and per-stage epilogues (wq4_tc.cu); they write the same workspace
 // traces as the persistent kernel.
 
+// Decode step of the graph path: one block per batch row rotates q and k of
+// layer l's QKV output (the same fp64 rotation as the persistent kernel),
+// writes the traces, appends k and v to the cache and sets the row's
+// sequence length (positions + 1; 0 for an invalid position).  Launched
+// after the QKV stage with programmatic dependent launch: it reads the QKV
+// output only after that grid has completed.
+struct RopeAppendArgs {
+    const uint16_t* qkv;        // [B][Nqkv]
+    uint16_t* qr;               // [B][H] rotated queries
+    uint16_t* kr;               // [B][Hkv 128] rotated keys
+    int32_t* seq_lens;          // [B]
+    const int32_t* positions;   // [B]
+    KvLayer kv;
+    int P, Hkv, H, Nqkv;
+    uint32_t* err;
+    double inv_freq[kAttnD / 2];
+};
+
+__global__ void __launch_bounds__(256) rope_append_kernel(const __grid_constant__ RopeAppendArgs a)
+{
+    __shared__ double2 rope[kAttnD / 2];
+    asm volatile("griddepcontrol.wait;" ::: "memory");
+    const int b = blockIdx.x;
+    const int pos = __ldg(a.positions + b);
+    if (threadIdx.x < kAttnD / 2) {
+        double sn, cn;
+        sincos(static_cast<double>(pos < 0 ? 0 : pos) * a.inv_freq[threadIdx.x], &sn, &cn);
+        rope[threadIdx.x] = make_double2(cn, sn);
+    }
+    if (threadIdx.x == 0) a.seq_lens[b] = pos < 0 ? 0 : pos + 1;
+    __syncthreads();
+    asm volatile("griddepcontrol.launch_dependents;" ::: "memory");
+    const int H = a.H, KD = a.Hkv * kAttnD;
+    const uint32_t* row = reinterpret_cast<const uint32_t*>(a.qkv + static_cast<size_t>(b) * a.Nqkv);
+    for (int w = threadIdx.x; w < (H + 2 * KD) / 2; w += blockDim.x) {
+        const int n = 2 * w;
+        const uint32_t x = row[w];
+        if (n < H + KD) {
+            const double2 cs = rope[(n & (kAttnD - 1)) >> 1];
+            const double u0 = half_bits_to_float(static_cast<uint16_t>(x & 0xFFFFu));
+            const double u1 = half_bits_to_float(static_cast<uint16_t>(x >> 16));
+            const uint32_t rw = pack2(double_to_half_bits(u0 * cs.x - u1 * cs.y), double_to_half_bits(u0 * cs.y + u1 * cs.x));
+            if (n < H) {
+                *reinterpret_cast<uint32_t*>(a.qr + static_cast<size_t>(b) * H + n) = rw;
+            } else {
+                const int kn = n - H;
+                *reinterpret_cast<uint32_t*>(a.kr + static_cast<size_t>(b) * KD + kn) = rw;
+                uint16_t* r = append_row(a.kv, a.P, a.Hkv, a.kv.k, b, pos, kn / kAttnD);
+                if (r) *reinterpret_cast<uint32_t*>(r + (kn & (kAttnD - 1))) = rw;
+                else if ((kn & (kAttnD - 1)) == 0) atomicOr(a.err, kErrAppend);
+            }
+        } else {
+            const int vn = n - H - KD;
+            uint16_t* r = append_row(a.kv, a.P, a.Hkv, a.kv.v, b, pos, vn / kAttnD);
+            if (r) *reinterpret_cast<uint32_t*>(r + (vn & (kAttnD - 1))) = x;
+        }
+    }
+}
+
 // ---------------------------------------------------------------- host --
 
 struct Layout {
     size_t header, llA, llX1, llM, llX, llV, pV, pX2, pQKV, pO, pX1, pGU, pM, pD, x_stage, logits_stage, rfac,
         xpH0, xpH1, xpF, cnt, part, total;
     size_t ll_begin, ll_end;
+    // decode step (after everything above, so that the chain's offsets stay):
+    // flagged words of the new keys, values and attention output (zeroed),
+    // traces, split partials and counters (batch 1-2), or the sequence
+    // lengths and wq4_paged_attention's workspace (batch 3-32)
+    size_t att_ll_begin, att_ll_end, llK, llVn, llAt, pQr, pKr, pAt, apart, acnt, seq_lens, attn_ws, attn_ws_bytes;
 };
 
 struct Dims {
     int L, H, F, Nqkv, V, B;
+    int nq, Hkv, Dh;     // query heads, kv heads, head dimension
 };
+
+// Heads the decode step's attention handles: head dimension 128, a whole
+// number of query heads (at most kAttnMaxGroup) per kv head.
+bool attn_heads_ok(const Dims& d)
+{
+    return d.Dh == kAttnD && d.Hkv >= 1 && d.nq % d.Hkv == 0 && d.nq / d.Hkv <= kAttnMaxGroup;
+}
 
 bool table_dims(const wq4_layer_table* t, Dims* d)
 {
@@ -928,10 +1346,13 @@ bool table_dims(const wq4_layer_table* t, Dims* d)
     d->Nqkv = static_cast<int>(nqkv);
     d->V = t->vocab;
     d->B = t->batch;
+    d->nq = t->n_q_heads;
+    d->Hkv = t->n_kv_heads;
+    d->Dh = t->head_dim;
     return true;
 }
 
-Layout make_layout(const Dims& d)
+Layout make_layout(const Dims& d, bool att = false, size_t attn_ws_bytes = 0)
 {
     Layout y;
     size_t o = 0;
@@ -971,6 +1392,27 @@ Layout make_layout(const Dims& d)
     } else {
         y.rfac = y.cnt = y.xpH0 = y.xpH1 = y.xpF = y.part = 0;
     }
+    y.att_ll_begin = y.att_ll_end = y.llK = y.llVn = y.llAt = y.pQr = y.pKr = y.pAt = 0;
+    y.apart = y.acnt = y.seq_lens = y.attn_ws = y.attn_ws_bytes = 0;
+    if (att) {
+        const size_t KD = static_cast<size_t>(d.Hkv) * kAttnD, G = d.Hkv > 0 ? d.nq / d.Hkv : 0;
+        y.att_ll_begin = o;
+        y.llK = take(8 * L * B * (KD / 2));
+        y.llVn = take(8 * L * B * (KD / 2));
+        y.llAt = take(8 * 2 * L * B * (H / 2));          // two replicas
+        y.att_ll_end = o;
+        y.pQr = take(2 * L * B * H);
+        y.pKr = take(2 * L * B * KD);
+        y.pAt = take(2 * L * B * H);
+        if (d.B <= kMaxChainBatch) {
+            y.apart = take(4 * L * B * d.Hkv * kAttnMaxSplits * G * kAttnPart);
+            y.acnt = take(4 * L * B * d.Hkv);
+        } else {
+            y.seq_lens = take(4 * B);
+            y.attn_ws = take(attn_ws_bytes);
+            y.attn_ws_bytes = attn_ws_bytes;
+        }
+    }
     y.total = o;
     return y;
 }
@@ -989,10 +1431,19 @@ struct Plan {
     int q[5];                // K parts per superpair, per stage type
     int spw[5];              // words per superpair, per stage type
     cudaGraphExec_t graph;   // graph path (batch > kMaxChainBatch), else null
+    // decode step only
+    bool att = false;
+    std::vector<wq4_kv_cache> kv;
+    const int32_t* positions = nullptr;
+    double theta = 0.0;
+    float scale = 0.f;
+    int S = 0;               // splits per (row, kv head)
+    uint32_t rope_off = 0;
 };
 
 std::mutex g_plan_mu;
-std::map<const wq4_layer_table*, Plan> g_plans;
+// plans by (table, decode step or chain)
+std::map<std::pair<const wq4_layer_table*, bool>, Plan> g_plans;
 
 // Test hook state (wq4_test_chain_waits): the limit of the chain kernel's
 // waits on flagged words and the stage whose input waits can never be
@@ -1001,10 +1452,40 @@ std::map<const wq4_layer_table*, Plan> g_plans;
 std::atomic<uint64_t> g_wait_ns{kWaitTimeoutNs};
 std::atomic<int> g_stall_stage{-1};
 
-bool same_contents(const Plan& pl, const wq4_layer_table* t)
+bool same_contents(const Plan& pl, const wq4_layer_table* t, const wq4_decode_attn* a)
 {
     if (std::memcmp(&pl.table, t, sizeof(*t)) != 0) return false;
-    return std::memcmp(pl.layers.data(), t->layers, sizeof(wq4_layer) * t->num_layers) == 0;
+    if (std::memcmp(pl.layers.data(), t->layers, sizeof(wq4_layer) * t->num_layers) != 0) return false;
+    if (pl.att != (a != nullptr)) return false;
+    if (!a) return true;
+    return pl.positions == a->positions && pl.theta == a->rope_theta && pl.scale == a->scale &&
+           std::memcmp(pl.kv.data(), a->layers, sizeof(wq4_kv_cache) * t->num_layers) == 0;
+}
+
+// The attention description of a decode step, checked against the table.
+int check_attn(const wq4_layer_table* t, const Dims& d, const wq4_decode_attn* a)
+{
+    if (!a || !a->layers || !a->positions) return WQ4_ERR_INVALID;
+    if (!attn_heads_ok(d)) return WQ4_ERR_UNSUPPORTED;
+    if (!(a->rope_theta > 1.0) || !std::isfinite(a->rope_theta)) return WQ4_ERR_INVALID;
+    if (!(a->scale > 0.f) || !std::isfinite(a->scale)) return WQ4_ERR_INVALID;
+    if (!aligned(a->positions, 4)) return WQ4_ERR_ALIGN;
+    const int P = a->layers[0].page_size;
+    for (int l = 0; l < d.L; ++l) {
+        const wq4_kv_cache& c = a->layers[l];
+        if (!c.k || !c.v || !c.page_table || c.num_pages < 1 || c.page_table_stride < 1) return WQ4_ERR_INVALID;
+        if (c.n_kv_heads != d.Hkv || c.head_dim != kAttnD) return WQ4_ERR_INVALID;
+        if (c.page_size != P || P < 16 || P % 16) return WQ4_ERR_INVALID;
+        if (!aligned(c.k, 16) || !aligned(c.v, 16) || !aligned(c.page_table, 4)) return WQ4_ERR_ALIGN;
+        const int64_t rows = static_cast<int64_t>(c.num_pages) * d.Hkv * P;
+        if (rows >= (int64_t(1) << 31)) return WQ4_ERR_UNSUPPORTED;
+        if (static_cast<int64_t>(c.page_table_stride) * P >= (int64_t(1) << 30)) return WQ4_ERR_UNSUPPORTED;
+        const size_t cb = static_cast<size_t>(rows) * kAttnD * 2;
+        if (overlaps(c.k, cb, c.v, cb) || overlaps(c.k, cb, t->workspace, t->workspace_bytes) ||
+            overlaps(c.v, cb, t->workspace, t->workspace_bytes))
+            return WQ4_ERR_INVALID;
+    }
+    return WQ4_OK;
 }
 
 bool mat_ok(const wq4_mat& m)
@@ -1012,10 +1493,10 @@ bool mat_ok(const wq4_mat& m)
     return m.W && m.s && aligned(m.W, 16) && aligned(m.s, 16);
 }
 
-template <int B>
+template <int B, bool ATT>
 cudaError_t set_chain_attr(int smem)
 {
-    return cudaFuncSetAttribute(chain_kernel<B, kChainWarps>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
+    return cudaFuncSetAttribute(chain_kernel<B, kChainWarps, ATT>, cudaFuncAttributeMaxDynamicSharedMemorySize, smem);
 }
 
 // Bytes of one output word of each stage type (two rows; gate_up four).
@@ -1183,9 +1664,75 @@ int check_scales_fp16(const wq4_layer_table* t, const Dims& d, uint32_t* scratch
     return m > kMaxFp16ScaleBits ? WQ4_ERR_UNSUPPORTED : WQ4_OK;
 }
 
+KvLayer kv_layer(const wq4_kv_cache& c)
+{
+    KvLayer k;
+    k.k = c.k;
+    k.v = c.v;
+    k.pt = c.page_table;
+    k.pt_stride = c.page_table_stride;
+    k.num_pages = c.num_pages;
+    return k;
+}
+
+void fill_inv_freq(double theta, double* out)
+{
+    for (int i = 0; i < kAttnD / 2; ++i) out[i] = std::pow(theta, -2.0 * i / kAttnD);
+}
+
+// The decode step's attention nodes of the graph path (see TcAttnHook): the
+// rotation/append kernel, wq4_paged_attention on the rotated queries, and the
+// token-start kernel on the attention output (O's permuted input).
+struct GraphAttn {
+    const Plan* pl;
+    const Dims* d;
+    const Layout* lay;
+    uint8_t* ws;
+};
+
+int record_graph_attention(void* ctx, int l, cudaStream_t cs, uint16_t* xp, float* sq)
+{
+    const GraphAttn& g = *static_cast<const GraphAttn*>(ctx);
+    const Dims& d = *g.d;
+    const Layout& y = *g.lay;
+    const size_t B = d.B, H = d.H, KD = static_cast<size_t>(d.Hkv) * kAttnD;
+    const wq4_kv_cache& c = g.pl->kv[l];
+    RopeAppendArgs a;
+    std::memset(&a, 0, sizeof(a));
+    a.qkv = reinterpret_cast<const uint16_t*>(g.ws + y.pQKV) + static_cast<size_t>(l) * B * d.Nqkv;
+    a.qr = reinterpret_cast<uint16_t*>(g.ws + y.pQr) + static_cast<size_t>(l) * B * H;
+    a.kr = reinterpret_cast<uint16_t*>(g.ws + y.pKr) + static_cast<size_t>(l) * B * KD;
+    a.seq_lens = reinterpret_cast<int32_t*>(g.ws + y.seq_lens);
+    a.positions = g.pl->positions;
+    a.kv = kv_layer(c);
+    a.P = c.page_size;
+    a.Hkv = d.Hkv;
+    a.H = d.H;
+    a.Nqkv = d.Nqkv;
+    a.err = status_word();
+    if (!a.err) return WQ4_ERR_CUDA;
+    fill_inv_freq(g.pl->theta, a.inv_freq);
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(d.B);
+    cfg.blockDim = dim3(256);
+    cfg.stream = cs;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    if (cudaLaunchKernelEx(&cfg, rope_append_kernel, a) != cudaSuccess) return WQ4_ERR_CUDA;
+    uint16_t* at = reinterpret_cast<uint16_t*>(g.ws + y.pAt) + static_cast<size_t>(l) * B * H;
+    int rc = wq4_paged_attention(&c, a.qr, d.H, a.seq_lens, at, d.H, d.B, d.nq, g.pl->scale, g.ws + y.attn_ws,
+                                 y.attn_ws_bytes, cs);
+    if (rc != WQ4_OK) return rc;
+    return tc_launch_prologue(at, d.H, d.B, sq, xp, cs);
+}
+
 // Records one token of the graph path on `cs`: every stage kernel of every
-// layer, reading the token input from the workspace staging area and writing
-// the logits to the workspace logits area.
+// layer (and with pl->att the attention of each), reading the token input
+// from the workspace staging area and writing the logits to the workspace
+// logits area.
 int build_graph_plan(const wq4_layer_table* t, const Dims& d, const Layout& lay, int dev, const DeviceInfo* di,
                      Plan* pl, cudaStream_t stream)
 {
@@ -1228,7 +1775,9 @@ int build_graph_plan(const wq4_layer_table* t, const Dims& d, const Layout& lay,
         int rrec = cudaMemsetAsync(ws + lay.cnt, 0, 4 * static_cast<size_t>(kTcCounterWords), cs) == cudaSuccess
                        ? WQ4_OK
                        : WQ4_ERR_CUDA;
-        if (rrec == WQ4_OK) rrec = tc_record_token(tc, cs);
+        GraphAttn ga{pl, &d, &lay, ws};
+        const TcAttnHook hook{record_graph_attention, &ga};
+        if (rrec == WQ4_OK) rrec = tc_record_token(tc, cs, pl->att ? &hook : nullptr);
         if (cudaStreamEndCapture(cs, &graph) == cudaSuccess && graph && rrec == WQ4_OK &&
             cudaGraphInstantiate(&exec, graph, 0) == cudaSuccess)
             rc = WQ4_OK;
@@ -1253,7 +1802,7 @@ int build_graph_plan(const wq4_layer_table* t, const Dims& d, const Layout& lay,
     return WQ4_OK;
 }
 
-int build_plan(const wq4_layer_table* t, Plan* pl, cudaStream_t stream)
+int build_plan(const wq4_layer_table* t, const wq4_decode_attn* a, Plan* pl, cudaStream_t stream)
 {
     Dims d;
     if (!table_dims(t, &d)) return WQ4_ERR_INVALID;
@@ -1263,26 +1812,57 @@ int build_plan(const wq4_layer_table* t, Plan* pl, cudaStream_t stream)
         if (!mat_ok(ly.qkv) || !mat_ok(ly.o) || !mat_ok(ly.gate_up) || !mat_ok(ly.down)) return WQ4_ERR_INVALID;
     }
     if (!mat_ok(t->lm_head)) return WQ4_ERR_INVALID;
-    const Layout lay = make_layout(d);
     if (!t->workspace || !aligned(t->workspace, 256)) return WQ4_ERR_ALIGN;
+    size_t attn_ws = 0;
+    if (a) {
+        const int ra = check_attn(t, d, a);
+        if (ra != WQ4_OK) return ra;
+        if (d.B > kMaxChainBatch) {
+            attn_ws = wq4_paged_attention_workspace_bytes(d.B, d.nq, d.Hkv, kAttnD);
+            if (attn_ws == 0) return WQ4_ERR_CUDA;
+        }
+    }
+    const Layout lay = make_layout(d, a != nullptr, attn_ws);
     if (t->workspace_bytes < lay.total) return WQ4_ERR_INVALID;
     int dev = 0;
     const DeviceInfo* di = current_device_info(&dev);
     if (!di) return WQ4_ERR_CUDA;
+    if (a) {
+        pl->att = true;
+        pl->kv.assign(a->layers, a->layers + d.L);
+        pl->positions = a->positions;
+        pl->theta = a->rope_theta;
+        pl->scale = a->scale;
+        uint8_t* ws = static_cast<uint8_t*>(t->workspace);
+        // flagged words start at zero (epoch 0 never matches); counters at zero
+        if (cudaMemsetAsync(ws + lay.att_ll_begin, 0, lay.att_ll_end - lay.att_ll_begin, stream) != cudaSuccess)
+            return WQ4_ERR_CUDA;
+        if (lay.acnt && cudaMemsetAsync(ws + lay.acnt, 0, 4 * static_cast<size_t>(d.L) * d.B * d.Hkv, stream) !=
+                            cudaSuccess)
+            return WQ4_ERR_CUDA;
+        if (lay.attn_ws && cudaMemsetAsync(ws + lay.attn_ws, 0, lay.attn_ws_bytes, stream) != cudaSuccess)
+            return WQ4_ERR_CUDA;
+    }
     if (d.B > kMaxChainBatch) {
         if (d.Nqkv % 8) return WQ4_ERR_UNSUPPORTED;   // the O stage reads qkv rows with 16-byte loads
         return build_graph_plan(t, d, lay, dev, di, pl, stream);
     }
     if (!di->coop_launch) return WQ4_ERR_UNSUPPORTED;
     if (d.L > kChainMaxLayers) return WQ4_ERR_UNSUPPORTED;
-    const uint32_t x_bytes = static_cast<uint32_t>(align_up(static_cast<size_t>(d.B) * 2 * (d.H > d.F ? d.H : d.F), 128));
+    size_t xb = align_up(static_cast<size_t>(d.B) * 2 * (d.H > d.F ? d.H : d.F), 128);
+    // the attention's scratch (queries of a group, per-warp partials) lives in the staging area
+    if (a) xb = std::max(xb, align_up(4 * static_cast<size_t>(kAttnMaxGroup * kAttnD + kChainWarps * kAttnPart), 128));
+    const uint32_t x_bytes = static_cast<uint32_t>(xb);
+    // the rotation table (double2 [B][64]), the positions and a flag sit after the ring
+    const size_t rope_bytes = a ? align_up(static_cast<size_t>(d.B) * (kAttnD / 2) * 16 + 16, 128) : 0;
     // the residual words of a CTA's words must fit in shared memory
     if (static_cast<long>((d.H / 2 + di->sm_count - 1) / di->sm_count) * d.B > kMaxResWords) return WQ4_ERR_UNSUPPORTED;
     int spw[5];
     choose_spw(d, spw);
     const uint32_t slot_bytes = choose_slot_bytes(d, spw);
     const int header = kChainHeader;
-    const long avail = static_cast<long>(di->smem_optin) - header - static_cast<long>(x_bytes);
+    const long avail = static_cast<long>(di->smem_optin) - header - static_cast<long>(x_bytes) -
+                       static_cast<long>(rope_bytes);
     int nslots = avail > 0 ? static_cast<int>(avail / slot_bytes) : 0;
     if (nslots > kChainMaxSlots) nslots = kChainMaxSlots;
     int q[5];
@@ -1291,14 +1871,21 @@ int build_plan(const wq4_layer_table* t, Plan* pl, cudaStream_t stream)
     // whose barriers cannot alias
     while (nslots >= 2 && !ring_ok(d, nslots, slot_bytes, kChainWarps, spw, q)) --nslots;
     if (nslots < 2) return WQ4_ERR_UNSUPPORTED;
-    const size_t smem = header + x_bytes + static_cast<size_t>(nslots) * slot_bytes;
+    const size_t smem = header + x_bytes + static_cast<size_t>(nslots) * slot_bytes + rope_bytes;
+    pl->rope_off = static_cast<uint32_t>(header + x_bytes + static_cast<size_t>(nslots) * slot_bytes);
+    if (a) {
+        int S = di->sm_count / (d.B * d.Hkv);
+        pl->S = S < 1 ? 1 : (S > kAttnMaxSplits ? kAttnMaxSplits : S);
+    }
     // The limit is a property of the kernel, shared by every plan: set it to
     // the device maximum so that no plan's launch depends on which plan was
     // built last.
     cudaError_t e = cudaSuccess;
-    switch (d.B) {
-        case 1: e = set_chain_attr<1>(di->smem_optin); break;
-        default: e = set_chain_attr<2>(di->smem_optin); break;
+    switch (d.B * 2 + (a ? 1 : 0)) {
+        case 2: e = set_chain_attr<1, false>(di->smem_optin); break;
+        case 3: e = set_chain_attr<1, true>(di->smem_optin); break;
+        case 4: e = set_chain_attr<2, false>(di->smem_optin); break;
+        default: e = set_chain_attr<2, true>(di->smem_optin); break;
     }
     if (e != cudaSuccess) return WQ4_ERR_CUDA;
 
@@ -1324,23 +1911,11 @@ int build_plan(const wq4_layer_table* t, Plan* pl, cudaStream_t stream)
     return WQ4_OK;
 }
 
-int launch_chain(const Plan& pl, const uint16_t* x, uint16_t* logits, cudaStream_t stream)
+template <class P>
+int fill_chain_params(P& p, const Plan& pl, const uint16_t* x, uint16_t* logits)
 {
     uint8_t* ws = static_cast<uint8_t*>(pl.table.workspace);
     const Layout& y = pl.lay;
-    if (pl.graph) {
-        // the graph reads the token from and writes the logits to the workspace
-        uint16_t* xs = reinterpret_cast<uint16_t*>(ws + y.x_stage);
-        uint16_t* ls = reinterpret_cast<uint16_t*>(ws + y.logits_stage);
-        const size_t xb = static_cast<size_t>(pl.dims.B) * pl.dims.H * 2;
-        const size_t lb = static_cast<size_t>(pl.dims.B) * pl.dims.V * 2;
-        if (x != xs && cudaMemcpyAsync(xs, x, xb, cudaMemcpyDeviceToDevice, stream) != cudaSuccess) return WQ4_ERR_CUDA;
-        if (cudaGraphLaunch(pl.graph, stream) != cudaSuccess) return WQ4_ERR_CUDA;
-        if (logits != ls && cudaMemcpyAsync(logits, ls, lb, cudaMemcpyDeviceToDevice, stream) != cudaSuccess)
-            return WQ4_ERR_CUDA;
-        return WQ4_OK;
-    }
-    ChainParams p = {};
     for (int l = 0; l < pl.dims.L; ++l) {
         const wq4_layer& ly = pl.layers[l];
         p.mats[4 * l + 0] = {ly.qkv.W, ly.qkv.s};
@@ -1393,6 +1968,25 @@ int launch_chain(const Plan& pl, const uint16_t* x, uint16_t* logits, cudaStream
     p.wait_ns = g_wait_ns.load();
     p.stall_stage = g_stall_stage.load();
 
+    return WQ4_OK;
+}
+
+int launch_chain(const Plan& pl, const uint16_t* x, uint16_t* logits, cudaStream_t stream)
+{
+    uint8_t* ws = static_cast<uint8_t*>(pl.table.workspace);
+    const Layout& y = pl.lay;
+    if (pl.graph) {
+        // the graph reads the token from and writes the logits to the workspace
+        uint16_t* xs = reinterpret_cast<uint16_t*>(ws + y.x_stage);
+        uint16_t* ls = reinterpret_cast<uint16_t*>(ws + y.logits_stage);
+        const size_t xb = static_cast<size_t>(pl.dims.B) * pl.dims.H * 2;
+        const size_t lb = static_cast<size_t>(pl.dims.B) * pl.dims.V * 2;
+        if (x != xs && cudaMemcpyAsync(xs, x, xb, cudaMemcpyDeviceToDevice, stream) != cudaSuccess) return WQ4_ERR_CUDA;
+        if (cudaGraphLaunch(pl.graph, stream) != cudaSuccess) return WQ4_ERR_CUDA;
+        if (logits != ls && cudaMemcpyAsync(logits, ls, lb, cudaMemcpyDeviceToDevice, stream) != cudaSuccess)
+            return WQ4_ERR_CUDA;
+        return WQ4_OK;
+    }
     cudaLaunchConfig_t cfg = {};
     cfg.gridDim = dim3(pl.grid);
     cfg.blockDim = dim3((pl.nw + 1) * 32);
@@ -1404,9 +1998,39 @@ int launch_chain(const Plan& pl, const uint16_t* x, uint16_t* logits, cudaStream
     cfg.attrs = attr;
     cfg.numAttrs = 1;
     cudaError_t e;
-    switch (pl.dims.B) {
-        case 1: e = cudaLaunchKernelEx(&cfg, chain_kernel<1, kChainWarps>, p); break;
-        default: e = cudaLaunchKernelEx(&cfg, chain_kernel<2, kChainWarps>, p); break;
+    if (!pl.att) {
+        ChainParams p = {};
+        if (fill_chain_params(p, pl, x, logits) != WQ4_OK) return WQ4_ERR_CUDA;
+        switch (pl.dims.B) {
+            case 1: e = cudaLaunchKernelEx(&cfg, chain_kernel<1, kChainWarps, false>, p); break;
+            default: e = cudaLaunchKernelEx(&cfg, chain_kernel<2, kChainWarps, false>, p); break;
+        }
+    } else {
+        ChainParamsA p = {};
+        if (fill_chain_params(p, pl, x, logits) != WQ4_OK) return WQ4_ERR_CUDA;
+        const size_t L = pl.dims.L, B = pl.dims.B, H = pl.dims.H;
+        p.Hkv = pl.dims.Hkv;
+        p.G = pl.dims.nq / pl.dims.Hkv;
+        p.P = pl.kv[0].page_size;
+        p.S = pl.S;
+        p.scale = pl.scale;
+        p.positions = pl.positions;
+        p.llK = reinterpret_cast<uint64_t*>(ws + y.llK);
+        p.llVn = reinterpret_cast<uint64_t*>(ws + y.llVn);
+        p.llAt = reinterpret_cast<uint64_t*>(ws + y.llAt);
+        p.repAt = static_cast<uint32_t>(L * B * (H / 2));
+        p.rope_off = pl.rope_off;
+        p.pQr = reinterpret_cast<uint16_t*>(ws + y.pQr);
+        p.pKr = reinterpret_cast<uint16_t*>(ws + y.pKr);
+        p.pAt = reinterpret_cast<uint16_t*>(ws + y.pAt);
+        p.apart = reinterpret_cast<float*>(ws + y.apart);
+        p.acnt = reinterpret_cast<uint32_t*>(ws + y.acnt);
+        fill_inv_freq(pl.theta, p.inv_freq);
+        for (int l = 0; l < pl.dims.L; ++l) p.kv[l] = kv_layer(pl.kv[l]);
+        switch (pl.dims.B) {
+            case 1: e = cudaLaunchKernelEx(&cfg, chain_kernel<1, kChainWarps, true>, p); break;
+            default: e = cudaLaunchKernelEx(&cfg, chain_kernel<2, kChainWarps, true>, p); break;
+        }
     }
     return e == cudaSuccess ? WQ4_OK : WQ4_ERR_CUDA;
 }
@@ -1414,7 +2038,8 @@ int launch_chain(const Plan& pl, const uint16_t* x, uint16_t* logits, cudaStream
 // Finds (or builds) the plan of `t`; returns a copy to launch from.  With
 // no_rebuild_in_capture, a plan that would have to be (re)built while
 // `stream` is capturing is refused with WQ4_ERR_UNSUPPORTED.
-int get_plan(const wq4_layer_table* t, Plan* out, cudaStream_t stream, bool no_rebuild_in_capture = false)
+int get_plan(const wq4_layer_table* t, const wq4_decode_attn* a, Plan* out, cudaStream_t stream,
+             bool no_rebuild_in_capture = false)
 {
     if (!t) return WQ4_ERR_INVALID;
     Dims d;
@@ -1422,8 +2047,9 @@ int get_plan(const wq4_layer_table* t, Plan* out, cudaStream_t stream, bool no_r
     int dev = 0;
     if (cudaGetDevice(&dev) != cudaSuccess) return WQ4_ERR_CUDA;
     std::lock_guard<std::mutex> lock(g_plan_mu);
-    auto it = g_plans.find(t);
-    if (it != g_plans.end() && it->second.device == dev && same_contents(it->second, t)) {
+    const std::pair<const wq4_layer_table*, bool> key(t, a != nullptr);
+    auto it = g_plans.find(key);
+    if (it != g_plans.end() && it->second.device == dev && same_contents(it->second, t, a)) {
         *out = it->second;
         return WQ4_OK;
     }
@@ -1433,14 +2059,14 @@ int get_plan(const wq4_layer_table* t, Plan* out, cudaStream_t stream, bool no_r
         if (cs != cudaStreamCaptureStatusNone) return WQ4_ERR_UNSUPPORTED;
     }
     Plan pl;
-    const int rc = build_plan(t, &pl, stream);
+    const int rc = build_plan(t, a, &pl, stream);
     if (rc != WQ4_OK) return rc;
     if (it != g_plans.end() && it->second.graph) {
         // a replaced graph may still run on the GPU: free it once it is done
         cudaStreamSynchronize(stream);
         cudaGraphExecDestroy(it->second.graph);
     }
-    g_plans[t] = pl;
+    g_plans[key] = pl;
     *out = pl;
     return WQ4_OK;
 }
@@ -1463,7 +2089,7 @@ extern "C" int wq4_decode_chain(const wq4_layer_table* table, const uint16_t* x,
     if (!aligned(x, 16) || !aligned(logits, 2)) return WQ4_ERR_ALIGN;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     Plan pl;
-    const int rc = get_plan(table, &pl, st);
+    const int rc = get_plan(table, nullptr, &pl, st);
     if (rc != WQ4_OK) return rc;
     const size_t lb = static_cast<size_t>(pl.dims.B) * pl.dims.V * 2;
     if (overlaps(logits, lb, x, static_cast<size_t>(pl.dims.B) * pl.dims.H * 2) ||
@@ -1478,7 +2104,7 @@ extern "C" int wq4_decode_chain_host(const wq4_layer_table* table, const uint16_
     if (!table || !x_host || !logits_host) return WQ4_ERR_INVALID;
     cudaStream_t st = static_cast<cudaStream_t>(stream);
     Plan pl;
-    int rc = get_plan(table, &pl, st);
+    int rc = get_plan(table, nullptr, &pl, st);
     if (rc != WQ4_OK) return rc;
     uint8_t* ws = static_cast<uint8_t*>(table->workspace);
     uint16_t* xd = reinterpret_cast<uint16_t*>(ws + pl.lay.x_stage);
@@ -1495,11 +2121,63 @@ extern "C" int wq4_decode_chain_host(const wq4_layer_table* table, const uint16_
 extern "C" int wq4_chain_plan_destroy(const wq4_layer_table* table)
 {
     std::lock_guard<std::mutex> lock(g_plan_mu);
-    auto it = g_plans.find(table);
-    if (it == g_plans.end()) return WQ4_ERR_INVALID;
-    if (it->second.graph) cudaGraphExecDestroy(it->second.graph);
-    g_plans.erase(it);
-    return WQ4_OK;
+    int found = 0;
+    for (bool att : {false, true}) {
+        auto it = g_plans.find(std::make_pair(table, att));
+        if (it == g_plans.end()) continue;
+        if (it->second.graph) cudaGraphExecDestroy(it->second.graph);
+        g_plans.erase(it);
+        ++found;
+    }
+    return found ? WQ4_OK : WQ4_ERR_INVALID;
+}
+
+extern "C" size_t wq4_decode_step_workspace_bytes(const wq4_layer_table* table)
+{
+    Dims d;
+    if (!table_dims(table, &d) || !attn_heads_ok(d)) return 0;
+    size_t attn_ws = 0;
+    if (d.B > kMaxChainBatch) {
+        attn_ws = wq4_paged_attention_workspace_bytes(d.B, d.nq, d.Hkv, kAttnD);
+        if (attn_ws == 0) return 0;
+    }
+    return make_layout(d, true, attn_ws).total;
+}
+
+extern "C" int wq4_decode_step(const wq4_layer_table* table, const wq4_decode_attn* attn, const uint16_t* x,
+                               uint16_t* logits, void* stream)
+{
+    if (!table || !attn || !x || !logits) return WQ4_ERR_INVALID;
+    if (!aligned(x, 16) || !aligned(logits, 2)) return WQ4_ERR_ALIGN;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    Plan pl;
+    const int rc = get_plan(table, attn, &pl, st);
+    if (rc != WQ4_OK) return rc;
+    const size_t lb = static_cast<size_t>(pl.dims.B) * pl.dims.V * 2;
+    if (overlaps(logits, lb, x, static_cast<size_t>(pl.dims.B) * pl.dims.H * 2) ||
+        overlaps(logits, lb, table->workspace, pl.lay.total))
+        return WQ4_ERR_INVALID;
+    return launch_chain(pl, x, logits, st);
+}
+
+extern "C" int wq4_decode_step_host(const wq4_layer_table* table, const wq4_decode_attn* attn, const uint16_t* x_host,
+                                    uint16_t* logits_host, void* stream)
+{
+    if (!table || !attn || !x_host || !logits_host) return WQ4_ERR_INVALID;
+    cudaStream_t st = static_cast<cudaStream_t>(stream);
+    Plan pl;
+    int rc = get_plan(table, attn, &pl, st);
+    if (rc != WQ4_OK) return rc;
+    uint8_t* ws = static_cast<uint8_t*>(table->workspace);
+    uint16_t* xd = reinterpret_cast<uint16_t*>(ws + pl.lay.x_stage);
+    uint16_t* ld = reinterpret_cast<uint16_t*>(ws + pl.lay.logits_stage);
+    const size_t xb = static_cast<size_t>(pl.dims.B) * pl.dims.H * 2;
+    const size_t lb = static_cast<size_t>(pl.dims.B) * pl.dims.V * 2;
+    if (cudaMemcpyAsync(xd, x_host, xb, cudaMemcpyHostToDevice, st) != cudaSuccess) return WQ4_ERR_CUDA;
+    rc = launch_chain(pl, xd, ld, st);
+    if (rc != WQ4_OK) return rc;
+    if (cudaMemcpyAsync(logits_host, ld, lb, cudaMemcpyDeviceToHost, st) != cudaSuccess) return WQ4_ERR_CUDA;
+    return cudaStreamSynchronize(st) == cudaSuccess ? WQ4_OK : WQ4_ERR_CUDA;
 }
 
 extern "C" int wq4_test_chain_waits(uint64_t wait_limit_ns, int stall_stage)
@@ -1526,6 +2204,15 @@ extern "C" int wq4_chain_trace_offsets(const wq4_layer_table* table, int layer, 
     out->act = y.pM + 2 * l * B * F;
     out->down = y.pD + 2 * l * B * H;
     out->x_out = y.pX2 + 2 * l * B * H;
+    if (attn_heads_ok(d)) {
+        // decode step: the attention regions come after the chain's, and their
+        // offsets do not depend on the size of wq4_paged_attention's workspace
+        const Layout ya = make_layout(d, true, 0);
+        const size_t KD = static_cast<size_t>(d.Hkv) * kAttnD;
+        out->q_rot = ya.pQr + 2 * l * B * H;
+        out->k_rot = ya.pKr + 2 * l * B * KD;
+        out->attn = ya.pAt + 2 * l * B * H;
+    }
     return WQ4_OK;
 }
 
@@ -1585,7 +2272,7 @@ extern "C" int wq4_decode_chain_noalloc(const wq4_layer_table* table, const uint
     nd.table.workspace = nd.scratch;
     nd.table.workspace_bytes = kNoAllocScratchBytes;
     Plan pl;
-    const int rc = get_plan(&nd.table, &pl, st, true);
+    const int rc = get_plan(&nd.table, nullptr, &pl, st, true);
     if (rc != WQ4_OK) return rc;
     const size_t lb = static_cast<size_t>(pl.dims.B) * pl.dims.V * 2;
     if (overlaps(logits, lb, x, static_cast<size_t>(pl.dims.B) * pl.dims.H * 2)) return WQ4_ERR_INVALID;

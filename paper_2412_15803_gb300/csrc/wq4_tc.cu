@@ -741,7 +741,21 @@ void tc_plan_destroy(TcPlan* p) { delete p; }
 // may overlap its set-up and weight stream with the tail of the previous one
 // (programmatic dependent launch); it reads the previous stage's outputs only
 // after that grid has completed.
-int tc_record_token(const TcPlan* p, cudaStream_t cs)
+int tc_launch_prologue(const uint16_t* x, int H, int B, float* sq, uint16_t* xp, cudaStream_t cs)
+{
+    cudaLaunchAttribute attr[1];
+    attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+    attr[0].val.programmaticStreamSerializationAllowed = 1;
+    cudaLaunchConfig_t cfg = {};
+    cfg.gridDim = dim3(B);
+    cfg.blockDim = dim3(128);
+    cfg.stream = cs;
+    cfg.attrs = attr;
+    cfg.numAttrs = 1;
+    return cudaLaunchKernelEx(&cfg, tc_prologue_kernel, x, H, B, sq, xp) == cudaSuccess ? WQ4_OK : WQ4_ERR_CUDA;
+}
+
+int tc_record_token(const TcPlan* p, cudaStream_t cs, const TcAttnHook* att)
 {
     const int B = p->B, H = p->H, F = p->F, L = p->L;
     const TcBuffers& u = p->buf;
@@ -806,6 +820,8 @@ int tc_record_token(const TcPlan* p, cudaStream_t cs)
         a.ldxp = H;
         stage(kTcQKV, m[0], p->xH[hb], a);
         hb ^= 1;
+        // decode step: the attention output replaces the query block as O's input
+        if (att) ok = ok && att->record(att->ctx, l, cs, u.xpH[hb], sq_a) == WQ4_OK;
 
         a = TcArgs{};
         a.sq_in = sq_a;

@@ -42,7 +42,21 @@ int tc_plan_create(const wq4_layer_table* t, int H, int F, int Nqkv, int V, int 
                    uint32_t* err, TcPlan** out);
 void tc_plan_destroy(TcPlan* p);
 
-// Records one token (prologue and every stage kernel) on `cs`.
-int tc_record_token(const TcPlan* p, cudaStream_t cs);
+// Records the decode step's attention of layer `layer` on `cs`, between its
+// QKV and O stages: it must leave the O stage's permuted input in xp and the
+// sums of squares of its 128-element tiles in sq ([H/128][B]).
+struct TcAttnHook {
+    int (*record)(void* ctx, int layer, cudaStream_t cs, uint16_t* xp, float* sq);
+    void* ctx;
+};
+
+// Records one token (prologue and every stage kernel) on `cs`; with `att`,
+// the attention of every layer between its QKV and O stages.
+int tc_record_token(const TcPlan* p, cudaStream_t cs, const TcAttnHook* att = nullptr);
+
+// Records the token-start kernel on `cs` for an arbitrary [B][H] input: its
+// permuted copy into xp and the sums of squares of its 128-element tiles
+// into sq (programmatic dependent launch, like the stage kernels).
+int tc_launch_prologue(const uint16_t* x, int H, int B, float* sq, uint16_t* xp, cudaStream_t cs);
 
 }  // namespace wq4

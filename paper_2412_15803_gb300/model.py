@@ -80,10 +80,11 @@ class DecodeModel:
     including 15, reaches every kernel; fine for a few layers)."""
 
     def __init__(self, shape: ModelShape, batch: int = 1, seed: int = 0, eps: float = 1e-5, device=None,
-                 symmetric: bool = True):
+                 symmetric: bool = True, step: bool = False):
         import torch
         self.shape, self.batch, self.seed, self.eps = shape, batch, seed, eps
         self.symmetric = symmetric
+        self.step = step           # workspace sized for wq4_decode_step as well
         dev = torch.device("cuda") if device is None else torch.device(device)
         self.weights = []          # per layer: dict name -> (W tensor, s tensor)
         self._keep = []
@@ -112,6 +113,10 @@ class DecodeModel:
         nbytes = _w.wq4_chain_workspace_bytes(t)
         if nbytes == 0:
             raise ValueError(f"invalid chain shape {shape} batch {batch}")
+        if step:
+            nbytes = _w.wq4_decode_step_workspace_bytes(t)
+            if nbytes == 0:
+                raise ValueError(f"decode step unsupported for {shape} batch {batch}")
         self.workspace = torch.zeros(nbytes + 256, dtype=torch.uint8, device=dev)
         base = self.workspace.data_ptr()
         aligned = (base + 255) // 256 * 256
@@ -131,6 +136,14 @@ class DecodeModel:
     def decode_host(self, x_host: np.ndarray, logits_host: np.ndarray, stream=None) -> int:
         return _w.wq4_decode_chain_host(self.table, x_host, logits_host, stream)
 
+    def decode_step(self, caches: "StepCaches", x, logits, stream=None, check=True) -> int:
+        """One decode step with attention over `caches` (wq4_decode_step)."""
+        return _w.wq4_decode_step(self.table, caches.desc, x, logits, stream, check=check)
+
+    def decode_step_host(self, caches: "StepCaches", x_host: np.ndarray, logits_host: np.ndarray,
+                         stream=None) -> int:
+        return _w.wq4_decode_step_host(self.table, caches.desc, x_host, logits_host, stream)
+
     def destroy_plan(self) -> None:
         _w.wq4_chain_plan_destroy(self.table)
 
@@ -141,6 +154,8 @@ class DecodeModel:
         sh, B = self.shape, self.batch
         lens = dict(x_in=sh.hidden, qkv=sh.n_qkv, o=sh.hidden, x_mid=sh.hidden,
                     gate_up=2 * sh.ffn, act=sh.ffn, down=sh.hidden, x_out=sh.hidden)
+        if self.step:
+            lens.update(q_rot=sh.hidden, k_rot=sh.n_kv_heads * sh.head_dim, attn=sh.hidden)
         out = {}
         for name, n in lens.items():
             o = getattr(off, name)
@@ -159,3 +174,53 @@ class DecodeModel:
         else:
             (N, K, mat), lay = [(N, K, m) for nm, N, K, m in sh.mats(layer) if nm == name][0], layer
         return synth.matrix(self.seed, N, K, lay, mat, row_start, nrows, symmetric=self.symmetric)
+
+
+class StepCaches:
+    """The paged key/value caches of every layer of a decode step, on the
+    device: one page table shared by the layers (sequence b holds
+    positions[b] + 1 tokens after the step, pages drawn from a seeded
+    permutation of the pool), a cache pool per layer filled with the seeded
+    sum4 values, and the rows' positions (tokens already cached)."""
+
+    def __init__(self, shape: ModelShape, positions, page_size: int = 16, seed: int = 0, spare_pages: int = 0,
+                 rope_theta: float = 500000.0, device=None):
+        import math
+        import torch
+        dev = torch.device("cuda") if device is None else torch.device(device)
+        self.shape, self.page_size, self.seed = shape, page_size, seed
+        self.positions = np.asarray(positions, np.int32)
+        self.batch = len(self.positions)
+        Hkv, D, P = shape.n_kv_heads, shape.head_dim, page_size
+        lens = self.positions.astype(np.int64) + 1
+        need = (lens + P - 1) // P
+        self.num_pages = int(need.sum()) + spare_pages
+        self.table_host = synth.page_table(seed, lens, P, self.num_pages)
+        self.table = torch.from_numpy(self.table_host).to(dev)
+        self.pos_dev = torch.from_numpy(self.positions.copy()).to(dev)
+        n = self.num_pages * Hkv * P * D
+        self.k, self.v = [], []
+        descs = (_w.wq4_kv_cache * shape.num_layers)()
+        for l in range(shape.num_layers):
+            k = torch.empty((self.num_pages, Hkv, P, D), dtype=torch.int16, device=dev)
+            v = torch.empty_like(k)
+            _w.wq4_synth_sum4(k, 0, n, seed, synth.stream_id(synth.KIND_K, l, 0))
+            _w.wq4_synth_sum4(v, 0, n, seed, synth.stream_id(synth.KIND_V, l, 0))
+            self.k.append(k)
+            self.v.append(v)
+            descs[l] = _w.kv_cache_desc(k, v, self.table, P)
+        self._descs = descs
+        self.rope_theta = rope_theta
+        self.scale = 1.0 / math.sqrt(D)
+        self.desc = _w.wq4_decode_attn(descs, self.pos_dev.data_ptr(), rope_theta, self.scale)
+
+    def cache_bytes_read(self) -> int:
+        """Key and value bytes one step reads from the caches: every cached
+        token of every sequence and layer (the new token's row comes from the
+        projection)."""
+        sh = self.shape
+        return int(self.positions.astype(np.int64).sum()) * sh.n_kv_heads * sh.head_dim * 2 * 2 * sh.num_layers
+
+    def host_cache(self, layer: int):
+        """(k, v) fp16 bits [num_pages][n_kv_heads][page_size][head_dim] as they are now on the device."""
+        return (self.k[layer].cpu().numpy().view(np.uint16), self.v[layer].cpu().numpy().view(np.uint16))

@@ -56,7 +56,13 @@ class wq4_kv_cache(ctypes.Structure):
 
 
 class wq4_chain_trace(ctypes.Structure):
-    _fields_ = [(n, _SZ) for n in ("x_in", "qkv", "o", "x_mid", "gate_up", "act", "down", "x_out")]
+    _fields_ = [(n, _SZ) for n in ("x_in", "qkv", "o", "x_mid", "gate_up", "act", "down", "x_out",
+                                   "q_rot", "k_rot", "attn")]
+
+
+class wq4_decode_attn(ctypes.Structure):
+    _fields_ = [("layers", ctypes.POINTER(wq4_kv_cache)), ("positions", _P), ("rope_theta", ctypes.c_double),
+                ("scale", ctypes.c_float)]
 
 
 _lib = None
@@ -93,6 +99,10 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
     L.wq4_chain_trace_offsets.argtypes = [ctypes.POINTER(wq4_layer_table), _I,
                                           ctypes.POINTER(wq4_chain_trace)]
     L.wq4_test_chain_waits.argtypes = [_U64, _I]
+    L.wq4_decode_step_workspace_bytes.argtypes = [ctypes.POINTER(wq4_layer_table)]
+    L.wq4_decode_step_workspace_bytes.restype = _SZ
+    L.wq4_decode_step.argtypes = [ctypes.POINTER(wq4_layer_table), ctypes.POINTER(wq4_decode_attn), _P, _P, _P]
+    L.wq4_decode_step_host.argtypes = [ctypes.POINTER(wq4_layer_table), ctypes.POINTER(wq4_decode_attn), _P, _P, _P]
     L.wq4_synth_codes.argtypes = [_P, _I64, _I64, _U64, _U64, _I, _P]
     L.wq4_synth_scales.argtypes = [_P, _I64, _I64, _U64, _U64, ctypes.c_double, ctypes.c_double, _P]
     L.wq4_synth_sum4.argtypes = [_P, _I64, _I64, _U64, _U64, _P]
@@ -109,7 +119,7 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
 EXPORTED = ["wq4_gemv", "wq4_gemm", "wq4_unpack_debug", "wq4_pack_host", "wq4_status_string",
             "wq4_device_status", "wq4_chain_workspace_bytes", "wq4_decode_chain",
             "wq4_decode_chain_host", "wq4_decode_chain_noalloc", "wq4_chain_plan_destroy", "wq4_chain_trace_offsets",
-            "wq4_test_chain_waits",
+            "wq4_test_chain_waits", "wq4_decode_step_workspace_bytes", "wq4_decode_step", "wq4_decode_step_host",
             "wq4_synth_codes", "wq4_synth_scales", "wq4_synth_sum4",
             "wq4_paged_attention_workspace_bytes", "wq4_paged_attention", "wq4_kv_append"]
 
@@ -204,6 +214,22 @@ def wq4_chain_trace_offsets(table: wq4_layer_table, layer: int) -> wq4_chain_tra
     out = wq4_chain_trace()
     _check("wq4_chain_trace_offsets", load().wq4_chain_trace_offsets(ctypes.byref(table), layer, ctypes.byref(out)))
     return out
+
+
+def wq4_decode_step_workspace_bytes(table: wq4_layer_table) -> int:
+    return load().wq4_decode_step_workspace_bytes(ctypes.byref(table))
+
+
+def wq4_decode_step(table: wq4_layer_table, attn: wq4_decode_attn, x, logits, stream=None, check: bool = True) -> int:
+    rc = load().wq4_decode_step(ctypes.byref(table), ctypes.byref(attn), _ptr(x), _ptr(logits), _stream(stream))
+    return _check("wq4_decode_step", rc) if check else rc
+
+
+def wq4_decode_step_host(table: wq4_layer_table, attn: wq4_decode_attn, x_host, logits_host, stream=None,
+                         check: bool = True) -> int:
+    rc = load().wq4_decode_step_host(ctypes.byref(table), ctypes.byref(attn), _ptr(x_host), _ptr(logits_host),
+                                     _stream(stream))
+    return _check("wq4_decode_step_host", rc) if check else rc
 
 
 def wq4_test_chain_waits(wait_limit_ns: int, stall_stage: int = -1) -> None:

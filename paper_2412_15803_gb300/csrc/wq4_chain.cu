@@ -572,7 +572,7 @@ __device__ __forceinline__ uint16_t* append_row(const KvLayer& kv, int P, int Hk
 // q published for the attention, k and v appended to the cache and published
 // as the new token's key and value.
 template <int B>
-__device__ __noinline__ void qkv_epilogue_attn(const ChainParamsA& p, int l, int w, int b, float v0, float v1,
+__device__ __forceinline__ void qkv_epilogue_attn(const ChainParamsA& p, int l, int w, int b, float v0, float v1,
                                                   float rf, uint32_t epoch, const double2* rope, const int* pos_sh)
 {
     const int H = p.H, n = 2 * w, KD = p.Hkv * kAttnD;
@@ -627,25 +627,47 @@ __device__ __forceinline__ float warp_allsum(float v)
 }
 
 // The decode attention of layer l, run by the consumer warps of every CTA at
-// the start of the O stage.  Split u = blockIdx.x + k * gridDim.x is (row b,
-// kv head h, token range c of S); its warps take U consecutive tokens at a
-// time (lane: dimensions 4 lane .. 4 lane + 3), keep a running maximum, sum
-// and weighted value sum per query head of the group, combine the warps in
-// shared memory (one head at a time) and store the split's (o, m, l).  The
-// last split of (b, h) to arrive merges all S of them in split order and
-// publishes a = o / l.  scratch: qs[G][128] then per-warp partials
-// [NW][kAttnPart] floats (inside the staging area, free at this point).
+// the start of the O stage.  Row b's T = positions[b] + 1 tokens are cut into
+// S_b = min(S, ceil(T / kAttnSplitTokens)) equal ranges; unit u = blockIdx.x
+// + k * gridDim.x is (row b, kv head h, range c), ranges c >= S_b are empty.
+// The unit's warps take U consecutive tokens at a time (lane: dimensions
+// 4 lane .. 4 lane + 3; the range's page ids are staged in shared memory
+// first), keeping a running maximum, sum and weighted value sum per query
+// head of the group; the warps are combined in shared memory in warp order
+// (one head at a time).  With one range the unit publishes a = o / l
+// itself; otherwise it stores its (o, m, l) and the last range of (b, h) to
+// arrive merges all S_b of them in range order and publishes a.
+// Shared memory: xs area = qs[G][128] | wp[NW][kAttnPart]; header area from
+// kHdrRes (res and part are free until the O stage's staging) = acc[G][kAttnPart] |
+// pages[kAttnPageWindow].
+constexpr int kAttnSplitTokens = 128;
+constexpr int kAttnPageWindow = 256;
+static_assert(kHdrRes + 4 * (kAttnMaxGroup * kAttnPart + kAttnPageWindow + kAttnD) <= kChainHeader,
+              "attention scratch overlaps the staged input");
+
 template <int B, int NW, int G>
-__device__ __noinline__ void attention_phase(const ChainParamsA& p, int l, uint32_t epoch, float* scratch, const int* pos_sh,
-                                int* flag_sh)
+__device__ __forceinline__ void attention_phase(const ChainParamsA& p, int l, uint32_t epoch, float* scratch, const int* pos_sh,
+                                             int* flag_sh, uint8_t* smem)
 {
     constexpr int kConsumers = NW * 32;
-    constexpr int U = G <= 4 ? 8 : 4;          // tokens a warp has in flight
+    constexpr int U = G <= 3 ? 4 : 2;          // tokens a warp has in flight
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
-    const int H = p.H, Hkv = p.Hkv, S = p.S, KD = Hkv * kAttnD;
-    const KvLayer& kv = p.kv[l];
+    const int H = p.H, Hkv = p.Hkv, S = p.S, KD = Hkv * kAttnD, P = p.P;
+    const float scale = p.scale;
+    // the layer's cache and the outputs in registers (the parameter block is
+    // reached through a generic pointer here)
+    const KvLayer kv = p.kv[l];
+    uint16_t* const pAt = p.pAt;
+    uint64_t* const llAt = p.llAt;
+    const uint32_t repAt = p.repAt;
+    float* const apart = p.apart;
+    uint32_t* const acnt = p.acnt;
+    uint32_t* const err = p.err;
     float* qs = scratch;
     float* wp = scratch + G * kAttnD;
+    float* acc = reinterpret_cast<float*>(smem + kHdrRes);                       // [G][kAttnPart]
+    int* pages = reinterpret_cast<int*>(smem + kHdrRes) + G * kAttnPart;          // [kAttnPageWindow]
+    uint32_t* newkv = reinterpret_cast<uint32_t*>(pages + kAttnPageWindow);      // [2][64] the new key, value words
     const int nunits = B * Hkv * S;
     const uint64_t* qsrc = p.llA + ((blockIdx.x & 1) ? p.rep.A : 0u) + static_cast<size_t>(l) * B * (H / 2);
     for (int u = blockIdx.x; u < nunits; u += gridDim.x) {
@@ -654,25 +676,35 @@ __device__ __noinline__ void attention_phase(const ChainParamsA& p, int l, uint3
         const int h = rr / S, c = rr - h * S;
         const int pos = pos_sh[b];
         int T = pos + 1;                                        // 0 for an invalid position
-        const int cap = kv.pt_stride * p.P;
+        const int cap = kv.pt_stride * P;
         if (T > cap) {
             T = cap;
-            if (threadIdx.x == 0 && c == 0) atomicOr(p.err, kErrSeqLen);
+            if (threadIdx.x == 0 && c == 0) atomicOr(err, kErrSeqLen);
         }
-        const int t0 = static_cast<int>(static_cast<int64_t>(c) * T / S);
-        const int t1 = static_cast<int>(static_cast<int64_t>(c + 1) * T / S);
+        int Sb = (T + kAttnSplitTokens - 1) / kAttnSplitTokens;
+        Sb = Sb < 1 ? 1 : (Sb > S ? S : Sb);
+        if (c >= Sb) continue;                                  // uniform over the CTA
+        const int t0 = static_cast<int>(static_cast<int64_t>(c) * T / Sb);
+        const int t1 = static_cast<int>(static_cast<int64_t>(c + 1) * T / Sb);
         named_barrier_sync(1, kConsumers);                      // scratch free
-        for (int e = threadIdx.x; e < G * (kAttnD / 2); e += kConsumers) {
-            const int j = e / (kAttnD / 2), w = e - j * (kAttnD / 2);
-            const uint32_t qw = ll_load(qsrc + static_cast<size_t>(b) * (H / 2) + (h * G + j) * (kAttnD / 2) + w, epoch,
-                                        epoch, p.err, p.abort, p.wait_ns);
-            qs[j * kAttnD + 2 * w] = lo_f(qw);
-            qs[j * kAttnD + 2 * w + 1] = hi_f(qw);
+        // the group's queries and, in the range holding the new token, its key
+        // and value words: all polled at once
+        const bool has_new = pos >= t0 && pos < t1;
+        for (int e = threadIdx.x; e < G * (kAttnD / 2) + (has_new ? kAttnD : 0); e += kConsumers) {
+            if (e < G * (kAttnD / 2)) {
+                const int j = e / (kAttnD / 2), w = e - j * (kAttnD / 2);
+                const uint32_t qw = ll_load(qsrc + static_cast<size_t>(b) * (H / 2) + (h * G + j) * (kAttnD / 2) + w,
+                                            epoch, epoch, p.err, p.abort, p.wait_ns);
+                qs[j * kAttnD + 2 * w] = lo_f(qw);
+                qs[j * kAttnD + 2 * w + 1] = hi_f(qw);
+            } else {
+                const int i = e - G * (kAttnD / 2);             // 0..63 key words, 64..127 value words
+                const uint64_t* src = (i < kAttnD / 2 ? p.llK : p.llVn) +
+                                      (static_cast<size_t>(l) * B + b) * (KD / 2) + h * (kAttnD / 2) + (i & 63);
+                newkv[i] = ll_load(src, epoch, epoch, p.err, p.abort, p.wait_ns);
+            }
         }
-        named_barrier_sync(1, kConsumers);
         float4 qv[G];
-#pragma unroll
-        for (int j = 0; j < G; ++j) qv[j] = reinterpret_cast<const float4*>(qs + j * kAttnD)[lane];
         float m[G], ls[G], o[G][4];
 #pragma unroll
         for (int j = 0; j < G; ++j) {
@@ -680,59 +712,98 @@ __device__ __noinline__ void attention_phase(const ChainParamsA& p, int l, uint3
             ls[j] = 0.f;
             o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
         }
-        const uint64_t* knew = p.llK + (static_cast<size_t>(l) * B + b) * (KD / 2) + h * (kAttnD / 2) + 2 * lane;
-        const uint64_t* vnew = p.llVn + (static_cast<size_t>(l) * B + b) * (KD / 2) + h * (kAttnD / 2) + 2 * lane;
-        for (int base = t0 + warp * U; base < t1; base += NW * U) {
-            uint2 kr[U], vr[U];
-#pragma unroll
-            for (int uu = 0; uu < U; ++uu) {
-                const int t = base + uu;
-                kr[uu] = make_uint2(0u, 0u);
-                vr[uu] = make_uint2(0u, 0u);
-                if (t < t1 && t != pos) {
-                    const int pi = t / p.P;
-                    const int page = kv.pt[static_cast<size_t>(b) * kv.pt_stride + pi];
-                    if (page >= 0 && page < kv.num_pages) {
-                        const size_t row = ((static_cast<size_t>(page) * Hkv + h) * p.P + (t - pi * p.P)) * kAttnD;
-                        kr[uu] = __ldg(reinterpret_cast<const uint2*>(kv.k + row) + lane);
-                        vr[uu] = __ldg(reinterpret_cast<const uint2*>(kv.v + row) + lane);
-                    } else if (lane == 0) {
-                        atomicOr(p.err, kErrPageId);
-                    }
-                } else if (t == pos && t < t1) {
-                    // the new token: the QKV epilogue's flagged words
-                    kr[uu].x = ll_load(knew, epoch, epoch, p.err, p.abort, p.wait_ns);
-                    kr[uu].y = ll_load(knew + 1, epoch, epoch, p.err, p.abort, p.wait_ns);
-                    vr[uu].x = ll_load(vnew, epoch, epoch, p.err, p.abort, p.wait_ns);
-                    vr[uu].y = ll_load(vnew + 1, epoch, epoch, p.err, p.abort, p.wait_ns);
-                }
+        const int32_t* ptb = kv.pt + static_cast<size_t>(b) * kv.pt_stride;
+        // the range in windows of kAttnPageWindow pages
+        for (int wbeg = t0; wbeg < t1; wbeg += kAttnPageWindow * P - (wbeg % P)) {
+            const int wp0 = wbeg / P;
+            const int wend = min(t1, (wp0 + kAttnPageWindow) * P);
+            const int npg = (wend - 1) / P - wp0 + 1;
+            named_barrier_sync(1, kConsumers);                  // previous window's pages consumed; qs written
+            for (int i = threadIdx.x; i < npg; i += kConsumers) {
+                const int pid = __ldg(ptb + wp0 + i);
+                pages[i] = (pid >= 0 && pid < kv.num_pages) ? pid : -1;
+                if (pid < 0 || pid >= kv.num_pages) atomicOr(err, kErrPageId);
             }
+            named_barrier_sync(1, kConsumers);
+            if (wbeg == t0) {
 #pragma unroll
-            for (int uu = 0; uu < U; ++uu) {
-                if (base + uu >= t1) break;
-                const float k0 = lo_f(kr[uu].x), k1 = hi_f(kr[uu].x), k2 = lo_f(kr[uu].y), k3 = hi_f(kr[uu].y);
-                const float w0 = lo_f(vr[uu].x), w1 = hi_f(vr[uu].x), w2 = lo_f(vr[uu].y), w3 = hi_f(vr[uu].y);
-                float sc[G];
+                for (int j = 0; j < G; ++j) qv[j] = reinterpret_cast<const float4*>(qs + j * kAttnD)[lane];
+            }
+            for (int base = wbeg + warp * U; base < wend; base += NW * U) {
+                uint2 kr[U], vr[U];
 #pragma unroll
-                for (int j = 0; j < G; ++j) sc[j] = fmaf(qv[j].x, k0, fmaf(qv[j].y, k1, fmaf(qv[j].z, k2, qv[j].w * k3)));
+                for (int uu = 0; uu < U; ++uu) {
+                    const int t = base + uu;
+                    kr[uu] = make_uint2(0u, 0u);
+                    vr[uu] = make_uint2(0u, 0u);
+                    if (t < wend && t != pos) {
+                        const int pi = t / P;
+                        const int page = pages[pi - wp0];
+                        if (page >= 0) {
+                            const size_t row = ((static_cast<size_t>(page) * Hkv + h) * P + (t - pi * P)) * kAttnD;
+                            kr[uu] = __ldg(reinterpret_cast<const uint2*>(kv.k + row) + lane);
+                            vr[uu] = __ldg(reinterpret_cast<const uint2*>(kv.v + row) + lane);
+                        }
+                    }
+                }
+                if (pos >= base && pos < base + U && pos < wend) {
+                    // the new token: the words polled at the unit's start
+                    const int uu = pos - base;
+                    const uint2 nk = make_uint2(newkv[2 * lane], newkv[2 * lane + 1]);
+                    const uint2 nv = make_uint2(newkv[64 + 2 * lane], newkv[64 + 2 * lane + 1]);
 #pragma unroll
-                for (int j = 0; j < G; ++j) sc[j] = warp_allsum(sc[j]) * p.scale;
+                    for (int i = 0; i < U; ++i)
+                        if (i == uu) {
+                            kr[i] = nk;
+                            vr[i] = nv;
+                        }
+                }
+                // the batch's scores: U x G independent lane sums, reduced together
+                float sc[U][G];
+#pragma unroll
+                for (int uu = 0; uu < U; ++uu) {
+                    const float k0 = lo_f(kr[uu].x), k1 = hi_f(kr[uu].x), k2 = lo_f(kr[uu].y), k3 = hi_f(kr[uu].y);
+#pragma unroll
+                    for (int j = 0; j < G; ++j)
+                        sc[uu][j] = fmaf(qv[j].x, k0, fmaf(qv[j].y, k1, fmaf(qv[j].z, k2, qv[j].w * k3)));
+                }
+#pragma unroll
+                for (int off = 16; off > 0; off >>= 1)
+#pragma unroll
+                    for (int uu = 0; uu < U; ++uu)
+#pragma unroll
+                        for (int j = 0; j < G; ++j) sc[uu][j] += __shfl_xor_sync(0xffffffffu, sc[uu][j], off);
+                // one running-maximum update per batch (the batch's first token is valid)
 #pragma unroll
                 for (int j = 0; j < G; ++j) {
-                    const float mn = fmaxf(m[j], sc[j]);
-                    const float corr = expf(m[j] - mn);
-                    const float pw = expf(sc[j] - mn);
-                    ls[j] = fmaf(ls[j], corr, pw);
-                    o[j][0] = fmaf(o[j][0], corr, pw * w0);
-                    o[j][1] = fmaf(o[j][1], corr, pw * w1);
-                    o[j][2] = fmaf(o[j][2], corr, pw * w2);
-                    o[j][3] = fmaf(o[j][3], corr, pw * w3);
-                    m[j] = mn;
+                    float mb = m[j];
+#pragma unroll
+                    for (int uu = 0; uu < U; ++uu) {
+                        sc[uu][j] *= scale;
+                        if (base + uu < wend) mb = fmaxf(mb, sc[uu][j]);
+                    }
+                    const float corr = expf(m[j] - mb);
+                    float lsum = ls[j] * corr;
+                    float o0 = o[j][0] * corr, o1 = o[j][1] * corr, o2 = o[j][2] * corr, o3 = o[j][3] * corr;
+#pragma unroll
+                    for (int uu = 0; uu < U; ++uu) {
+                        const float pw = (base + uu < wend) ? expf(sc[uu][j] - mb) : 0.f;
+                        lsum += pw;
+                        o0 = fmaf(pw, lo_f(vr[uu].x), o0);
+                        o1 = fmaf(pw, hi_f(vr[uu].x), o1);
+                        o2 = fmaf(pw, lo_f(vr[uu].y), o2);
+                        o3 = fmaf(pw, hi_f(vr[uu].y), o3);
+                    }
+                    ls[j] = lsum;
+                    o[j][0] = o0;
+                    o[j][1] = o1;
+                    o[j][2] = o2;
+                    o[j][3] = o3;
+                    m[j] = mb;
                 }
             }
         }
-        // combine the warps, one query head at a time; store the split's partial
-        float* dst = p.apart + ((((static_cast<size_t>(l) * B + b) * Hkv + h) * S + c) * G) * kAttnPart;
+        // combine the warps in warp order, one query head at a time, into acc
 #pragma unroll
         for (int j = 0; j < G; ++j) {
             float* mine = wp + warp * kAttnPart;
@@ -745,55 +816,94 @@ __device__ __noinline__ void attention_phase(const ChainParamsA& p, int l, uint3
             if (threadIdx.x < kAttnD) {
                 const int d = threadIdx.x;
                 float M = -INFINITY;
+#pragma unroll
                 for (int w = 0; w < NW; ++w) M = fmaxf(M, wp[w * kAttnPart + kAttnD]);
                 float Ls = 0.f, Od = 0.f;
                 if (M != -INFINITY) {
+#pragma unroll
                     for (int w = 0; w < NW; ++w) {
                         const float f = expf(wp[w * kAttnPart + kAttnD] - M);   // 0 for a warp without tokens
                         Ls = fmaf(f, wp[w * kAttnPart + kAttnD + 1], Ls);
                         Od = fmaf(f, wp[w * kAttnPart + d], Od);
                     }
                 }
-                dst[j * kAttnPart + d] = Od;
+                acc[j * kAttnPart + d] = Od;
                 if (d == 0) {
-                    dst[j * kAttnPart + kAttnD] = M;
-                    dst[j * kAttnPart + kAttnD + 1] = Ls;
+                    acc[j * kAttnPart + kAttnD] = M;
+                    acc[j * kAttnPart + kAttnD + 1] = Ls;
                 }
-                __threadfence();
             }
             named_barrier_sync(1, kConsumers);
         }
+        if (Sb == 1) {
+            // one range: this unit's result is the attention output
+            for (int e = threadIdx.x; e < G * (kAttnD / 2); e += kConsumers) {
+                const int j = e / (kAttnD / 2), w = e - j * (kAttnD / 2);
+                const float Ls = acc[j * kAttnPart + kAttnD + 1];
+                const float a0 = Ls > 0.f ? acc[j * kAttnPart + 2 * w] / Ls : 0.f;
+                const float a1 = Ls > 0.f ? acc[j * kAttnPart + 2 * w + 1] / Ls : 0.f;
+                const uint32_t aw = pack2(float_to_half_bits(a0), float_to_half_bits(a1));
+                const int n = (h * G + j) * kAttnD + 2 * w;
+                *reinterpret_cast<uint32_t*>(pAt + (static_cast<size_t>(l) * B + b) * H + n) = aw;
+                ll_store2(llAt + (static_cast<size_t>(l) * B + b) * (H / 2) + n / 2, repAt, aw, epoch);
+            }
+            continue;                                           // the next unit starts with a barrier
+        }
+        // store the range's partial, then arrive
+        float* dst = apart + ((((static_cast<size_t>(l) * B + b) * Hkv + h) * S + c) * G) * kAttnPart;
+        for (int e = threadIdx.x; e < G * (kAttnD + 2); e += kConsumers) {
+            const int j = e / (kAttnD + 2), d = e - j * (kAttnD + 2);
+            dst[j * kAttnPart + d] = acc[j * kAttnPart + d];
+        }
+        __threadfence();
+        named_barrier_sync(1, kConsumers);
         if (threadIdx.x == 0) {
-            __threadfence();
-            const uint32_t prev = atomicAdd(p.acnt + (static_cast<size_t>(l) * B + b) * Hkv + h, 1u);
-            *flag_sh = (prev == static_cast<uint32_t>(S - 1)) ? 1 : 0;
+            const uint32_t prev = atomicAdd(acnt + (static_cast<size_t>(l) * B + b) * Hkv + h, 1u);
+            *flag_sh = (prev == static_cast<uint32_t>(Sb - 1)) ? 1 : 0;
             __threadfence();
         }
         named_barrier_sync(1, kConsumers);
         if (*flag_sh) {
-            // every split of (b, h) is in: merge them in split order
-            const float* src = p.apart + (((static_cast<size_t>(l) * B + b) * Hkv + h) * S) * G * kAttnPart;
+            // every range of (b, h) is in: merge them in range order; the ranges'
+            // (m, l) first (all loads in flight), then per thread a pair of
+            // dimensions of a head with its Sb loads in flight
+            const float* src = apart + (((static_cast<size_t>(l) * B + b) * Hkv + h) * S) * G * kAttnPart;
+            float2* ml = reinterpret_cast<float2*>(wp);              // [Sb][G]
+            for (int e = threadIdx.x; e < Sb * G; e += kConsumers)
+                ml[e] = __ldcg(reinterpret_cast<const float2*>(src + e * kAttnPart + kAttnD));
+            named_barrier_sync(1, kConsumers);
             for (int e = threadIdx.x; e < G * (kAttnD / 2); e += kConsumers) {
                 const int j = e / (kAttnD / 2), w = e - j * (kAttnD / 2);
                 float M = -INFINITY;
-                for (int cc = 0; cc < S; ++cc) M = fmaxf(M, __ldcg(src + (cc * G + j) * kAttnPart + kAttnD));
+                for (int cc = 0; cc < Sb; ++cc) M = fmaxf(M, ml[cc * G + j].x);
                 float Ls = 0.f, O0 = 0.f, O1 = 0.f;
                 if (M != -INFINITY) {
-                    for (int cc = 0; cc < S; ++cc) {
-                        const float* pc = src + (cc * G + j) * kAttnPart;
-                        const float f = expf(__ldcg(pc + kAttnD) - M);
-                        Ls = fmaf(f, __ldcg(pc + kAttnD + 1), Ls);
-                        O0 = fmaf(f, __ldcg(pc + 2 * w), O0);
-                        O1 = fmaf(f, __ldcg(pc + 2 * w + 1), O1);
+                    constexpr int kBatch = 16;                  // loads in flight per thread
+                    for (int c0 = 0; c0 < Sb; c0 += kBatch) {
+                        float2 ov[kBatch];
+#pragma unroll
+                        for (int i = 0; i < kBatch; ++i)
+                            ov[i] = (c0 + i < Sb)
+                                        ? __ldcg(reinterpret_cast<const float2*>(src + ((c0 + i) * G + j) * kAttnPart) + w)
+                                        : make_float2(0.f, 0.f);
+#pragma unroll
+                        for (int i = 0; i < kBatch; ++i) {
+                            if (c0 + i >= Sb) break;
+                            const float2 mlc = ml[(c0 + i) * G + j];
+                            const float f = expf(mlc.x - M);
+                            Ls = fmaf(f, mlc.y, Ls);
+                            O0 = fmaf(f, ov[i].x, O0);
+                            O1 = fmaf(f, ov[i].y, O1);
+                        }
                     }
                 }
                 const float a0 = Ls > 0.f ? O0 / Ls : 0.f, a1 = Ls > 0.f ? O1 / Ls : 0.f;
                 const uint32_t aw = pack2(float_to_half_bits(a0), float_to_half_bits(a1));
                 const int n = (h * G + j) * kAttnD + 2 * w;
-                *reinterpret_cast<uint32_t*>(p.pAt + (static_cast<size_t>(l) * B + b) * H + n) = aw;
-                ll_store2(p.llAt + (static_cast<size_t>(l) * B + b) * (H / 2) + n / 2, p.repAt, aw, epoch);
+                *reinterpret_cast<uint32_t*>(pAt + (static_cast<size_t>(l) * B + b) * H + n) = aw;
+                ll_store2(llAt + (static_cast<size_t>(l) * B + b) * (H / 2) + n / 2, repAt, aw, epoch);
             }
-            if (threadIdx.x == 0) p.acnt[(static_cast<size_t>(l) * B + b) * Hkv + h] = 0u;   // for the next token
+            if (threadIdx.x == 0) acnt[(static_cast<size_t>(l) * B + b) * Hkv + h] = 0u;   // for the next token
         }
     }
     named_barrier_sync(1, kConsumers);                          // scratch free for the staging
@@ -801,17 +911,17 @@ __device__ __noinline__ void attention_phase(const ChainParamsA& p, int l, uint3
 
 template <int B, int NW>
 __device__ __forceinline__ void attention_dispatch(const ChainParamsA& p, int l, uint32_t epoch, float* scratch,
-                                                   const int* pos_sh, int* flag_sh)
+                                                   const int* pos_sh, int* flag_sh, uint8_t* smem)
 {
     switch (p.G) {
-        case 1: attention_phase<B, NW, 1>(p, l, epoch, scratch, pos_sh, flag_sh); break;
-        case 2: attention_phase<B, NW, 2>(p, l, epoch, scratch, pos_sh, flag_sh); break;
-        case 3: attention_phase<B, NW, 3>(p, l, epoch, scratch, pos_sh, flag_sh); break;
-        case 4: attention_phase<B, NW, 4>(p, l, epoch, scratch, pos_sh, flag_sh); break;
-        case 5: attention_phase<B, NW, 5>(p, l, epoch, scratch, pos_sh, flag_sh); break;
-        case 6: attention_phase<B, NW, 6>(p, l, epoch, scratch, pos_sh, flag_sh); break;
-        case 7: attention_phase<B, NW, 7>(p, l, epoch, scratch, pos_sh, flag_sh); break;
-        default: attention_phase<B, NW, 8>(p, l, epoch, scratch, pos_sh, flag_sh); break;
+        case 1: attention_phase<B, NW, 1>(p, l, epoch, scratch, pos_sh, flag_sh, smem); break;
+        case 2: attention_phase<B, NW, 2>(p, l, epoch, scratch, pos_sh, flag_sh, smem); break;
+        case 3: attention_phase<B, NW, 3>(p, l, epoch, scratch, pos_sh, flag_sh, smem); break;
+        case 4: attention_phase<B, NW, 4>(p, l, epoch, scratch, pos_sh, flag_sh, smem); break;
+        case 5: attention_phase<B, NW, 5>(p, l, epoch, scratch, pos_sh, flag_sh, smem); break;
+        case 6: attention_phase<B, NW, 6>(p, l, epoch, scratch, pos_sh, flag_sh, smem); break;
+        case 7: attention_phase<B, NW, 7>(p, l, epoch, scratch, pos_sh, flag_sh, smem); break;
+        default: attention_phase<B, NW, 8>(p, l, epoch, scratch, pos_sh, flag_sh, smem); break;
     }
 }
 
@@ -849,15 +959,12 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1)
     }
     if (threadIdx.x < kMaxChainBatch * 32) red[threadIdx.x] = 0.f;   // warps >= NW stay zero
     // decode step: the rotation table (cos, sin of pos * theta^(-2i/128) per
-    // row, fp64) and the rows' positions (-1 for an invalid one)
-    double2* rope = nullptr;
-    int* pos_sh = nullptr;
-    int* flag_sh = nullptr;
+    // row, fp64) and the rows' positions (-1 for an invalid one), after the
+    // ring; their addresses are recomputed where used (no registers held)
+    constexpr uint32_t kPosOff = B * (kAttnD / 2) * sizeof(double2);
     if constexpr (ATT) {
-        rope = reinterpret_cast<double2*>(smem + p.rope_off);
-        pos_sh = reinterpret_cast<int*>(smem + p.rope_off + B * (kAttnD / 2) * sizeof(double2));
-        flag_sh = pos_sh + kMaxChainBatch;
-        rope_table<B>(p, rope);
+        rope_table<B>(p, reinterpret_cast<double2*>(smem + p.rope_off));
+        int* pos_sh = reinterpret_cast<int*>(smem + p.rope_off + kPosOff);
         if (threadIdx.x < B) {
             const int pos = __ldg(p.positions + threadIdx.x);
             pos_sh[threadIdx.x] = pos < 0 ? -1 : pos;
@@ -937,8 +1044,11 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1)
             const StageInfo& in = info[g.type];
             if constexpr (ATT) {
                 // every CTA takes its splits of the layer's attention, words or not
-                if (g.type == kO)
-                    attention_dispatch<B, NW>(p, g.layer, epoch, reinterpret_cast<float*>(xs), pos_sh, flag_sh);
+                if (g.type == kO) {
+                    int* pos_sh = reinterpret_cast<int*>(smem + p.rope_off + kPosOff);
+                    attention_dispatch<B, NW>(p, g.layer, epoch, reinterpret_cast<float*>(xs), pos_sh,
+                                              pos_sh + kMaxChainBatch, smem);
+                }
             }
             if (in.nwords <= 0) continue;
             const int l = g.layer;
@@ -1200,6 +1310,8 @@ __global__ void __launch_bounds__((NW + 1) * 32, 1)
                     if (bb != b) continue;
                     if constexpr (ATT) {
                         if (g.type == kQKV) {
+                            const double2* rope = reinterpret_cast<const double2*>(smem + p.rope_off);
+                            const int* pos_sh = reinterpret_cast<const int*>(smem + p.rope_off + kPosOff);
                             qkv_epilogue_attn<B>(p, l, w0 + wc, bb, sum.x, sum.y, rf[bb], epoch, rope, pos_sh);
                             if (spw == 2 && wc + 1 < nwd)
                                 qkv_epilogue_attn<B>(p, l, w0 + wc + 1, bb, sum.z, sum.w, rf[bb], epoch, rope, pos_sh);

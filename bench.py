@@ -48,6 +48,8 @@ PERSISTENT_MAX_BATCH = 2      # larger batches run the tensor-core graph path
 # the paper's batch-1 decode rates for these model shapes (Table 1, WebLLM in
 # Chrome on an Apple M3 Max, 4-bit weights): another machine's numbers, context only
 PAPER_DECODE_TOKS = {"8b": 41.1, "phi3.5": 71.1}
+# rotary base of the model families the shapes follow (Llama-3.x, Phi-3.5)
+ROPE_THETA = {"3b": 500000.0, "8b": 500000.0, "phi3.5": 10000.0}
 FALLBACK_HBM_GBS = 6800.0
 L2_BYTES = 129 * 1024 * 1024
 
@@ -64,6 +66,9 @@ def parse():
     ap.add_argument("--tokens", type=int, default=2048, help="prompt tokens of the prefill workload")
     ap.add_argument("--batch", type=int, default=1)
     ap.add_argument("--layers", type=int, default=0, help="override the layer count (profiling runs)")
+    ap.add_argument("--context", type=int, default=0,
+                    help="decode step with attention (wq4_decode_step) at this many tokens of context "
+                         "(0: the GEMV-bound chain with the query-block stand-in)")
     ap.add_argument("--no-cpu-baseline", action="store_true")
     return ap.parse_args()
 
@@ -99,11 +104,12 @@ def chain_source_sha(kernel: str) -> str:
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(workload: str, batch: int):
+def profiled_traffic(workload: str, batch: int, context: int = 0):
     """DRAM bytes per launch from the committed ncu summary, if it was taken
     on the current kernel source (else None)."""
     name = "chain_kernel" if batch <= PERSISTENT_MAX_BATCH else "tc_stage_kernel"
-    path = os.path.join(ROOT, "profiles", f"{name}_{workload}_b{batch}.md")
+    ctx = f"_ctx{context}" if context else ""
+    path = os.path.join(ROOT, "profiles", f"{name}_{workload}_b{batch}{ctx}.md")
     if not os.path.exists(path):
         return None
     text = open(path).read()
@@ -264,7 +270,23 @@ def all_core_line(value: float, unit: str, threads: int, sample: str) -> dict:
             "sample": sample}
 
 
-def cpu_baseline(shape, batch, target_s=12.0):
+def oracle_attention_layer_s(shape, batch: int, context: int, seed: int = 0) -> float:
+    """Seconds of the fp64 oracle's paged attention for one layer of a decode
+    step: every row attends to `context` tokens of a seeded paged cache."""
+    import oracle
+    from paper_2412_15803_gb300 import synth
+    P, D = 16, shape.head_dim
+    lens = np.full(batch, context, np.int32)
+    num_pages = int(((lens + P - 1) // P).sum())
+    table = synth.page_table(seed, lens, P, num_pages)
+    k, v = synth.kv_cache(seed, num_pages, shape.n_kv_heads, P, D)
+    q = synth.queries(seed, batch, shape.n_q_heads, D)
+    t0 = time.perf_counter()
+    oracle.paged_attention(q, k, v, table, lens, 1.0 / np.sqrt(D), shape.n_q_heads)
+    return time.perf_counter() - t0
+
+
+def cpu_baseline(shape, batch, target_s=12.0, context: int = 0):
     per_w = oracle_rate_estimate(shape, batch)
     frac = min(1.0, target_s / max(per_w * shape.weight_count(), 1e-9))
     t, w = oracle_sample(shape, batch, frac)
@@ -273,13 +295,24 @@ def cpu_baseline(shape, batch, target_s=12.0):
     pool = RowPool(host["nproc"])
     tp, wp = oracle_sample(shape, batch, frac, pool=pool)
     pool.close()
-    return {"value": tokens / t, "unit": "tokens/s", "cores": 1, "kind": "oracle",
+    line = {"value": tokens / t, "unit": "tokens/s", "cores": 1, "kind": "oracle",
             "sample": f"first {frac:.4f} of the rows of all {4 * shape.num_layers + 1} projections "
                       f"({w} weights = {w / shape.weight_count():.4f} of a token), batch {batch}, "
                       f"single-threaded fp64 C oracle, {t:.1f} s",
             **host,
             "all_core": all_core_line(batch * wp / shape.weight_count() / tp, "tokens/s", pool.threads,
                                       f"the same rows, {tp:.1f} s")}
+    if context:
+        # a step adds every layer's attention: timed on one layer, counted L times
+        ta = oracle_attention_layer_s(shape, batch, context)
+        step_s = t * shape.weight_count() / w + shape.num_layers * ta
+        line["value"] = batch / step_s
+        line["sample"] += (f"; plus the oracle's attention of one layer over {context} tokens x {batch} rows "
+                           f"({ta:.2f} s), counted for all {shape.num_layers} layers")
+        step_p = tp * shape.weight_count() / wp + shape.num_layers * ta
+        line["all_core"]["value"] = batch / step_p
+        line["all_core"]["sample"] += " (the attention single-threaded)"
+    return line
 
 
 def chain_step_bytes(shape, B: int) -> int:
@@ -288,13 +321,18 @@ def chain_step_bytes(shape, B: int) -> int:
     return shape.weight_bytes() + 2 * B * (shape.hidden * (4 * shape.num_layers + 1) + shape.vocab)
 
 
-def chain_config(shape, B: int, world: int) -> dict:
+def chain_config(shape, B: int, world: int, context: int = 0) -> dict:
     """The workload's config object, the same for both arms."""
-    return {"workload": f"{shape.name}-shaped decode chain: {shape.num_layers} layers x "
+    what = "decode chain" if not context else \
+        f"decode step with attention ({shape.n_q_heads} q / {shape.n_kv_heads} kv heads of {shape.head_dim}, " \
+        f"RoPE, paged KV cache of 16-token pages, {context} tokens of context per row)"
+    kv = 0 if not context else context - 1
+    kv_bytes = B * kv * shape.n_kv_heads * shape.head_dim * 2 * 2 * shape.num_layers
+    return {"workload": f"{shape.name}-shaped {what}: {shape.num_layers} layers x "
                         f"(QKV {shape.n_qkv}x{shape.hidden}, O {shape.hidden}x{shape.hidden}, "
                         f"gate_up {2 * shape.ffn}x{shape.hidden}, down {shape.hidden}x{shape.ffn}) "
                         f"+ LM head {shape.vocab}x{shape.hidden}, batch {B}",
-            "batch": B, "bytes_per_token": chain_step_bytes(shape, B),
+            "batch": B, "context": context, "bytes_per_token": chain_step_bytes(shape, B) + kv_bytes,
             "l2": "inputs larger than L2 (1.8+ GB of weights per step), no flush",
             "codes": "drawn uniform on 0..14 (zero-mean q - 7), not 0..15: with 0..15 the mean offset of "
                      "+0.5 per weight compounds through 28-32 layers and overflows fp16 in the oracle's own "
@@ -308,26 +346,33 @@ def run_reference(args, rank, world):
     if rank != 0:
         return
     shape = SHAPES[args.workload]
+    T = args.context
     per_w = oracle_rate_estimate(shape, args.batch)
     nsteps = args.steps + args.warmup
     step_s = min(10.0, 120.0 / max(nsteps, 1))
     frac = min(1.0, step_s / (per_w * shape.weight_count()))
-    times, wsum = [], 0
+    # with attention, one layer's attention is timed once per step as well
+    times, wsum, atimes = [], 0, []
     for i in range(nsteps):
         t, w = oracle_sample(shape, args.batch, frac)
+        a = oracle_attention_layer_s(shape, args.batch, T, seed=i) if T and i >= args.warmup else 0.0
         if i >= args.warmup:
             times.append(t)
+            atimes.append(a)
             wsum += w
-    tok = args.batch * wsum / shape.weight_count()
-    value = tok / sum(times)
+    steps = len(times)
+    token_s = sum(times) * shape.weight_count() / wsum + shape.num_layers * (sum(atimes) / steps if T else 0.0)
+    value = args.batch / token_s
+    sample = (f"each step: first {frac:.5f} of the rows of every projection "
+              f"(all {4 * shape.num_layers + 1}), scaled to a token by weights")
+    if T:
+        sample += f"; plus one layer's attention over {T} tokens, counted for all {shape.num_layers} layers"
     line = {"metric": METRIC, "value": value, "unit": "tokens/s", "n_gpus": world, "steps": args.steps,
-            "warmup": args.warmup, "ms_per_step": 1e3 * sum(times) / len(times), "higher_is_better": True,
+            "warmup": args.warmup, "ms_per_step": 1e3 * token_s, "higher_is_better": True,
             "scaling": "weak", "vs_baseline": None, "dtype": "f64",
             "data": "synthetic (seeded SplitMix64 weights and activations)", "impl": "reference",
-            "config": chain_config(shape, args.batch, world),
-            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle",
-                             "sample": f"each step: first {frac:.5f} of the rows of every projection "
-                                       f"(all {4 * shape.num_layers + 1}), scaled to a token by weights",
+            "config": chain_config(shape, args.batch, world, T),
+            "cpu_baseline": {"value": value, "unit": "tokens/s", "cores": 1, "kind": "oracle", "sample": sample,
                              **host_info()},
             "e2e": {"value": value, "unit": "tokens/s", "h2d_bytes_per_step": 0, "d2h_bytes_per_step": 0}}
     print(json.dumps(line), flush=True)
@@ -356,7 +401,7 @@ def run_ours(args, rank, world, local):
     import torch
     import torch.distributed as dist
     from paper_2412_15803_gb300 import synth, wq4
-    from paper_2412_15803_gb300.model import SHAPES, DecodeModel
+    from paper_2412_15803_gb300.model import SHAPES, DecodeModel, StepCaches
 
     torch.cuda.set_device(local)
     if world > 1:
@@ -366,16 +411,33 @@ def run_ours(args, rank, world, local):
         import dataclasses
         shape = dataclasses.replace(shape, name=f"{shape.name}-{args.layers}l", num_layers=args.layers)
     B = args.batch
-    model = DecodeModel(shape, batch=B, seed=0)
+    T = args.context
+    model = DecodeModel(shape, batch=B, seed=0, step=T > 0)
     x_np = synth.activations(1000 + rank, B, shape.hidden)
     x = torch.from_numpy(x_np.view(np.int16)).cuda()
     logits = torch.empty((B, shape.vocab), dtype=torch.int16, device="cuda")
     stream = torch.cuda.current_stream()
 
     step_bytes = chain_step_bytes(shape, B)
+    if T > 0:
+        # every row decodes the token at position T - 1: it attends to T tokens
+        caches = StepCaches(shape, [T - 1] * B, seed=1, rope_theta=ROPE_THETA.get(args.workload, 500000.0))
+        step_bytes += caches.cache_bytes_read()
+
+        def decode():
+            model.decode_step(caches, x, logits, stream)
+
+        def decode_host(xh, lh):
+            model.decode_step_host(caches, xh, lh, stream)
+    else:
+        def decode():
+            model.decode(x, logits, stream)
+
+        def decode_host(xh, lh):
+            model.decode_host(xh, lh, stream)
 
     for _ in range(args.warmup):
-        model.decode(x, logits, stream)
+        decode()
     torch.cuda.synchronize()
     if wq4.wq4_device_status(stream) != 0:
         raise RuntimeError("device wait timed out during warm-up")
@@ -390,7 +452,7 @@ def run_ours(args, rank, world, local):
     torch.cuda.synchronize()
     for i in range(args.steps):
         starts[i].record(stream)
-        model.decode(x, logits, stream)
+        decode()
         ends[i].record(stream)
     torch.cuda.synchronize()
     if world > 1:
@@ -406,10 +468,10 @@ def run_ours(args, rank, world, local):
     l_host = torch.empty((B, shape.vocab), dtype=torch.int16).pin_memory()
     e2e_steps = max(10, min(args.steps, 500))
     for _ in range(3):
-        model.decode_host(x_host.numpy(), l_host.numpy(), stream)
+        decode_host(x_host.numpy(), l_host.numpy())
     t0 = time.perf_counter()
     for _ in range(e2e_steps):
-        model.decode_host(x_host.numpy(), l_host.numpy(), stream)
+        decode_host(x_host.numpy(), l_host.numpy())
     e2e_s = time.perf_counter() - t0
     tokens_per_s, e2e_val, total_ms_max = aggregate_replicas(total_ms, e2e_s / e2e_steps, B, args.steps, "cuda")
 
@@ -417,8 +479,10 @@ def run_ours(args, rank, world, local):
         # one cooperative launch of the persistent chain kernel per token
         kernel_name, launches_per_step = "chain_kernel", 1
     else:
-        # one CUDA-graph replay: a prologue and one tensor-core stage kernel per projection
-        kernel_name, launches_per_step = "tc_stage_kernel", 4 * shape.num_layers + 2
+        # one CUDA-graph replay: a prologue and one tensor-core stage kernel per
+        # projection (with attention, three more a layer: rotation/append,
+        # paged attention, the O input's token-start kernel)
+        kernel_name, launches_per_step = "tc_stage_kernel", 4 * shape.num_layers + 2 + (3 * shape.num_layers if T else 0)
     if rank == 0:
         ms = total_ms_max / args.steps
         avg_launch_ms = statistics.mean(launch_ms)
@@ -429,17 +493,18 @@ def run_ours(args, rank, world, local):
             "steps": args.steps, "warmup": args.warmup, "ms_per_step": ms, "higher_is_better": True,
             "scaling": "weak",
             "vs_baseline": (tokens_per_s / PAPER_DECODE_TOKS[args.workload]
-                            if B == 1 and args.workload in PAPER_DECODE_TOKS and not args.layers else None),
+                            if B == 1 and args.workload in PAPER_DECODE_TOKS and not args.layers and not T
+                            else None),
             "dtype": "f32",
             "precision": "int4 codes (group 32, fp16 scale, zero point 7), fp16 activations, fp32 accumulation",
             "data": "synthetic (seeded SplitMix64 weights and activations)",
-            "config": chain_config(shape, B, world),
+            "config": chain_config(shape, B, world, T),
             "hbm_gbs": step_bytes * args.steps / (total_ms_max / 1e3) / 1e9,
             "hbm_frac_of_nominal_8tbs": step_bytes * args.steps / (total_ms_max / 1e3) / 1e9 / NOMINAL_HBM_GBS,
             "roofline": {"bound": "hbm", "kernel": kernel_name, "achieved": achieved, "peak": peak,
                          "peak_source": peak_src, "unit": "GB/s", "frac": achieved / peak,
                          "frac_of_nominal_8tbs": achieved / NOMINAL_HBM_GBS,
-                         "traffic": profiled_traffic(args.workload, B),
+                         "traffic": profiled_traffic(args.workload, B, T),
                          "algorithmic_bytes_per_launch": step_bytes,
                          "avg_launch_ms": avg_launch_ms},
             "e2e": {"value": e2e_val, "unit": "tokens/s", "h2d_bytes_per_step": 2 * B * shape.hidden,
@@ -451,7 +516,7 @@ def run_ours(args, rank, world, local):
             line["vs_baseline_ref"] = (f"paper Table 1: {PAPER_DECODE_TOKS[args.workload]} tok/s, WebLLM on an Apple "
                                        "M3 Max (other hardware, trained weights)")
         if world == 1 and not args.no_cpu_baseline:
-            line["cpu_baseline"] = cpu_baseline(shape, B)
+            line["cpu_baseline"] = cpu_baseline(shape, B, context=T)
         print(json.dumps(line), flush=True)
     if world > 1:
         dist.destroy_process_group()

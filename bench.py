@@ -90,7 +90,7 @@ def measured_peak():
 
 
 KERNEL_SOURCES = {
-    "chain_kernel": ("wq4_chain.cu", "wq4_device.cuh"),
+    "chain_kernel": ("wq4_chain.cu", "wq4_items.cuh", "wq4_device.cuh"),
     "tc_stage_kernel": ("wq4_tc.cu", "wq4_tc.cuh", "wq4_device.cuh"),
 }
 
@@ -545,19 +545,29 @@ def gemv_copies(mats) -> int:
     return -(-4 * L2_BYTES // gemv_set_bytes(mats)) + 1
 
 
+def gemv_kernel_names(mats, B: int) -> str:
+    """The kernels wq4_gemv's size rule picks for the set (batch 1-2, K % 256 == 0)."""
+    names = []
+    for _, N, K in mats:
+        k = "gemv_mma_kernel" if B <= 2 and K % 256 == 0 and N * K >= 32 << 20 else "gemv_tma_kernel"
+        if k not in names:
+            names.append(k)
+    return "+".join(names)
+
+
 def gemv_io_bytes(mats, B: int) -> int:
     return sum(2 * B * (N + K) for _, N, K in mats)
 
 
 def gemv_source_sha() -> str:
     h = hashlib.sha256()
-    for f in ("wq4_gemv.cu", "wq4_device.cuh"):
+    for f in ("wq4_gemv.cu", "wq4_items.cuh", "wq4_device.cuh"):
         h.update(open(os.path.join(ROOT, "paper_2412_15803_gb300", "csrc", f), "rb").read())
     return h.hexdigest()[:16]
 
 
 def gemv_profiled_traffic(workload: str):
-    path = os.path.join(ROOT, "profiles", f"gemv_tma_kernel_{workload}.md")
+    path = os.path.join(ROOT, "profiles", f"gemv_kernels_{workload}.md")
     if not os.path.exists(path):
         return None
     text = open(path).read()
@@ -765,7 +775,7 @@ def run_gemv(args, rank, world, local):
                                       "warm_l2_median": 1e3 * statistics.median(warm),
                                       "launches": len(mats)},
             "hbm_frac_of_nominal_8tbs": achieved / NOMINAL_HBM_GBS,
-            "roofline": {"bound": "hbm", "kernel": "gemv_tma_kernel", "achieved": achieved, "peak": peak,
+            "roofline": {"bound": "hbm", "kernel": gemv_kernel_names(mats, B), "achieved": achieved, "peak": peak,
                          "peak_source": src, "unit": "GB/s", "frac": achieved / peak,
                          "traffic": traffic, "traffic_unit": "bytes per set (ncu, cold L2)",
                          "algorithmic_bytes_per_set": step_bytes, "avg_set_ms": per_set_ms},

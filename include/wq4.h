@@ -68,7 +68,9 @@ enum wq4_status {
  * memory).
  *   W_packed : uint32 [N][K/8], 16-byte aligned.
  *   scales   : fp16 bits [N][K/32], 2-byte aligned (16-byte aligned and
- *              K % 256 == 0 select the TMA-staged fast path).
+ *              K % 256 == 0 select the TMA-staged fast paths: at batch 1-2
+ *              from 32 Mi weights the legacy-tensor-path kernel, exact in
+ *              fp16 products with fp32 sums, else the CUDA-core one).
  *   x        : fp16 bits [batch][K], 16-byte aligned.
  *   y        : fp16 bits [batch][N], 2-byte aligned; must not overlap x, W or
  *              scales.
@@ -117,6 +119,16 @@ int wq4_unpack_debug(const uint32_t* W_packed, const uint16_t* scales,
  * null pointers or bad sizes (K % 8 != 0).
  */
 int wq4_pack_host(const uint8_t* q_host, uint32_t* W_host, int N, int K);
+
+/*
+ * Test hook: which kernel wq4_gemv takes at batch 1-2 with K % 256 == 0 and
+ * 16-byte aligned scales, for every later call in this process.  0 (the
+ * default) picks by size (the legacy-tensor-path kernel from 32 Mi weights
+ * up, the CUDA-core kernel below), 1 always the legacy-tensor-path kernel,
+ * 2 always the CUDA-core kernel.  Results agree within the tolerance; no
+ * counterpart in the paper.  WQ4_ERR_INVALID for another value.
+ */
+int wq4_test_gemv_path(int path);
 
 /* Static, human-readable text of a status code. */
 const char* wq4_status_string(int status);

@@ -22,7 +22,7 @@ BUILD = os.path.join(HERE, "_build")
 LIB = os.path.join(BUILD, "libwq4.so")
 
 SOURCES = ["wq4_gemv.cu", "wq4_chain.cu", "wq4_synth.cu", "wq4_tc.cu", "wq4_attn.cu", "wq4_gemm.cu"]
-HEADERS = ["wq4_device.cuh", "wq4_host.h", "wq4_tc.cuh", "wq4_tc_host.h"]
+HEADERS = ["wq4_device.cuh", "wq4_host.h", "wq4_items.cuh", "wq4_tc.cuh", "wq4_tc_host.h"]
 ARCH = ["-gencode", "arch=compute_103a,code=sm_103a"]
 
 

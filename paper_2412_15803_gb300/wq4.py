@@ -99,6 +99,7 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
     L.wq4_chain_trace_offsets.argtypes = [ctypes.POINTER(wq4_layer_table), _I,
                                           ctypes.POINTER(wq4_chain_trace)]
     L.wq4_test_chain_waits.argtypes = [_U64, _I]
+    L.wq4_test_gemv_path.argtypes = [_I]
     L.wq4_decode_step_workspace_bytes.argtypes = [ctypes.POINTER(wq4_layer_table)]
     L.wq4_decode_step_workspace_bytes.restype = _SZ
     L.wq4_decode_step.argtypes = [ctypes.POINTER(wq4_layer_table), ctypes.POINTER(wq4_decode_attn), _P, _P, _P]
@@ -119,7 +120,7 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
 EXPORTED = ["wq4_gemv", "wq4_gemm", "wq4_unpack_debug", "wq4_pack_host", "wq4_status_string",
             "wq4_device_status", "wq4_chain_workspace_bytes", "wq4_decode_chain",
             "wq4_decode_chain_host", "wq4_decode_chain_noalloc", "wq4_chain_plan_destroy", "wq4_chain_trace_offsets",
-            "wq4_test_chain_waits", "wq4_decode_step_workspace_bytes", "wq4_decode_step", "wq4_decode_step_host",
+            "wq4_test_chain_waits", "wq4_test_gemv_path", "wq4_decode_step_workspace_bytes", "wq4_decode_step", "wq4_decode_step_host",
             "wq4_synth_codes", "wq4_synth_scales", "wq4_synth_sum4",
             "wq4_paged_attention_workspace_bytes", "wq4_paged_attention", "wq4_kv_append"]
 
@@ -230,6 +231,11 @@ def wq4_decode_step_host(table: wq4_layer_table, attn: wq4_decode_attn, x_host, 
     rc = load().wq4_decode_step_host(ctypes.byref(table), ctypes.byref(attn), _ptr(x_host), _ptr(logits_host),
                                      _stream(stream))
     return _check("wq4_decode_step_host", rc) if check else rc
+
+
+def wq4_test_gemv_path(path: int) -> None:
+    """Test hook: 0 size rule, 1 legacy-tensor-path kernel, 2 CUDA-core kernel (batch 1-2)."""
+    _check("wq4_test_gemv_path", load().wq4_test_gemv_path(path))
 
 
 def wq4_test_chain_waits(wait_limit_ns: int, stall_stage: int = -1) -> None:

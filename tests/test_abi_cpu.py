@@ -216,3 +216,10 @@ def test_chain_wait_hook_rejects_bad_values():
     assert lib.wq4_test_chain_waits(500_000_001, -1) == wq4.WQ4_ERR_INVALID
     assert lib.wq4_test_chain_waits(1000, -2) == wq4.WQ4_ERR_INVALID
     assert lib.wq4_test_chain_waits(500_000_000, -1) == wq4.WQ4_OK
+
+
+def test_gemv_path_hook_rejects_bad_values():
+    lib = wq4.load()
+    assert lib.wq4_test_gemv_path(-1) == wq4.WQ4_ERR_INVALID
+    assert lib.wq4_test_gemv_path(3) == wq4.WQ4_ERR_INVALID
+    assert lib.wq4_test_gemv_path(0) == wq4.WQ4_OK

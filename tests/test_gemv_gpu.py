@@ -118,6 +118,39 @@ def test_edge_shapes_full(N, K, batch):
     check(run_gemv(W, s, x, N, K, batch), W, s, x)
 
 
+@pytest.mark.parametrize("N,K,batch", [
+    (1, 256, 1), (2, 256, 2), (3, 512, 1), (151, 256, 2), (152, 768, 1), (153, 1024, 2), (303, 2048, 1),
+    (304, 2048, 2), (305, 3072, 1), (999, 14336, 1), (2047, 8192, 2), (4097, 256, 1),
+])
+def test_mma_path_shapes_full(N, K, batch):
+    """Batch 1-2 with K % 256 == 0 on the legacy-tensor-path kernel (forced
+    by the test hook; the size rule would take it only from 32 Mi weights):
+    odd row counts (a last word of one row), fewer words than SMs, CTA
+    boundaries, one 256-code unit per row, the longest rows, every element."""
+    W, s = synth.matrix(N + 7 * K, N, K)
+    x = synth.activations(N + K + 3 * batch, batch, K)
+    try:
+        wq4.wq4_test_gemv_path(1)
+        y = run_gemv(W, s, x, N, K, batch)
+    finally:
+        wq4.wq4_test_gemv_path(0)
+    check(y, W, s, x)
+
+
+@pytest.mark.parametrize("path", [1, 2])
+def test_config1_both_batch1_kernels(path):
+    """Config 1 on each batch 1 kernel; the two agree within the tolerance."""
+    N = K = 2048
+    W, s = synth.matrix(0, N, K)
+    x = synth.activations(0, 1, K)
+    try:
+        wq4.wq4_test_gemv_path(path)
+        y = run_gemv(W, s, x, N, K, 1)
+    finally:
+        wq4.wq4_test_gemv_path(0)
+    check(y, W, s, x)
+
+
 def test_unaligned_scales_take_generic_path():
     N, K = 64, 1024
     W, s = synth.matrix(8, N, K)

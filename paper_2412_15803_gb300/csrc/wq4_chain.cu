@@ -514,6 +514,30 @@ __device__ __noinline__ void rope_table(const ChainParamsA& p, double2* rope)
     }
 }
 
+// 2^x (ex2.approx: relative error ~2^-22; 2^-inf = 0).  The attention keeps
+// its scores in the base-2 domain (scale * log2 e folded into the score
+// scale), so one instruction replaces the range reduction of expf.
+__device__ __forceinline__ float fast_exp2(float x)
+{
+    float y;
+    asm("ex2.approx.ftz.f32 %0, %1;" : "=f"(y) : "f"(x));
+    return y;
+}
+
+// acc + a.lo * b.lo + a.hi * b.hi for two fp16 pairs: products exact in fp32,
+// fp32 adds (the mixed-precision fma of sm_100+).
+__device__ __forceinline__ float fma_h2(float acc, uint32_t a, uint32_t b)
+{
+    asm("{\n\t.reg .f16 a0, a1, b0, b1;\n\t"
+        "mov.b32 {a0, a1}, %1;\n\t"
+        "mov.b32 {b0, b1}, %2;\n\t"
+        "fma.rn.f32.f16 %0, a0, b0, %0;\n\t"
+        "fma.rn.f32.f16 %0, a1, b1, %0;\n\t}"
+        : "+f"(acc)
+        : "r"(a), "r"(b));
+    return acc;
+}
+
 // Sum over the 32 lanes, every lane gets it.
 __device__ __forceinline__ float warp_allsum(float v)
 {
@@ -546,10 +570,10 @@ __device__ __forceinline__ void attention_phase(const ChainParamsA& p, int l, ui
                                              int* flag_sh, uint8_t* smem)
 {
     constexpr int kConsumers = NW * 32;
-    constexpr int U = G <= 3 ? 4 : 2;          // tokens a warp has in flight
+    constexpr int kBlk = 16;                   // tokens of a warp's block: one per lane pair
     const int warp = threadIdx.x >> 5, lane = threadIdx.x & 31;
     const int H = p.H, Hkv = p.Hkv, S = p.S, KD = Hkv * kAttnD, P = p.P;
-    const float scale = p.scale;
+    const float scale = p.scale * 1.4426950408889634f;   // base-2 scores
     // the layer's cache and the outputs in registers (the parameter block is
     // reached through a generic pointer here)
     const KvLayer kv = p.kv[l];
@@ -559,7 +583,7 @@ __device__ __forceinline__ void attention_phase(const ChainParamsA& p, int l, ui
     float* const apart = p.apart;
     uint32_t* const acnt = p.acnt;
     uint32_t* const err = p.err;
-    float* qs = scratch;
+    uint32_t* qh = reinterpret_cast<uint32_t*>(scratch);                        // [G][64] fp16 pairs of q
     float* wp = scratch + G * kAttnD;
     float* acc = reinterpret_cast<float*>(smem + kHdrRes);                       // [G][kAttnPart]
     int* pages = reinterpret_cast<int*>(smem + kHdrRes) + G * kAttnPart;          // [kAttnPageWindow]
@@ -589,10 +613,8 @@ __device__ __forceinline__ void attention_phase(const ChainParamsA& p, int l, ui
         for (int e = threadIdx.x; e < G * (kAttnD / 2) + (has_new ? kAttnD : 0); e += kConsumers) {
             if (e < G * (kAttnD / 2)) {
                 const int j = e / (kAttnD / 2), w = e - j * (kAttnD / 2);
-                const uint32_t qw = ll_load(qsrc + static_cast<size_t>(b) * (H / 2) + (h * G + j) * (kAttnD / 2) + w,
-                                            epoch, epoch, p.err, p.abort, p.wait_ns);
-                qs[j * kAttnD + 2 * w] = lo_f(qw);
-                qs[j * kAttnD + 2 * w + 1] = hi_f(qw);
+                qh[j * (kAttnD / 2) + w] = ll_load(qsrc + static_cast<size_t>(b) * (H / 2) + (h * G + j) * (kAttnD / 2) + w,
+                                                   epoch, epoch, p.err, p.abort, p.wait_ns);
             } else {
                 const int i = e - G * (kAttnD / 2);             // 0..63 key words, 64..127 value words
                 const uint64_t* src = (i < kAttnD / 2 ? p.llK : p.llVn) +
@@ -600,7 +622,6 @@ __device__ __forceinline__ void attention_phase(const ChainParamsA& p, int l, ui
                 newkv[i] = ll_load(src, epoch, epoch, p.err, p.abort, p.wait_ns);
             }
         }
-        float4 qv[G];
         float m[G], ls[G], o[G][4];
 #pragma unroll
         for (int j = 0; j < G; ++j) {
@@ -609,93 +630,115 @@ __device__ __forceinline__ void attention_phase(const ChainParamsA& p, int l, ui
             o[j][0] = o[j][1] = o[j][2] = o[j][3] = 0.f;
         }
         const int32_t* ptb = kv.pt + static_cast<size_t>(b) * kv.pt_stride;
+        const int half = lane & 1, ti = lane >> 1;
         // the range in windows of kAttnPageWindow pages
         for (int wbeg = t0; wbeg < t1; wbeg += kAttnPageWindow * P - (wbeg % P)) {
             const int wp0 = wbeg / P;
             const int wend = min(t1, (wp0 + kAttnPageWindow) * P);
             const int npg = (wend - 1) / P - wp0 + 1;
-            named_barrier_sync(1, kConsumers);                  // previous window's pages consumed; qs written
+            named_barrier_sync(1, kConsumers);                  // previous window's pages consumed; q written
             for (int i = threadIdx.x; i < npg; i += kConsumers) {
                 const int pid = __ldg(ptb + wp0 + i);
                 pages[i] = (pid >= 0 && pid < kv.num_pages) ? pid : -1;
                 if (pid < 0 || pid >= kv.num_pages) atomicOr(err, kErrPageId);
             }
             named_barrier_sync(1, kConsumers);
-            if (wbeg == t0) {
+            // blocks of 16 tokens per warp: lane pair (2 i, 2 i + 1) scores token
+            // base + i over dimensions 64 half .. 64 half + 63 (fp16 products
+            // exact in fp32, fp32 sums), then every lane accumulates the value
+            // rows' dimensions 4 lane .. 4 lane + 3 with the broadcast weights
+            for (int base = wbeg + warp * kBlk; base < wend; base += NW * kBlk) {
+                const int t = base + ti;
+                const bool valid = t < wend;
+                float sp[G][2];
 #pragma unroll
-                for (int j = 0; j < G; ++j) qv[j] = reinterpret_cast<const float4*>(qs + j * kAttnD)[lane];
-            }
-            for (int base = wbeg + warp * U; base < wend; base += NW * U) {
-                uint2 kr[U], vr[U];
+                for (int j = 0; j < G; ++j) sp[j][0] = sp[j][1] = 0.f;
+                // the key half-row in two passes of four 16-byte chunks
+                const uint4* krow = nullptr;
+                const uint4* knew4 = nullptr;
+                if (valid && t == pos) {
+                    knew4 = reinterpret_cast<const uint4*>(newkv + 32 * half);
+                } else if (valid) {
+                    const int pi = t / P;
+                    const int page = pages[pi - wp0];
+                    if (page >= 0)
+                        krow = reinterpret_cast<const uint4*>(
+                            kv.k + ((static_cast<size_t>(page) * Hkv + h) * P + (t - pi * P)) * kAttnD + 64 * half);
+                }
 #pragma unroll
-                for (int uu = 0; uu < U; ++uu) {
-                    const int t = base + uu;
-                    kr[uu] = make_uint2(0u, 0u);
-                    vr[uu] = make_uint2(0u, 0u);
-                    if (t < wend && t != pos) {
-                        const int pi = t / P;
-                        const int page = pages[pi - wp0];
-                        if (page >= 0) {
-                            const size_t row = ((static_cast<size_t>(page) * Hkv + h) * P + (t - pi * P)) * kAttnD;
-                            kr[uu] = __ldg(reinterpret_cast<const uint2*>(kv.k + row) + lane);
-                            vr[uu] = __ldg(reinterpret_cast<const uint2*>(kv.v + row) + lane);
+                for (int ps = 0; ps < 2; ++ps) {
+                    uint4 kc[4];
+#pragma unroll
+                    for (int cc = 0; cc < 4; ++cc)
+                        kc[cc] = knew4 ? knew4[4 * ps + cc] : (krow ? __ldg(krow + 4 * ps + cc) : make_uint4(0u, 0u, 0u, 0u));
+#pragma unroll
+                    for (int cc = 0; cc < 4; ++cc) {
+#pragma unroll
+                        for (int j = 0; j < G; ++j) {
+                            // a shared-memory load per use: held in registers across the
+                            // blocks, the group's queries would spill
+                            const uint4 qc = lds_v4(smem_addr(qh + j * (kAttnD / 2) + 32 * half + 4 * (4 * ps + cc)));
+                            float& a = sp[j][cc & 1];
+                            a = fma_h2(a, qc.x, kc[cc].x);
+                            a = fma_h2(a, qc.y, kc[cc].y);
+                            a = fma_h2(a, qc.z, kc[cc].z);
+                            a = fma_h2(a, qc.w, kc[cc].w);
                         }
                     }
                 }
-                if (pos >= base && pos < base + U && pos < wend) {
-                    // the new token: the words polled at the unit's start
-                    const int uu = pos - base;
-                    const uint2 nk = make_uint2(newkv[2 * lane], newkv[2 * lane + 1]);
-                    const uint2 nv = make_uint2(newkv[64 + 2 * lane], newkv[64 + 2 * lane + 1]);
-#pragma unroll
-                    for (int i = 0; i < U; ++i)
-                        if (i == uu) {
-                            kr[i] = nk;
-                            vr[i] = nv;
-                        }
-                }
-                // the batch's scores: U x G independent lane sums, reduced together
-                float sc[U][G];
-#pragma unroll
-                for (int uu = 0; uu < U; ++uu) {
-                    const float k0 = lo_f(kr[uu].x), k1 = hi_f(kr[uu].x), k2 = lo_f(kr[uu].y), k3 = hi_f(kr[uu].y);
-#pragma unroll
-                    for (int j = 0; j < G; ++j)
-                        sc[uu][j] = fmaf(qv[j].x, k0, fmaf(qv[j].y, k1, fmaf(qv[j].z, k2, qv[j].w * k3)));
-                }
-#pragma unroll
-                for (int off = 16; off > 0; off >>= 1)
-#pragma unroll
-                    for (int uu = 0; uu < U; ++uu)
-#pragma unroll
-                        for (int j = 0; j < G; ++j) sc[uu][j] += __shfl_xor_sync(0xffffffffu, sc[uu][j], off);
-                // one running-maximum update per batch (the batch's first token is valid)
+                float pw[G];
 #pragma unroll
                 for (int j = 0; j < G; ++j) {
-                    float mb = m[j];
+                    float sc = sp[j][0] + sp[j][1];
+                    sc = (sc + __shfl_xor_sync(0xffffffffu, sc, 1)) * scale;
+                    if (!valid) sc = -INFINITY;
+                    float bm = sc;                             // the block's maximum (token base is valid)
 #pragma unroll
-                    for (int uu = 0; uu < U; ++uu) {
-                        sc[uu][j] *= scale;
-                        if (base + uu < wend) mb = fmaxf(mb, sc[uu][j]);
-                    }
-                    const float corr = expf(m[j] - mb);
-                    float lsum = ls[j] * corr;
-                    float o0 = o[j][0] * corr, o1 = o[j][1] * corr, o2 = o[j][2] * corr, o3 = o[j][3] * corr;
+                    for (int off = 16; off > 1; off >>= 1) bm = fmaxf(bm, __shfl_xor_sync(0xffffffffu, bm, off));
+                    const float mn = fmaxf(m[j], bm);
+                    const float corr = fast_exp2(m[j] - mn);
+                    pw[j] = valid ? fast_exp2(sc - mn) : 0.f;
+                    float bs = half ? 0.f : pw[j];             // each token once
 #pragma unroll
-                    for (int uu = 0; uu < U; ++uu) {
-                        const float pw = (base + uu < wend) ? expf(sc[uu][j] - mb) : 0.f;
-                        lsum += pw;
-                        o0 = fmaf(pw, lo_f(vr[uu].x), o0);
-                        o1 = fmaf(pw, hi_f(vr[uu].x), o1);
-                        o2 = fmaf(pw, lo_f(vr[uu].y), o2);
-                        o3 = fmaf(pw, hi_f(vr[uu].y), o3);
+                    for (int off = 16; off > 0; off >>= 1) bs += __shfl_xor_sync(0xffffffffu, bs, off);
+                    ls[j] = fmaf(ls[j], corr, bs);
+                    o[j][0] *= corr;
+                    o[j][1] *= corr;
+                    o[j][2] *= corr;
+                    o[j][3] *= corr;
+                    m[j] = mn;
+                }
+                const int nb = min(kBlk, wend - base);
+                // every value row of the block in flight at once, then the sums
+                uint2 vv[kBlk];
+#pragma unroll
+                for (int i = 0; i < kBlk; ++i) {
+                    const int tt = base + i;
+                    vv[i] = make_uint2(0u, 0u);
+                    if (i < nb) {
+                        if (tt == pos) {
+                            vv[i] = make_uint2(newkv[64 + 2 * lane], newkv[64 + 2 * lane + 1]);
+                        } else {
+                            const int pi = tt / P;
+                            const int page = pages[pi - wp0];
+                            if (page >= 0)
+                                vv[i] = __ldg(reinterpret_cast<const uint2*>(
+                                                  kv.v + ((static_cast<size_t>(page) * Hkv + h) * P + (tt - pi * P)) * kAttnD) +
+                                              lane);
+                        }
                     }
-                    ls[j] = lsum;
-                    o[j][0] = o0;
-                    o[j][1] = o1;
-                    o[j][2] = o2;
-                    o[j][3] = o3;
-                    m[j] = mb;
+                }
+#pragma unroll
+                for (int i = 0; i < kBlk; ++i) {
+                    const float w0 = lo_f(vv[i].x), w1 = hi_f(vv[i].x), w2 = lo_f(vv[i].y), w3 = hi_f(vv[i].y);
+#pragma unroll
+                    for (int j = 0; j < G; ++j) {
+                        const float pi_ = __shfl_sync(0xffffffffu, pw[j], 2 * i);   // 0 past the window's end
+                        o[j][0] = fmaf(pi_, w0, o[j][0]);
+                        o[j][1] = fmaf(pi_, w1, o[j][1]);
+                        o[j][2] = fmaf(pi_, w2, o[j][2]);
+                        o[j][3] = fmaf(pi_, w3, o[j][3]);
+                    }
                 }
             }
         }
@@ -718,7 +761,7 @@ __device__ __forceinline__ void attention_phase(const ChainParamsA& p, int l, ui
                 if (M != -INFINITY) {
 #pragma unroll
                     for (int w = 0; w < NW; ++w) {
-                        const float f = expf(wp[w * kAttnPart + kAttnD] - M);   // 0 for a warp without tokens
+                        const float f = fast_exp2(wp[w * kAttnPart + kAttnD] - M);   // 0 for a warp without tokens
                         Ls = fmaf(f, wp[w * kAttnPart + kAttnD + 1], Ls);
                         Od = fmaf(f, wp[w * kAttnPart + d], Od);
                     }
@@ -786,7 +829,7 @@ __device__ __forceinline__ void attention_phase(const ChainParamsA& p, int l, ui
                         for (int i = 0; i < kBatch; ++i) {
                             if (c0 + i >= Sb) break;
                             const float2 mlc = ml[(c0 + i) * G + j];
-                            const float f = expf(mlc.x - M);
+                            const float f = fast_exp2(mlc.x - M);
                             Ls = fmaf(f, mlc.y, Ls);
                             O0 = fmaf(f, ov[i].x, O0);
                             O1 = fmaf(f, ov[i].y, O1);

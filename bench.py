@@ -549,7 +549,7 @@ def gemv_kernel_names(mats, B: int) -> str:
     """The kernels wq4_gemv's size rule picks for the set (batch 1-2, K % 256 == 0)."""
     names = []
     for _, N, K in mats:
-        k = "gemv_mma_kernel" if B <= 2 and K % 256 == 0 and N * K >= 32 << 20 else "gemv_tma_kernel"
+        k = "gemv_mma_kernel" if B <= 2 and K % 256 == 0 and N * K >= 12 << 20 else "gemv_tma_kernel"
         if k not in names:
             names.append(k)
     return "+".join(names)

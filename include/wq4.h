@@ -69,7 +69,7 @@ enum wq4_status {
  *   W_packed : uint32 [N][K/8], 16-byte aligned.
  *   scales   : fp16 bits [N][K/32], 2-byte aligned (16-byte aligned and
  *              K % 256 == 0 select the TMA-staged fast paths: at batch 1-2
- *              from 32 Mi weights the legacy-tensor-path kernel, exact in
+ *              from 12 Mi weights the legacy-tensor-path kernel, exact in
  *              fp16 products with fp32 sums, else the CUDA-core one).
  *   x        : fp16 bits [batch][K], 16-byte aligned.
  *   y        : fp16 bits [batch][N], 2-byte aligned; must not overlap x, W or
@@ -77,6 +77,11 @@ enum wq4_status {
  *   N >= 1, K >= 32 with K % 32 == 0, 1 <= batch <= WQ4_MAX_BATCH.
  * Returns WQ4_OK, WQ4_ERR_INVALID (sizes, null, overlap), WQ4_ERR_ALIGN, or
  * WQ4_ERR_CUDA.  Deterministic: the same inputs give the same bits.
+ * Launched with programmatic dependent launch: x is read and y written only
+ * after the previous kernel in `stream` has completed, but the weight
+ * stream may start while it finishes if that kernel lets its dependents
+ * launch early (griddepcontrol.launch_dependents), so such a kernel must not
+ * write W_packed or scales.
  */
 int wq4_gemv(const uint32_t* W_packed, const uint16_t* scales, const uint16_t* x,
              uint16_t* y, int N, int K, int batch, void* stream);
@@ -123,7 +128,7 @@ int wq4_pack_host(const uint8_t* q_host, uint32_t* W_host, int N, int K);
 /*
  * Test hook: which kernel wq4_gemv takes at batch 1-2 with K % 256 == 0 and
  * 16-byte aligned scales, for every later call in this process.  0 (the
- * default) picks by size (the legacy-tensor-path kernel from 32 Mi weights
+ * default) picks by size (the legacy-tensor-path kernel from 12 Mi weights
  * up, the CUDA-core kernel below), 1 always the legacy-tensor-path kernel,
  * 2 always the CUDA-core kernel.  Results agree within the tolerance; no
  * counterpart in the paper.  WQ4_ERR_INVALID for another value.

@@ -36,6 +36,12 @@ namespace wq4 {
 
 __device__ uint32_t g_status_word;
 
+// Programmatic dependent launch: wait for the previous grid of the stream
+// (complete, memory visible) / let the next one launch.  No effect when the
+// launch did not ask for it.
+__device__ __forceinline__ void grid_dependency_wait() { asm volatile("griddepcontrol.wait;" ::: "memory"); }
+__device__ __forceinline__ void grid_dependents_launch() { asm volatile("griddepcontrol.launch_dependents;" ::: "memory"); }
+
 constexpr int kGemvConsumerWarps = 8;
 constexpr int kGemvThreads = (kGemvConsumerWarps + 1) * 32;
 constexpr int kMaxSlots = 32;
@@ -82,6 +88,7 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_tma_kernel(const GemvTma
         mbar_fence_init();
     }
     __syncthreads();
+    grid_dependents_launch();     // the next launch in the stream may start its set-up
 
     if (warp == kGemvConsumerWarps) {
         // ---------------- producer: one elected lane issues the bulk copies
@@ -108,7 +115,10 @@ __global__ void __launch_bounds__(kGemvThreads, 1) gemv_tma_kernel(const GemvTma
         return;
     }
 
-    // ---------------- consumers: stage x (swizzled) once
+    // ---------------- consumers: stage x (swizzled) once, after the previous
+    // grid in the stream is complete (programmatic dependent launch: the
+    // producer's weight copies may start earlier)
+    grid_dependency_wait();
     {
         const uint4* xg = reinterpret_cast<const uint4*>(p.x);
         const int chunks_per_row = p.K >> 3;
@@ -204,6 +214,7 @@ __global__ void __launch_bounds__(kMmaThreads, 1) gemv_mma_kernel(const GemvMmaP
         mbar_fence_init();
     }
     __syncthreads();
+    grid_dependents_launch();     // the next launch in the stream may start its set-up
 
     if (warp == kMmaWarps) {
         // ---------------- producer: one lane issues the bulk copies
@@ -235,7 +246,9 @@ __global__ void __launch_bounds__(kMmaThreads, 1) gemv_mma_kernel(const GemvMmaP
         return;
     }
 
-    // ---------------- consumers: x once, in the MMA's pair-permuted order
+    // ---------------- consumers: x once, in the MMA's pair-permuted order,
+    // after the previous grid in the stream is complete
+    grid_dependency_wait();
     {
         const uint4* xg = reinterpret_cast<const uint4*>(p.x);
         for (int i = threadIdx.x; i < B * cpr; i += kConsumers) xs[i] = pair_permute(xg[i]);
@@ -571,12 +584,14 @@ bool plan_mma(const DeviceInfo* di, int N, int K, int B, MmaPlan* pl)
 // 1 the legacy-tensor-path kernel wherever it applies, 2 the CUDA-core one.
 std::atomic<int> g_gemv_path{0};
 
-// Below ~32 M weights a launch is bound by its fixed costs (x staging, the
+// Below ~12 M weights a launch is bound by its fixed costs (x staging, the
 // first chunk's round trip, the epilogue), which the smaller CUDA-core
-// kernel pays less of (measured: 2048 x 2048, 3.6 against 4.0 us a launch in
-// a graph); above it the legacy-tensor-path kernel streams faster (16384 x
-// 3072: 13.0 against 15.2 us, cold).
-constexpr int64_t kMmaMinWeights = int64_t(32) << 20;
+// kernel pays less of; above it the legacy-tensor-path kernel streams
+// faster.  Measured per launch in a graph of launches over rotated copies,
+// batch 1 (legacy tensor path / CUDA cores, us): 2048 x 2048 3.34 / 2.72,
+// 3072 x 3072 4.11 / 3.85, 5120 x 3072 5.02 / 5.21, 3072 x 8192 6.21 / 6.62,
+// 16384 x 3072 8.69 / 12.20, 128256 x 3072 45.1 / 75.1.
+constexpr int64_t kMmaMinWeights = int64_t(12) << 20;
 
 int launch_gemv(const uint32_t* W, const uint16_t* s, const uint16_t* x, uint16_t* y, int N, int K, int batch,
                 cudaStream_t stream)
@@ -603,9 +618,19 @@ int launch_gemv(const uint32_t* W, const uint16_t* s, const uint16_t* x, uint16_
         p.spw = mp.spw;
         p.q = mp.q;
         p.err = status_word();
-        if (batch == 1) gemv_mma_kernel<1><<<mp.grid, kMmaThreads, mp.smem, stream>>>(p);
-        else gemv_mma_kernel<2><<<mp.grid, kMmaThreads, mp.smem, stream>>>(p);
-        return cudaGetLastError() == cudaSuccess ? WQ4_OK : WQ4_ERR_CUDA;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(mp.grid);
+        cfg.blockDim = dim3(kMmaThreads);
+        cfg.dynamicSmemBytes = mp.smem;
+        cfg.stream = stream;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        const cudaError_t e = batch == 1 ? cudaLaunchKernelEx(&cfg, gemv_mma_kernel<1>, p)
+                                         : cudaLaunchKernelEx(&cfg, gemv_mma_kernel<2>, p);
+        return e == cudaSuccess ? WQ4_OK : WQ4_ERR_CUDA;
     }
     const size_t row_bytes = static_cast<size_t>(K) / 2 + static_cast<size_t>(K) / 16;
     const size_t x_bytes = align_up(static_cast<size_t>(batch) * K * 2, 128);
@@ -640,12 +665,24 @@ int launch_gemv(const uint32_t* W, const uint16_t* s, const uint16_t* x, uint16_
         p.x_bytes = static_cast<uint32_t>(x_bytes);
         p.err = status_word();
         const size_t smem = kHeaderBytes + x_bytes + static_cast<size_t>(nslots) * slot_bytes;
+        cudaLaunchAttribute attr[1];
+        attr[0].id = cudaLaunchAttributeProgrammaticStreamSerialization;
+        attr[0].val.programmaticStreamSerializationAllowed = 1;
+        cudaLaunchConfig_t cfg = {};
+        cfg.gridDim = dim3(grid);
+        cfg.blockDim = dim3(kGemvThreads);
+        cfg.dynamicSmemBytes = smem;
+        cfg.stream = stream;
+        cfg.attrs = attr;
+        cfg.numAttrs = 1;
+        cudaError_t e;
         switch (batch) {
-            case 1: gemv_tma_kernel<1><<<grid, kGemvThreads, smem, stream>>>(p); break;
-            case 2: gemv_tma_kernel<2><<<grid, kGemvThreads, smem, stream>>>(p); break;
-            case 3: gemv_tma_kernel<3><<<grid, kGemvThreads, smem, stream>>>(p); break;
-            default: gemv_tma_kernel<4><<<grid, kGemvThreads, smem, stream>>>(p); break;
+            case 1: e = cudaLaunchKernelEx(&cfg, gemv_tma_kernel<1>, p); break;
+            case 2: e = cudaLaunchKernelEx(&cfg, gemv_tma_kernel<2>, p); break;
+            case 3: e = cudaLaunchKernelEx(&cfg, gemv_tma_kernel<3>, p); break;
+            default: e = cudaLaunchKernelEx(&cfg, gemv_tma_kernel<4>, p); break;
         }
+        if (e != cudaSuccess) return WQ4_ERR_CUDA;
     } else {
         const int warps_per_block = 8;
         int grid = (N + warps_per_block - 1) / warps_per_block;

@@ -124,7 +124,7 @@ def test_edge_shapes_full(N, K, batch):
 ])
 def test_mma_path_shapes_full(N, K, batch):
     """Batch 1-2 with K % 256 == 0 on the legacy-tensor-path kernel (forced
-    by the test hook; the size rule would take it only from 32 Mi weights):
+    by the test hook; the size rule would take it only from 12 Mi weights):
     odd row counts (a last word of one row), fewer words than SMs, CTA
     boundaries, one 256-code unit per row, the longest rows, every element."""
     W, s = synth.matrix(N + 7 * K, N, K)

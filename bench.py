@@ -44,7 +44,6 @@ sys.path.insert(0, ROOT)
 
 METRIC = "GEMV-bound decode tokens/s (batch 1) and achieved HBM GB/s vs ~8 TB/s peak"
 NOMINAL_HBM_GBS = 8000.0
-PERSISTENT_MAX_BATCH = 2      # larger batches run the tensor-core graph path
 # the paper's batch-1 decode rates for these model shapes (Table 1, WebLLM in
 # Chrome on an Apple M3 Max, 4-bit weights): another machine's numbers, context only
 PAPER_DECODE_TOKS = {"8b": 41.1, "phi3.5": 71.1}
@@ -104,10 +103,9 @@ def chain_source_sha(kernel: str) -> str:
     return h.hexdigest()[:16]
 
 
-def profiled_traffic(workload: str, batch: int, context: int = 0):
-    """DRAM bytes per launch from the committed ncu summary, if it was taken
-    on the current kernel source (else None)."""
-    name = "chain_kernel" if batch <= PERSISTENT_MAX_BATCH else "tc_stage_kernel"
+def profiled_traffic(name: str, workload: str, batch: int, context: int = 0):
+    """DRAM bytes per launch of kernel `name` from the committed ncu summary,
+    if it was taken on the current kernel source (else None)."""
     ctx = f"_ctx{context}" if context else ""
     path = os.path.join(ROOT, "profiles", f"{name}_{workload}_b{batch}{ctx}.md")
     if not os.path.exists(path):
@@ -441,6 +439,9 @@ def run_ours(args, rank, world, local):
     torch.cuda.synchronize()
     if wq4.wq4_device_status(stream) != 0:
         raise RuntimeError("device wait timed out during warm-up")
+    # the library's choice for this table: the persistent chain kernel, or the
+    # stage graph (batches above its limit, or a ring that does not fit)
+    persistent = wq4.wq4_chain_path(model.table, decode_step=T > 0) == 1
 
     starts = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
     ends = [torch.cuda.Event(enable_timing=True) for _ in range(args.steps)]
@@ -475,7 +476,7 @@ def run_ours(args, rank, world, local):
     e2e_s = time.perf_counter() - t0
     tokens_per_s, e2e_val, total_ms_max = aggregate_replicas(total_ms, e2e_s / e2e_steps, B, args.steps, "cuda")
 
-    if B <= PERSISTENT_MAX_BATCH:
+    if persistent:
         # one cooperative launch of the persistent chain kernel per token
         kernel_name, launches_per_step = "chain_kernel", 1
     else:
@@ -504,7 +505,7 @@ def run_ours(args, rank, world, local):
             "roofline": {"bound": "hbm", "kernel": kernel_name, "achieved": achieved, "peak": peak,
                          "peak_source": peak_src, "unit": "GB/s", "frac": achieved / peak,
                          "frac_of_nominal_8tbs": achieved / NOMINAL_HBM_GBS,
-                         "traffic": profiled_traffic(args.workload, B, T),
+                         "traffic": profiled_traffic(kernel_name, args.workload, B, T),
                          "algorithmic_bytes_per_launch": step_bytes,
                          "avg_launch_ms": avg_launch_ms},
             "e2e": {"value": e2e_val, "unit": "tokens/s", "h2d_bytes_per_step": 2 * B * shape.hidden,

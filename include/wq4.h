@@ -284,6 +284,16 @@ int wq4_decode_chain_host(const wq4_layer_table* table, const uint16_t* x_host,
 int wq4_decode_chain_noalloc(const wq4_layer_table* table, const uint16_t* x,
                              uint16_t* logits, void* stream);
 
+/*
+ * Which kernel the cached plan of `table` runs (an inspection call, no
+ * counterpart in the paper): 1 for the persistent chain kernel (batch 1-2),
+ * 2 for the CUDA graph of tensor-core stage kernels (batch 3-32);
+ * decode_step != 0 asks about the plan of wq4_decode_step, else of
+ * wq4_decode_chain.  Returns WQ4_ERR_INVALID when no plan exists yet (the
+ * first call builds it).
+ */
+int wq4_chain_path(const wq4_layer_table* table, int decode_step);
+
 /* Releases the cached plan of `table` (host-side state only; the workspace
  * stays the caller's).  A batch 3-32 plan owns a CUDA graph: synchronize every
  * stream that ran the table before calling this.  Plans are cached by the

@@ -2183,6 +2183,14 @@ extern "C" int wq4_chain_plan_destroy(const wq4_layer_table* table)
     return found ? WQ4_OK : WQ4_ERR_INVALID;
 }
 
+extern "C" int wq4_chain_path(const wq4_layer_table* table, int decode_step)
+{
+    std::lock_guard<std::mutex> lock(g_plan_mu);
+    auto it = g_plans.find(std::make_pair(table, decode_step != 0));
+    if (it == g_plans.end()) return WQ4_ERR_INVALID;
+    return it->second.graph ? 2 : 1;
+}
+
 extern "C" size_t wq4_decode_step_workspace_bytes(const wq4_layer_table* table)
 {
     Dims d;

@@ -96,6 +96,7 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
     L.wq4_decode_chain_host.argtypes = [ctypes.POINTER(wq4_layer_table), _P, _P, _P]
     L.wq4_decode_chain_noalloc.argtypes = [ctypes.POINTER(wq4_layer_table), _P, _P, _P]
     L.wq4_chain_plan_destroy.argtypes = [ctypes.POINTER(wq4_layer_table)]
+    L.wq4_chain_path.argtypes = [ctypes.POINTER(wq4_layer_table), _I]
     L.wq4_chain_trace_offsets.argtypes = [ctypes.POINTER(wq4_layer_table), _I,
                                           ctypes.POINTER(wq4_chain_trace)]
     L.wq4_test_chain_waits.argtypes = [_U64, _I]
@@ -119,7 +120,8 @@ def load(build_if_missing: bool = True) -> ctypes.CDLL:
 # names every C entry point of include/*.h (checked by the tests)
 EXPORTED = ["wq4_gemv", "wq4_gemm", "wq4_unpack_debug", "wq4_pack_host", "wq4_status_string",
             "wq4_device_status", "wq4_chain_workspace_bytes", "wq4_decode_chain",
-            "wq4_decode_chain_host", "wq4_decode_chain_noalloc", "wq4_chain_plan_destroy", "wq4_chain_trace_offsets",
+            "wq4_decode_chain_host", "wq4_decode_chain_noalloc", "wq4_chain_plan_destroy", "wq4_chain_path",
+            "wq4_chain_trace_offsets",
             "wq4_test_chain_waits", "wq4_test_gemv_path", "wq4_decode_step_workspace_bytes", "wq4_decode_step", "wq4_decode_step_host",
             "wq4_synth_codes", "wq4_synth_scales", "wq4_synth_sum4",
             "wq4_paged_attention_workspace_bytes", "wq4_paged_attention", "wq4_kv_append"]
@@ -209,6 +211,15 @@ def wq4_decode_chain_noalloc(table: wq4_layer_table, x, logits, stream=None, che
 
 def wq4_chain_plan_destroy(table: wq4_layer_table) -> int:
     return load().wq4_chain_plan_destroy(ctypes.byref(table))
+
+
+def wq4_chain_path(table: wq4_layer_table, decode_step: bool = False) -> int:
+    """1: the table's cached plan runs the persistent chain kernel; 2: the
+    tensor-core stage graph.  Raises if no plan exists yet."""
+    rc = load().wq4_chain_path(ctypes.byref(table), 1 if decode_step else 0)
+    if rc < 0:
+        raise Wq4Error("wq4_chain_path", rc)
+    return rc
 
 
 def wq4_chain_trace_offsets(table: wq4_layer_table, layer: int) -> wq4_chain_trace:

@@ -145,6 +145,7 @@ def test_chain_rejects_null_and_misaligned_io():
     assert L.wq4_decode_chain(ctypes.byref(t), None, A16, None) == wq4.WQ4_ERR_INVALID
     assert L.wq4_decode_chain(ctypes.byref(t), A16 + 8, 2 * A16, None) == wq4.WQ4_ERR_ALIGN
     assert L.wq4_chain_plan_destroy(ctypes.byref(t)) == wq4.WQ4_ERR_INVALID
+    assert L.wq4_chain_path(ctypes.byref(t), 0) == wq4.WQ4_ERR_INVALID      # no plan was built
 
 
 def test_synth_rejects_bad_arguments():

@@ -12,7 +12,7 @@ import torch
 
 import oracle
 from oracle import chain as ochain
-from paper_2412_15803_gb300 import synth
+from paper_2412_15803_gb300 import synth, wq4
 from paper_2412_15803_gb300.model import SHAPE_3B, SHAPE_8B, SHAPE_PHI, DecodeModel, ModelShape
 
 pytestmark = pytest.mark.gpu
@@ -109,6 +109,7 @@ def test_tiny_chain_every_stage_every_element(batch):
     model = DecodeModel(TINY, batch=batch, seed=batch)
     x = synth.activations(100 + batch, batch, TINY.hidden)
     logits = run(model, x)
+    assert wq4.wq4_chain_path(model.table) == (1 if batch <= 2 else 2)
     for l in range(TINY.num_layers):
         check_stages(model, l, u=x if l == 0 else None)
     check_logits(model, logits)
@@ -121,7 +122,8 @@ def test_tiny_chain_every_stage_every_element(batch):
     assert rel < 2e-2, rel
 
 
-@pytest.mark.parametrize("shape,batch", [(TINY, 1), (TINY, 2), (TINY, 3), (TINY, 8), (TINY, 32), (SMALL, 1), (SMALL, 4)])
+@pytest.mark.parametrize("shape,batch", [(TINY, 1), (TINY, 2), (TINY, 3), (TINY, 8), (TINY, 32), (SMALL, 1), (SMALL, 4),
+                                         (SMALL, 6)])
 def test_chain_full_range_codes_every_element(shape, batch):
     """Codes uniform on 0..15 (every code value, code 15 = weight 8 s, on
     every path: the persistent kernel's exact tensor-path dequantization at
@@ -189,6 +191,7 @@ def test_3b_chain_full_size_sampled():
     model = DecodeModel(SHAPE_3B, batch=1, seed=0)
     x = synth.activations(0, 1, SHAPE_3B.hidden)
     logits = run(model, x)
+    assert wq4.wq4_chain_path(model.table) == 1
     rng = np.random.default_rng(0)
     sh = SHAPE_3B
 
@@ -215,6 +218,7 @@ def test_8b_chain_full_size_sampled(batch):
     model = DecodeModel(sh, batch=batch, seed=3)
     x = synth.activations(5, batch, sh.hidden)
     logits = run(model, x)
+    assert wq4.wq4_chain_path(model.table) == (1 if batch <= 2 else 2)
     rng = np.random.default_rng(1)
 
     def pick(N):
@@ -281,7 +285,7 @@ def test_small_chain_graph_path_repeat_and_rebuild(batch):
     assert np.array_equal(run(model, x), a)          # a new plan and graph give the same bits
 
 
-@pytest.mark.parametrize("batch", [1, 2, 3])
+@pytest.mark.parametrize("batch", [1, 2, 3, 5])
 def test_cached_plan_on_a_zeroed_workspace(batch):
     """A table whose workspace was freed and came back zero-filled at the same
     address (same table contents, so the cached plan is reused without

@@ -101,7 +101,7 @@ def check_logits(model, logits, rows=None):
     within(logits[:, idx], y, A, "lm_head")
 
 
-@pytest.mark.parametrize("batch", [1, 2, 3, 4, 5, 8, 13, 17, 32])
+@pytest.mark.parametrize("batch", [1, 2, 3, 4, 5, 6, 7, 8, 9, 13, 17, 32])
 def test_tiny_chain_every_stage_every_element(batch):
     """Batch 1-2: the persistent kernel; 3-32: the graph of tensor-core stage
     kernels (batch padded to 16 up to 16, else to 32; 13 and 17 leave a
@@ -122,8 +122,8 @@ def test_tiny_chain_every_stage_every_element(batch):
     assert rel < 2e-2, rel
 
 
-@pytest.mark.parametrize("shape,batch", [(TINY, 1), (TINY, 2), (TINY, 3), (TINY, 8), (TINY, 32), (SMALL, 1), (SMALL, 4),
-                                         (SMALL, 6)])
+@pytest.mark.parametrize("shape,batch", [(TINY, 1), (TINY, 2), (TINY, 3), (TINY, 8), (TINY, 12), (TINY, 32), (SMALL, 1),
+                                         (SMALL, 4), (SMALL, 6), (SMALL, 8), (SMALL, 10)])
 def test_chain_full_range_codes_every_element(shape, batch):
     """Codes uniform on 0..15 (every code value, code 15 = weight 8 s, on
     every path: the persistent kernel's exact tensor-path dequantization at
@@ -185,13 +185,15 @@ def test_plan_rebuilds_when_table_changes():
     model.destroy_plan()
 
 
-def test_3b_chain_full_size_sampled():
-    """The 28-layer 3B-shaped chain at batch 1, as the benchmark runs it:
+@pytest.mark.parametrize("batch", [1, 3, 8])
+def test_3b_chain_full_size_sampled(batch):
+    """The 28-layer 3B-shaped chain at batch 1 (the persistent kernel, as the
+    benchmark runs it) and at batch 3 and 8 (the tensor-core stage graph):
     sampled rows of every projection of three layers, and of the LM head."""
-    model = DecodeModel(SHAPE_3B, batch=1, seed=0)
-    x = synth.activations(0, 1, SHAPE_3B.hidden)
+    model = DecodeModel(SHAPE_3B, batch=batch, seed=0)
+    x = synth.activations(0, batch, SHAPE_3B.hidden)
     logits = run(model, x)
-    assert wq4.wq4_chain_path(model.table) == 1
+    assert wq4.wq4_chain_path(model.table) == (1 if batch == 1 else 2)
     rng = np.random.default_rng(0)
     sh = SHAPE_3B
 
@@ -207,13 +209,14 @@ def test_3b_chain_full_size_sampled():
     assert np.array_equal(run(model, x), logits)
 
 
-@pytest.mark.parametrize("batch", [1, 2, 4, 8, 16, 32])
+@pytest.mark.parametrize("batch", [1, 2, 4, 5, 8, 16, 32])
 def test_8b_chain_full_size_sampled(batch):
     """The 32-layer 8B-shaped chain over the batch sweep: batch 1-2 on the
     persistent kernel (the longest rows, K = 14336 in the down projection,
-    one row pair per item), 4-32 on the tensor-core stage graph (batch 17-32:
-    32-column tiles and 8-part K splits at K = 14336).  Sampled rows of three
-    layers and of the LM head, and twenty tokens with identical bits."""
+    one row pair per item), 4-32 on the tensor-core stage graph (batch 5: a
+    partly padded group of four batch rows; batch 17-32: 32-column tiles and
+    8-part K splits at K = 14336).  Sampled rows of three layers and of the
+    LM head, and twenty tokens with identical bits."""
     sh = SHAPE_8B
     model = DecodeModel(sh, batch=batch, seed=3)
     x = synth.activations(5, batch, sh.hidden)
@@ -269,12 +272,14 @@ def test_two_models_with_different_rings_alternate():
     check_logits(a, la)
 
 
-@pytest.mark.parametrize("batch", [6, 16])
-def test_small_chain_graph_path_repeat_and_rebuild(batch):
+@pytest.mark.parametrize("batch", [6, 12, 16])
+def test_small_chain_repeat_and_rebuild(batch):
+    """The stage graph: repeated tokens, the host-buffer call and a rebuilt
+    plan (a new graph) give the same bits."""
     model = DecodeModel(SMALL, batch=batch, seed=60 + batch)
     x = synth.activations(61, batch, SMALL.hidden)
     a = run(model, x)
-    assert np.array_equal(run(model, x), a)          # graph replays are deterministic
+    assert np.array_equal(run(model, x), a)          # repeated tokens are deterministic
     for l in range(SMALL.num_layers):
         check_stages(model, l, u=x if l == 0 else None)
     check_logits(model, a)
@@ -282,10 +287,10 @@ def test_small_chain_graph_path_repeat_and_rebuild(batch):
     model.decode_host(np.ascontiguousarray(x), lh)
     assert np.array_equal(lh, a)
     model.destroy_plan()
-    assert np.array_equal(run(model, x), a)          # a new plan and graph give the same bits
+    assert np.array_equal(run(model, x), a)          # a new plan gives the same bits
 
 
-@pytest.mark.parametrize("batch", [1, 2, 3, 5])
+@pytest.mark.parametrize("batch", [1, 2, 3, 5, 12])
 def test_cached_plan_on_a_zeroed_workspace(batch):
     """A table whose workspace was freed and came back zero-filled at the same
     address (same table contents, so the cached plan is reused without

@@ -109,7 +109,7 @@ def patch_lm_head(model, scales, seed):
     return W, s
 
 
-@pytest.mark.parametrize("batch", [1, 2, 3, 4, 8])
+@pytest.mark.parametrize("batch", [1, 2, 3, 4, 8, 12])
 def test_chain_lm_head_extreme_scales(batch):
     """The LM head with scales from the smallest subnormal to 128 and codes
     uniform on 0..15, on the persistent kernel (batch 1-2) and the stage
@@ -128,11 +128,11 @@ def test_chain_lm_head_extreme_scales(batch):
 
 @pytest.mark.parametrize("bad", [0x7000, 0xFBFF])
 def test_chain_batched_refuses_scale_beyond_fp16_range(bad):
-    model = DecodeModel(TINY, batch=5, seed=70)
+    model = DecodeModel(TINY, batch=12, seed=70)
     model.weights[1]["down"][1].view(-1)[5] = int(np.int16(np.uint16(bad).view(np.int16)))
     torch.cuda.synchronize()
-    x = torch.from_numpy(synth.activations(71, 5, TINY.hidden).view(np.int16)).cuda()
-    logits = torch.empty((5, TINY.vocab), dtype=torch.int16, device="cuda")
+    x = torch.from_numpy(synth.activations(71, 12, TINY.hidden).view(np.int16)).cuda()
+    logits = torch.empty((12, TINY.vocab), dtype=torch.int16, device="cuda")
     with pytest.raises(wq4.Wq4Error) as e:
         model.decode(x, logits)
     assert e.value.status == -3   # WQ4_ERR_UNSUPPORTED

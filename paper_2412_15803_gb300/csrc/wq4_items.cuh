@@ -84,7 +84,7 @@ __device__ __forceinline__ void item_units(const uint32_t (&ca)[NP], const uint3
     }
     const uint32_t xbase = xs + 16 * lane;
     const float zero[4] = {0.f, 0.f, 0.f, 0.f};
-#pragma unroll(NP == 1 ? 2 : 1)
+#pragma unroll(B == 1 || NP == 1 ? 2 : 1)   // two group sets an iteration at batch 1 (measured ~1 % faster), not at 2
     for (int j = j0; j < j1; ++j) {
         uint4 xv[B];
 #pragma unroll

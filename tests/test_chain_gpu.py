@@ -6,6 +6,9 @@ residual adds must be bit-exact; silu(gate) * up within one fp16 ulp of the
 fp64 value; the LM head like a projection.  End-to-end logits of the small
 model are compared with the oracle chain by relative L2 (information only).
 """
+import os
+from concurrent.futures import ThreadPoolExecutor
+
 import numpy as np
 import pytest
 import torch
@@ -47,12 +50,14 @@ def check_norm(v_gpu, u, eps, what):
     assert np.all(err <= oracle.ulp16_array(np.abs(ref))), what
 
 
-def check_stages(model, layer, rows=None, u=None):
+def check_stages(model, layer, rows=None, u=None, t=None):
     """Stage-wise parity of one layer; rows: None = all, else a dict name -> row
-    index array; u: the layer's raw input (None: the previous layer's output)."""
+    index array; u: the layer's raw input (None: the previous layer's output);
+    t: the layer's trace, if already read back."""
     sh, eps = model.shape, model.eps
     H, F = sh.hidden, sh.ffn
-    t = model.trace(layer)
+    if t is None:
+        t = model.trace(layer)
     if u is None:
         u = model.trace(layer - 1)["x_out"]
     check_norm(t["x_in"], u, eps, f"layer {layer} input normalisation")
@@ -207,6 +212,43 @@ def test_3b_chain_full_size_sampled(batch):
     # the whole output is finite and the chain is deterministic
     assert np.all(np.isfinite(oracle.half_to_double(logits)))
     assert np.array_equal(run(model, x), logits)
+
+
+@pytest.mark.parametrize("shape,batch", [(SHAPE_3B, 1), (SHAPE_3B, 8), (SHAPE_8B, 1)], ids=["3b-b1", "3b-b8", "8b-b1"])
+def test_full_size_every_layer_every_element(shape, batch):
+    """Full-size chains checked whole: the 28-layer 3B shape at batch 1 (the
+    benchmarked configuration, persistent kernel) and 8 (tensor-core stage
+    graph), the 32-layer 8B shape at batch 1: every output element of every
+    projection of every layer (stage by stage, each on the GPU's own input to
+    that stage; residual adds bit-exact) and every logit, against the oracle.
+    The host side (weights regenerated from the seeded generator, the fp64
+    GEMVs) runs on a thread pool: numpy and the oracle's C calls release the
+    interpreter lock."""
+    sh = shape
+    model = DecodeModel(sh, batch=batch, seed=11 + batch)
+    x = synth.activations(13 + batch, batch, sh.hidden)
+    logits = run(model, x)
+    assert wq4.wq4_chain_path(model.table) == (1 if batch <= 2 else 2)
+    traces = [model.trace(l) for l in range(sh.num_layers + 1)]   # every device read before the threads
+    xL = traces[sh.num_layers - 1]["x_out"]
+    check_norm(traces[sh.num_layers]["x_in"], xL, model.eps, "LM head input normalisation")
+    r = ochain.rms_factors(xL, model.eps)
+    oracle.lib()
+
+    def layer(l):
+        check_stages(model, l, u=x if l == 0 else traces[l - 1]["x_out"], t=traces[l])
+
+    def lm_block(r0):
+        n = min(8192, sh.vocab - r0)
+        W, s = model.host_rows(sh.num_layers, "lm_head", r0, n)
+        y, A, _ = oracle.gemv(W, s, xL, r)
+        within(logits[:, r0:r0 + n], y, A, f"lm_head rows {r0}..{r0 + n - 1}")
+
+    with ThreadPoolExecutor(max_workers=max(1, min(16, os.cpu_count() or 1))) as ex:
+        jobs = [ex.submit(layer, l) for l in range(sh.num_layers)]
+        jobs += [ex.submit(lm_block, r0) for r0 in range(0, sh.vocab, 8192)]
+        for j in jobs:
+            j.result()
 
 
 @pytest.mark.parametrize("batch", [1, 2, 4, 5, 8, 16, 32])

@@ -15,6 +15,9 @@ stage (read back from the workspace traces and the caches):
 Batch 1-2 runs the attention inside the persistent kernel; 3-32 the graph
 path (rotation/append kernel, wq4_paged_attention, the stage kernels).
 """
+import os
+from concurrent.futures import ThreadPoolExecutor
+
 import numpy as np
 import pytest
 import torch
@@ -56,13 +59,15 @@ def _rows(model, layer, name, idx):
     return np.concatenate(Ws), np.concatenate(ss)
 
 
-def check_step_layer(model, caches, layer, before, rows=None, u=None):
+def check_step_layer(model, caches, layer, before, rows=None, u=None, t=None, after=None):
     """Every stage of one layer of a step.  before: (k, v) host copies of the
-    layer's cache pools taken before the step."""
+    layer's cache pools taken before the step; t, after: the layer's trace and
+    its (k, v) pools after the step, if already read back."""
     sh, eps = model.shape, model.eps
     H, F, D, Hkv = sh.hidden, sh.ffn, sh.head_dim, sh.n_kv_heads
     KD = Hkv * D
-    t = model.trace(layer)
+    if t is None:
+        t = model.trace(layer)
     if u is None:
         u = model.trace(layer - 1)["x_out"]
     r = ochain.rms_factors(u, eps)
@@ -84,7 +89,7 @@ def check_step_layer(model, caches, layer, before, rows=None, u=None):
         err = np.abs(oracle.half_to_double(t[name]) - r64)
         assert np.all(err <= oracle.ulp16_array(np.abs(r64))), f"layer {layer} {name}"
     # the append: new rows bit-exact, the rest untouched
-    k_after, v_after = caches.host_cache(layer)
+    k_after, v_after = caches.host_cache(layer) if after is None else after
     k_exp, v_exp = before[0].copy(), before[1].copy()
     P = caches.page_size
     for b in range(model.batch):
@@ -218,6 +223,43 @@ def test_3b_step_full_size_sampled(batch):
                                               layers=(0, 13, 27))
     check_logits(model, logits, rows=pick(sh.vocab))
     assert np.all(np.isfinite(oracle.half_to_double(logits)))
+
+
+def test_3b_step_batch1_every_layer_every_element():
+    """The decode step of the 3B shape at batch 1 with 4096 tokens in context
+    (the token at position 4095) checked whole: every stage of every one of
+    the 28 layers -- all projection outputs, the rotated q and k, the cache
+    append, the whole attention output -- and every logit.  The host side
+    runs on a thread pool after every device read."""
+    sh = SHAPE_3B
+    model = DecodeModel(sh, batch=1, seed=91, step=True)
+    caches = StepCaches(sh, [4095], page_size=16, seed=92, spare_pages=3, rope_theta=500000.0)
+    L = sh.num_layers
+    before = [caches.host_cache(l) for l in range(L)]
+    x = synth.activations(93, 1, sh.hidden)
+    logits = run_step(model, caches, x)
+    assert wq4.wq4_chain_path(model.table, decode_step=True) == 1
+    traces = [model.trace(l) for l in range(L + 1)]
+    after = [caches.host_cache(l) for l in range(L)]
+    xL = traces[L - 1]["x_out"]
+    r = ochain.rms_factors(xL, model.eps)
+    oracle.lib()
+
+    def layer(l):
+        check_step_layer(model, caches, l, before[l], u=x if l == 0 else traces[l - 1]["x_out"], t=traces[l],
+                         after=after[l])
+
+    def lm_block(r0):
+        n = min(8192, sh.vocab - r0)
+        W, s = model.host_rows(L, "lm_head", r0, n)
+        y, A, _ = oracle.gemv(W, s, xL, r)
+        within(logits[:, r0:r0 + n], y, A, f"lm_head rows {r0}..{r0 + n - 1}")
+
+    with ThreadPoolExecutor(max_workers=max(1, min(16, os.cpu_count() or 1))) as ex:
+        jobs = [ex.submit(layer, l) for l in range(L)]
+        jobs += [ex.submit(lm_block, r0) for r0 in range(0, sh.vocab, 8192)]
+        for j in jobs:
+            j.result()
 
 
 def test_8b_step_full_size_sampled():
